@@ -1,0 +1,386 @@
+"""Pins for the fp64 oracle: closed forms, invariants, special cases and the
+paper's printed numbers.  None of these re-types an oracle formula; each is
+chosen so that a plausible slip (a dropped term, a wrong sign or index, a
+transposed operand) fails at least one of them."""
+import json
+import math
+import os
+
+import numpy as np
+import pytest
+import torch
+
+import oracle as O
+
+GOLDEN = os.path.join(os.path.dirname(__file__), "golden")
+rng = np.random.default_rng(1234)
+
+
+# --------------------------------------------------------------------------
+# storage rounding
+# --------------------------------------------------------------------------
+
+def test_bf16_round_matches_torch_conversion():
+    # torch's float32 -> bfloat16 cast is an independent round-to-nearest-even.
+    x32 = torch.randn(200000, dtype=torch.float32) * 10
+    # add exact ties: values halfway between two bf16 neighbours
+    base = torch.randn(1000, dtype=torch.float32).to(torch.bfloat16).float()
+    ulp = torch.ldexp(torch.ones_like(base), torch.frexp(base).exponent - 8)
+    ties = base + ulp / 2
+    x32 = torch.cat([x32, ties])
+    ref = x32.to(torch.bfloat16).double().numpy()
+    got = O.bf16_round(x32.double().numpy())
+    assert np.array_equal(ref, got)
+
+
+def test_store_f32_is_float32_rounding():
+    x = rng.standard_normal(1000)
+    assert np.array_equal(O.store(x, "f32"), x.astype(np.float32).astype(np.float64))
+
+
+# --------------------------------------------------------------------------
+# Eq. 1 reducer
+# --------------------------------------------------------------------------
+
+def _H(N, m, d):
+    return rng.standard_normal((N, m, d))
+
+
+def test_reduce_m1_identity_under_unit_gate():
+    H = O.bf16_round(_H(5, 1, 16))
+    y, _ = O.gated_reduce(H, np.zeros((1, 16)), np.zeros(1),
+                          alpha_override=np.ones((5, 1)), out_dtype="bf16")
+    assert np.array_equal(y, H[:, 0, :])
+
+
+def test_reduce_one_hot_selects_path():
+    H = O.bf16_round(_H(6, 4, 32))
+    for j in range(4):
+        a = np.zeros((6, 4))
+        a[:, j] = 1.0
+        y, _ = O.gated_reduce(H, np.zeros((4, 128)), np.zeros(4),
+                              alpha_override=a, out_dtype="bf16")
+        assert np.array_equal(y, H[:, j, :])
+
+
+def test_reduce_equal_weights_is_path_mean():
+    H = _H(7, 4, 24)
+    y, _ = O.gated_reduce(H, np.zeros((4, 96)), np.zeros(4),
+                          alpha_override=np.full((7, 4), 0.25), out_dtype="f64")
+    np.testing.assert_allclose(y, H.mean(axis=1), rtol=1e-15, atol=1e-15)
+
+
+def test_reduce_zero_gate_weight_gives_sigmoid_of_bias():
+    # sigmoid(0) = 1/2, sigmoid(ln 3) = 3/4, sigmoid(-ln 3) = 1/4, sigmoid(ln 9) = 9/10
+    b = np.array([0.0, math.log(3.0), -math.log(3.0), math.log(9.0)])
+    H = _H(3, 4, 8)
+    y, a = O.gated_reduce(H, np.zeros((4, 32)), b, out_dtype="f64")
+    expect_a = np.array([0.5, 0.75, 0.25, 0.9])
+    np.testing.assert_allclose(a, np.broadcast_to(expect_a, (3, 4)), rtol=1e-14)
+    np.testing.assert_allclose(
+        y, 0.5 * H[:, 0] + 0.75 * H[:, 1] + 0.25 * H[:, 2] + 0.9 * H[:, 3], rtol=1e-13)
+
+
+def test_reduce_gate_reads_path_major_vec_with_sign_and_scale():
+    # H = +1 everywhere except one entry -1 => mean(H^2) = 1, r = 1 (eps 0).
+    # W_f picks that single entry for gate 2 with weight 1: logit_2 = s*(-1) + b_2.
+    m, d = 4, 8
+    p, e = 2, 5
+    H = np.ones((1, m, d))
+    H[0, p, e] = -1.0
+    Wf = np.zeros((m, m * d))
+    Wf[2, p * d + e] = 1.0
+    b = np.array([0.0, 0.0, 0.25, 0.0])
+    s = 1.7
+    g = O.gate_logits(H, Wf, b, rms_eps=0.0, gate_scale=s)
+    np.testing.assert_allclose(g[0], [0.0, 0.0, -s + 0.25, 0.0], rtol=0, atol=1e-15)
+    # the transposed (element-major) vec would have read a +1 entry
+    assert g[0, 2] < 0
+
+
+def test_reduce_rms_uses_all_md_entries_and_eps():
+    # H = c everywhere -> x~ = c / sqrt(c^2 + eps); W_f = 1/(md) sums x~ once.
+    m, d, c, eps = 2, 4, 3.0, 7.0
+    H = np.full((1, m, d), c)
+    Wf = np.full((m, m * d), 1.0 / (m * d))
+    g = O.gate_logits(H, Wf, np.zeros(m), rms_eps=eps)
+    np.testing.assert_allclose(g[0], c / math.sqrt(c * c + eps), rtol=1e-15)  # 3/4
+
+
+def test_reduce_scale_invariance():
+    H = _H(4, 4, 16)
+    Wf = rng.standard_normal((4, 64)) * 0.1
+    b = rng.standard_normal(4)
+    y1, a1 = O.gated_reduce(H, Wf, b, rms_eps=0.0, out_dtype="f64")
+    y2, a2 = O.gated_reduce(3.5 * H, Wf, b, rms_eps=0.0, out_dtype="f64")
+    np.testing.assert_allclose(a1, a2, rtol=1e-13)
+    np.testing.assert_allclose(y2, 3.5 * y1, rtol=1e-12)
+
+
+def test_reduce_gates_are_not_a_softmax():
+    H = _H(16, 4, 32)
+    _, a = O.gated_reduce(H, rng.standard_normal((4, 128)) * 0.1, np.zeros(4), out_dtype="f64")
+    assert np.all((a > 0) & (a < 1))
+    assert np.max(np.abs(a.sum(axis=1) - 1.0)) > 1e-3
+
+
+def test_reduce_offset_and_scale_terms():
+    H = _H(3, 4, 8)
+    Wf = rng.standard_normal((4, 32))
+    b = rng.standard_normal(4)
+    _, a0 = O.gated_reduce(H, Wf, b, out_dtype="f64")
+    _, a1 = O.gated_reduce(H, Wf, b, gate_offset=0.125, out_dtype="f64")
+    np.testing.assert_allclose(a1 - a0, 0.125, rtol=0, atol=1e-15)
+    _, az = O.gated_reduce(H, Wf, b, gate_scale=0.0, out_dtype="f64")
+    np.testing.assert_allclose(az, np.broadcast_to(1 / (1 + np.exp(-b)), az.shape), rtol=1e-14)
+
+
+def test_reduce_path_norm_constant_magnitude_paths():
+    # path j = +-c_j -> RMSNorm_gamma(H_j) = sign * gamma_j (eps 0)
+    m, d = 3, 6
+    c = np.array([0.5, 2.0, 7.0])
+    sign = np.where(rng.standard_normal((1, m, d)) > 0, 1.0, -1.0)
+    H = sign * c[None, :, None]
+    gamma = rng.standard_normal((m, d))
+    a = np.array([[0.2, 0.3, 0.9]])
+    y, _ = O.gated_reduce(H, np.zeros((m, m * d)), np.zeros(m), alpha_override=a,
+                          path_norm_w=gamma, path_norm_eps=0.0, out_dtype="f64")
+    expect = (a[0, :, None] * sign[0] * gamma).sum(axis=0)
+    np.testing.assert_allclose(y[0], expect, rtol=1e-14)
+
+
+def test_table1_parameter_counts():
+    g = json.load(open(os.path.join(GOLDEN, "table1_reducer_params.json")))
+    m, d = g["m"], g["d"]
+    hc = O.hc_gate_param_count(m, d)
+    fc = O.fc_param_count(m, d)
+    assert hc == 65536
+    assert hc // 1000 == g["hc_gate_thousands_printed"]   # printed "65K"
+    assert fc // 10**6 == g["fc_millions_printed"]         # printed "67M"
+    assert fc // hc == d // m == 1024       # "three orders of magnitude fewer"
+
+
+# --------------------------------------------------------------------------
+# drafter pieces
+# --------------------------------------------------------------------------
+
+def test_rmsnorm_constant_vector():
+    x = np.where(rng.standard_normal(10) > 0, 4.0, -4.0)
+    w = rng.standard_normal(10)
+    np.testing.assert_allclose(O.rmsnorm(x, w, 0.0), np.sign(x) * w, rtol=1e-15)
+
+
+def test_rope_head_dim_two_is_plain_rotation():
+    x = np.array([[[1.0, 0.0]], [[0.0, 1.0]]])       # [n=2, heads=1, hd=2]
+    p = np.array([0.3, 1.1])
+    out = O.rope(x, p, theta=10000.0)
+    np.testing.assert_allclose(out[0, 0], [math.cos(0.3), math.sin(0.3)], rtol=1e-15)
+    np.testing.assert_allclose(out[1, 0], [-math.sin(1.1), math.cos(1.1)], rtol=1e-15)
+
+
+def test_rope_second_pair_frequency():
+    # hd = 4, pair i = 1 turns at theta^(-2/4) = 1/10 for theta = 100
+    x = np.array([[[0.0, 0.0, 1.0, 0.0]]])
+    out = O.rope(x, np.array([5.0]), theta=100.0)
+    np.testing.assert_allclose(out[0, 0], [0, 0, math.cos(0.5), math.sin(0.5)], atol=1e-15)
+
+
+def test_rope_position_zero_identity_and_norm():
+    x = rng.standard_normal((3, 2, 8))
+    np.testing.assert_allclose(O.rope(x, np.zeros(3), 10000.0), x, rtol=0, atol=0)
+    y = O.rope(x, np.array([3.0, 77.0, 1234.0]), 10000.0)
+    np.testing.assert_allclose(np.linalg.norm(y, axis=-1), np.linalg.norm(x, axis=-1), rtol=1e-14)
+
+
+def test_rope_scores_depend_on_relative_position_only():
+    q = rng.standard_normal((1, 1, 16))
+    k = rng.standard_normal((1, 1, 16))
+    s1 = (O.rope(q, [40.0], 1e4) * O.rope(k, [13.0], 1e4)).sum()
+    s2 = (O.rope(q, [527.0], 1e4) * O.rope(k, [500.0], 1e4)).sum()
+    np.testing.assert_allclose(s1, s2, rtol=1e-10)
+
+
+def test_attention_zero_query_is_value_mean():
+    k = rng.standard_normal((9, 8))
+    v = rng.standard_normal((9, 8))
+    out = O.softmax_attention(np.zeros((2, 8)), k, v)
+    np.testing.assert_allclose(out, np.broadcast_to(v.mean(0), (2, 8)), rtol=1e-14)
+
+
+def test_attention_single_key_returns_value():
+    v = rng.standard_normal((1, 8))
+    out = O.softmax_attention(rng.standard_normal((3, 8)), rng.standard_normal((1, 8)), v)
+    np.testing.assert_allclose(out, np.broadcast_to(v, (3, 8)), rtol=1e-14)
+
+
+def test_attention_two_keys_closed_form():
+    q = rng.standard_normal((1, 4))
+    k = rng.standard_normal((2, 4))
+    v = rng.standard_normal((2, 4))
+    delta = (q[0] @ k[0] - q[0] @ k[1]) / 2.0     # sqrt(hd) = 2
+    w0 = 1.0 / (1.0 + math.exp(-delta))
+    np.testing.assert_allclose(O.softmax_attention(q, k, v)[0], w0 * v[0] + (1 - w0) * v[1], rtol=1e-13)
+
+
+def test_attention_key_permutation_invariance():
+    q = rng.standard_normal((4, 8))
+    k = rng.standard_normal((11, 8))
+    v = rng.standard_normal((11, 8))
+    perm = rng.permutation(11)
+    np.testing.assert_allclose(O.softmax_attention(q, k, v),
+                               O.softmax_attention(q, k[perm], v[perm]), rtol=1e-13)
+
+
+def test_silu_points():
+    assert O.silu(np.array([0.0]))[0] == 0.0
+    np.testing.assert_allclose(O.silu(np.array([math.log(3.0)]))[0], 0.75 * math.log(3.0), rtol=1e-15)
+    np.testing.assert_allclose(O.silu(np.array([-40.0]))[0], -40.0 / (1 + math.exp(40.0)), rtol=1e-12)
+
+
+# --------------------------------------------------------------------------
+# draft block wiring
+# --------------------------------------------------------------------------
+
+def _tiny_weights(d=16, F=32, V=50, L=1, seed=0):
+    r = np.random.default_rng(seed)
+    W = {"embed": r.standard_normal((V, d)) * 0.5, "mask_vec": r.standard_normal(d) * 0.5,
+         "ctx_norm": 1 + 0.1 * r.standard_normal(d), "final_norm": 1 + 0.1 * r.standard_normal(d),
+         "layers": []}
+    for _ in range(L):
+        W["layers"].append({
+            "attn_norm": 1 + 0.1 * r.standard_normal(d), "mlp_norm": 1 + 0.1 * r.standard_normal(d),
+            "wq": r.standard_normal((d, d)) * 0.3, "wk": r.standard_normal((d, d)) * 0.3,
+            "wv": r.standard_normal((d, d)) * 0.3, "wo": r.standard_normal((d, d)) * 0.3,
+            "wg": r.standard_normal((F, d)) * 0.3, "wu": r.standard_normal((F, d)) * 0.3,
+            "wd": r.standard_normal((d, F)) * 0.3})
+    return W
+
+
+def test_draft_block_zero_output_projections_keep_block_input():
+    # W_o = W_d = 0: the residual stream stays the block input, so the output is
+    # RMSNorm_final of [embed[anchor]; mask_vec ...].  With +-a entries that is
+    # sign * final_norm exactly (eps 0).
+    d = 16
+    W = _tiny_weights(d=d)
+    W["embed"] = np.where(W["embed"] > 0, 0.25, -0.25)
+    W["mask_vec"] = np.where(W["mask_vec"] > 0, 2.0, -2.0)
+    for lw in W["layers"]:
+        lw["wo"][:] = 0
+        lw["wd"][:] = 0
+    ctx = rng.standard_normal((10, d))
+    out = O.draft_block(W, ctx, [0, 4, 10], [7, 3], block=4, n_heads=2, head_dim=8,
+                        rope_theta=1e4, norm_eps=0.0, act_dtype="f64")
+    for i, a in enumerate([7, 3]):
+        np.testing.assert_allclose(out[i * 4], np.sign(W["embed"][a]) * W["final_norm"], rtol=1e-14)
+        for k in range(1, 4):
+            np.testing.assert_allclose(out[i * 4 + k], np.sign(W["mask_vec"]) * W["final_norm"], rtol=1e-14)
+
+
+def test_draft_block_zero_query_averages_own_sequence_context_and_block():
+    # W_q = 0 -> uniform attention over this sequence's T_i context keys plus its
+    # B block keys, and over nothing else (ragged sequences do not mix).
+    d, B = 16, 4
+    W = _tiny_weights(d=d)
+    W["layers"][0]["wq"][:] = 0
+    ctx = rng.standard_normal((10, d))
+    cu = [0, 3, 10]
+    inter = {}
+    O.draft_block(W, ctx, cu, [1, 2], block=B, n_heads=2, head_dim=8, rope_theta=1e4,
+                  norm_eps=1e-6, act_dtype="f64", intermediates=inter)
+    L0 = inter["layers"][0]
+    for i in range(2):
+        v_all = np.concatenate([L0["Vc"][cu[i]:cu[i + 1]], L0["Vb"][i * B:(i + 1) * B]], axis=0)
+        for k in range(B):
+            np.testing.assert_allclose(L0["O"][i * B + k], v_all.mean(axis=0), rtol=1e-12)
+
+
+def test_draft_block_sequences_are_independent():
+    d, B = 16, 4
+    W = _tiny_weights(d=d)
+    ctx = rng.standard_normal((10, d))
+    cu = [0, 3, 10]
+    a = O.draft_block(W, ctx, cu, [1, 2], block=B, n_heads=2, head_dim=8, rope_theta=1e4,
+                      norm_eps=1e-6, act_dtype="f64")
+    ctx2 = ctx.copy()
+    ctx2[5:] += 1.0                     # only sequence 1's context changes
+    b = O.draft_block(W, ctx2, cu, [1, 2], block=B, n_heads=2, head_dim=8, rope_theta=1e4,
+                      norm_eps=1e-6, act_dtype="f64")
+    np.testing.assert_array_equal(a[:B], b[:B])
+    assert np.abs(a[B:] - b[B:]).max() > 1e-6
+
+
+# --------------------------------------------------------------------------
+# LM head, accept, tau, KL
+# --------------------------------------------------------------------------
+
+def test_lm_head_argmax_first_index_on_ties_brute_force():
+    h = rng.standard_normal((6, 8))
+    W = rng.standard_normal((40, 8))
+    W[17] = W[5]                       # exact duplicate rows -> exact tie in z
+    h[2] = W[5] * 10                   # row 2's max is the (5, 17) tie
+    res = O.lm_head(h, W)
+    z = h @ W.T
+    for i in range(6):
+        best, bi = -math.inf, -1
+        for v in range(40):
+            if z[i, v] > best:
+                best, bi = z[i, v], v
+        assert res["tok"][i] == bi
+    assert res["tok"][2] == 5
+
+
+def test_logsoftmax_normalised_and_argmax_preserved():
+    h = rng.standard_normal((5, 8))
+    W = rng.standard_normal((30, 8))
+    for it in (1.0, 0.5, 3.0):
+        res = O.lm_head(h, W, inv_temp=it, logsoftmax=True)
+        np.testing.assert_allclose(np.log(np.exp(res["logsoftmax"]).sum(1)), 0.0, atol=1e-13)
+        assert np.array_equal(np.argmax(res["logsoftmax"], 1), res["tok"])
+
+
+def test_logsoftmax_two_class_closed_form():
+    h = np.array([[1.0]])
+    W = np.array([[2.0], [0.5]])
+    res = O.lm_head(h, W, inv_temp=1.0, logsoftmax=True)
+    np.testing.assert_allclose(res["logsoftmax"][0], [-math.log1p(math.exp(-1.5)),
+                                                      -math.log1p(math.exp(1.5))], rtol=1e-14)
+
+
+def test_accept_len_against_cumprod_and_edges():
+    d = rng.integers(0, 5, size=(200, 7))
+    t = rng.integers(0, 5, size=(200, 7))
+    t[::3] = d[::3]
+    expect = np.cumprod(d == t, axis=1).sum(axis=1)
+    assert np.array_equal(O.accept_len(d, t), expect)
+    assert O.accept_len(d[:1], d[:1])[0] == 7
+    t2 = d[:1].copy()
+    t2[0, 0] += 1
+    assert O.accept_len(d[:1], t2)[0] == 0
+
+
+def test_tau_counts_bonus_token_table2():
+    g = json.load(open(os.path.join(GOLDEN, "table2_mtp3_tau.json")))
+    k = g["drafted_steps"]
+    taus = list(g["tau_per_benchmark"].values())
+    # a drafts-only count can never exceed k; the printed values do
+    assert max(taus) > k
+    # with the bonus token tau lies in [1, k + 1] and reaches k + 1 on full acceptance
+    assert all(1.0 <= t <= k + 1 for t in taus)
+    assert O.mean_accepted_length([k, k]) == k + 1
+    assert O.mean_accepted_length([0]) == 1.0
+    # the Average column is the arithmetic mean of the seven benchmarks
+    assert round(sum(taus) / len(taus), 2) == g["tau_average_printed"]
+
+
+def test_kl_pins():
+    z = rng.standard_normal((2, 9))
+    assert abs(O.kl_distill(z, z, 1.0)) < 1e-14
+    assert O.kl_distill(z, rng.standard_normal((2, 9)), 2.0) > 0
+    # two classes: p = (3/4, 1/4), q = (1/2, 1/2) -> KL = 3/4 ln 3/2 + 1/4 ln 1/2
+    t = np.array([[math.log(3.0), 0.0]])
+    s = np.array([[0.0, 0.0]])
+    np.testing.assert_allclose(O.kl_distill(t, s, 1.0),
+                               0.75 * math.log(1.5) + 0.25 * math.log(0.5), rtol=1e-14)
+    # T^2 factor: logits scaled with T keep p, q fixed, loss scales by T^2
+    np.testing.assert_allclose(O.kl_distill(2 * t, 2 * s, 2.0),
+                               4 * O.kl_distill(t, s, 1.0), rtol=1e-13)
