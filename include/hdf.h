@@ -1,0 +1,232 @@
+/*
+ * hdf.h — C ABI of the GB300 (sm_103a) HyperDFlash block-drafting library.
+ *
+ * One draft step is four calls, in the order of the method:
+ *   hdf_gated_reduce    Eq. 1 (Sec. 2.2): m-path pre-collapse residual -> [T, d]
+ *   hdf_draft_block     Sec. 2.1/2.3: conditioning projection + one non-causal
+ *                       block forward of [anchor, mask x (B-1)] over the context
+ *   hdf_lm_head_argmax  Sec. 2.3: logits, argmax drafts, optional log-softmax
+ *                       at temperature T_KD (the q^{T_KD} of Eq. 2)
+ *   hdf_accept_len      Sec. 3.4: accepted-prefix length of each block
+ *
+ * Conventions shared by every call
+ *   - All tensor arguments are DEVICE pointers owned by the caller, row-major,
+ *     16-byte aligned, densely packed unless a stride argument says otherwise.
+ *     The library keeps no pointer after a call returns.
+ *   - The library allocates nothing.  Scratch comes from a caller workspace
+ *     (256-byte aligned) whose size the matching *_workspace_size() returns.
+ *   - Every call is asynchronous on the caller's CUDA stream (a cudaStream_t
+ *     passed as hdf_stream_t; NULL = legacy default stream).  No call
+ *     synchronises, and there is no host fallback: if the CUDA kernels cannot
+ *     run the call returns HDF_ERR_CUDA.
+ *   - Arguments are validated on the host before any launch; a rejected call
+ *     launches nothing and returns a non-zero status.  hdf_last_error() gives
+ *     a human-readable reason (thread-local, valid until the next call).
+ *   - dtype is HDF_BF16 (bf16 storage, fp32 accumulation) or HDF_F32 (fp32
+ *     storage; GEMMs then run on the tensor cores' tf32 mode).
+ *   - Kernels that wait on hardware barriers give up after a bounded time and
+ *     record HDF_ERR_DEVICE_CHECK in a device status word that
+ *     hdf_device_status() reads; they never trap.
+ */
+#ifndef HDF_H
+#define HDF_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#if defined(__GNUC__)
+#define HDF_API __attribute__((visibility("default")))
+#else
+#define HDF_API
+#endif
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef struct CUstream_st* hdf_stream_t; /* ABI-identical to cudaStream_t */
+
+enum hdf_status {
+  HDF_OK = 0,
+  HDF_ERR_INVALID_ARG = 1,  /* null pointer, non-finite or out-of-range scalar */
+  HDF_ERR_SHAPE = 2,        /* sizes inconsistent or outside the supported set */
+  HDF_ERR_DTYPE = 3,        /* unknown dtype */
+  HDF_ERR_ALIGNMENT = 4,    /* a pointer is not 16-byte aligned */
+  HDF_ERR_WORKSPACE = 5,    /* workspace missing, misaligned or too small */
+  HDF_ERR_CUDA = 6,         /* a CUDA runtime/driver call or launch failed */
+  HDF_ERR_UNSUPPORTED = 7,  /* valid request this build does not implement */
+  HDF_ERR_DEVICE_CHECK = 8  /* a kernel's bounded wait gave up (device word) */
+};
+
+enum hdf_dtype { HDF_F32 = 0, HDF_BF16 = 1 };
+
+/* Version of this ABI (major * 100 + minor). */
+HDF_API int hdf_version(void);
+/* Static string for a status code. */
+HDF_API const char* hdf_status_str(int status);
+/* Detail of the last failed call on this host thread ("" if none). */
+HDF_API const char* hdf_last_error(void);
+/* Synchronises the current device, returns the device status word
+ * (HDF_OK or HDF_ERR_DEVICE_CHECK) and clears it when reset != 0. */
+HDF_API int hdf_device_status(int reset);
+
+/* ------------------------------------------------------------------------
+ * (1) Inherited HC-Gate reducer — Eq. 1 and the paragraph after it (Sec. 2.2)
+ *
+ *   r_t     = (mean_{m*d}(vec H_t ^2) + rms_eps)^(-1/2)
+ *   g_tj    = gate_scale * r_t * (W_f vec H_t)_j + b_j
+ *   alpha_tj= sigmoid(g_tj) + gate_offset        (independent per-path gates)
+ *   y_t     = sum_j alpha_tj * H^_tj
+ * with H^_tj = H_tj, or, when path_norm_w != NULL, the drafter-side per-path
+ * RMSNorm H_tj * (mean_d(H_tj^2) + path_norm_eps)^(-1/2) * path_norm_w[j].
+ * vec() is path-major: vec(H_t)[p*d + e] = H_t[p][e].
+ *
+ *   H            [n_tokens, m, d]  dtype     pre-collapse residual
+ *   Wf           [m, m*d]          dtype     gate weight (RMSNorm weight folded in)
+ *   b            [m]               fp32      gate bias
+ *   path_norm_w  [m, d] dtype or NULL
+ *   alpha_override [n_tokens, m] fp32 or NULL: use these gates instead
+ *                (alpha = 1/m gives mean pooling, one-hot selects a path);
+ *                Wf and b are then not read and may be NULL
+ *   y            [n_tokens, d]     dtype     output (may not alias H)
+ *   alpha_out    [n_tokens, m] fp32 or NULL: the gates actually applied
+ * Supported: 1 <= m <= 8 (m in {1,2,3,4,8}), d % 8 == 0 (bf16) or d % 4 == 0
+ * (fp32), d <= 16384, n_tokens >= 0 (0 launches nothing).
+ * ---------------------------------------------------------------------- */
+HDF_API int hdf_gated_reduce(const void* H, int dtype, int64_t n_tokens, int m, int d,
+                     const void* Wf, const float* b,
+                     float rms_eps, float gate_scale, float gate_offset,
+                     const void* path_norm_w, float path_norm_eps,
+                     const float* alpha_override,
+                     void* y, float* alpha_out, hdf_stream_t stream);
+
+/* Generic fc reducer of vanilla DFlash (Sec. 2.2, Table 1 "generic fc"),
+ * kept as the comparison path and the fallback the paper names:
+ *   y_t = W_fc vec(H_t),   W_fc [d, m*d] dtype, y [n_tokens, d] dtype.
+ * Runs on the tcgen05 GEMM.  Workspace: hdf_fc_reduce_workspace_size(). */
+HDF_API size_t hdf_fc_reduce_workspace_size(int64_t n_tokens, int m, int d, int dtype);
+HDF_API int hdf_fc_reduce(const void* H, int dtype, int64_t n_tokens, int m, int d,
+                  const void* W_fc, void* y, void* ws, size_t ws_bytes,
+                  hdf_stream_t stream);
+
+/* ------------------------------------------------------------------------
+ * (2) Drafter block forward — anchor-plus-mask block input (Sec. 2.1),
+ *     conditioning on the reduced pre-collapse residual (Sec. 2.1/2.2),
+ *     block slot k predicts the token at a+k (Sec. 2.3).
+ *
+ * For every sequence i with context rows ctx[cu_ctx[i] .. cu_ctx[i+1]):
+ *   c      = RMSNorm_{ctx_norm}(ctx)
+ *   h      = [embed[anchor_i]; mask_vec x (B-1)]          (fp32 residual)
+ *   per layer:
+ *     K_c  = RoPE(c W_k^T, t),  V_c = c W_v^T             (t = 0 .. T_i-1)
+ *     x    = RMSNorm_{attn_norm}(h)
+ *     Q, K_b, V_b = RoPE(x W_q^T), RoPE(x W_k^T), x W_v^T (positions T_i + k)
+ *     O    = softmax(Q [K_c; K_b]^T / sqrt(hd)) [V_c; V_b] per head, no mask
+ *     h   += O W_o^T
+ *     x    = RMSNorm_{mlp_norm}(h)
+ *     h   += (silu(x W_g^T) * (x W_u^T)) W_d^T
+ *   h_out  = RMSNorm_{final_norm}(h)
+ * RoPE turns pairs (2i, 2i+1) of each head by pos * theta^(-2i/hd), using the
+ * caller's tables from hdf_rope_table().  All RMSNorms use shape.norm_eps.
+ * bf16 storage points: c, K_c, V_c, x, Q, K_b, V_b, O, silu(.)*(.), h_out.
+ * ---------------------------------------------------------------------- */
+typedef struct {
+  const void* attn_norm; /* [d] */
+  const void* wq;        /* [d, d]  (out, in) */
+  const void* wk;        /* [d, d] */
+  const void* wv;        /* [d, d] */
+  const void* wo;        /* [d, d] */
+  const void* mlp_norm;  /* [d] */
+  const void* wg;        /* [F, d] */
+  const void* wu;        /* [F, d] */
+  const void* wd;        /* [d, F] */
+} hdf_layer_weights;
+
+typedef struct {
+  const void* embed;       /* [V, d] */
+  const void* mask_vec;    /* [d]   the learned mask-token vector */
+  const void* ctx_norm;    /* [d] */
+  const void* final_norm;  /* [d] */
+  const float* rope_cos;   /* [rope_max_pos, head_dim/2] fp32 */
+  const float* rope_sin;   /* [rope_max_pos, head_dim/2] fp32 */
+  int64_t rope_max_pos;    /* must exceed max_ctx + block - 1 */
+  const hdf_layer_weights* layers; /* HOST array of n_layers entries */
+} hdf_drafter_weights;
+
+typedef struct {
+  int dtype;       /* HDF_BF16 or HDF_F32, for weights and activations */
+  int batch;       /* sequences */
+  int block;       /* B: anchor + B-1 mask slots, 2..16 */
+  int d;           /* hidden width, d % 128 == 0 */
+  int n_heads;     /* n_heads * head_dim == d */
+  int head_dim;    /* 64 or 128 */
+  int ffn;         /* SwiGLU width F, F % 64 == 0 */
+  int vocab;       /* V (embedding rows) */
+  int n_layers;    /* >= 1 */
+  int max_ctx;     /* upper bound on every T_i (host-side grid sizing) */
+  int64_t n_ctx;   /* sum of T_i == cu_ctx[batch] */
+  float norm_eps;  /* RMSNorm epsilon */
+} hdf_draft_shape;
+
+/* Optional per-stage timing: events[k] (cudaEvent_t) is recorded on the
+ * stream before stage k and events[last] after the final stage, so
+ * n_events = 3 + HDF_DRAFT_STAGES_PER_LAYER * n_layers (or pass NULL).
+ * Stages: context norm, then per layer {context K/V GEMM, block
+ * norm (+embedding), QKV GEMM, attention (+combine), O GEMM, MLP norm,
+ * gate/up GEMM, down GEMM}, then the final norm. */
+#define HDF_DRAFT_STAGES_PER_LAYER 8
+typedef struct {
+  void* const* events;
+  int n_events;
+} hdf_trace;
+
+HDF_API size_t hdf_draft_block_workspace_size(const hdf_draft_shape* shape);
+HDF_API int hdf_draft_block(const hdf_drafter_weights* w, const hdf_draft_shape* shape,
+                    const void* ctx,        /* [n_ctx, d] dtype (y of Eq. 1) */
+                    const int32_t* cu_ctx,  /* [batch + 1] prefix sums of T_i */
+                    const int32_t* anchor,  /* [batch] anchor token ids */
+                    void* h_out,            /* [batch * block, d] dtype */
+                    void* ws, size_t ws_bytes,
+                    const hdf_trace* trace, /* NULL: no timing events */
+                    hdf_stream_t stream);
+
+/* cos/sin tables for the drafter's RoPE: entry [p][i] = cos/sin of
+ * p * theta^(-2i/head_dim), computed in fp64 on the device and stored fp32.
+ * A per-model constant: build once, pass through hdf_drafter_weights. */
+HDF_API int hdf_rope_table(double theta, int head_dim, int64_t max_pos,
+                   float* cos_out, float* sin_out, hdf_stream_t stream);
+
+/* ------------------------------------------------------------------------
+ * (3) LM head — draft logits z = h W_lm^T (Sec. 2.3), greedy drafts
+ *     tok = argmax_v z (lowest index wins ties), optional fp32 log-softmax
+ *     of z * inv_temp, the log of q^{T_KD} in Eq. 2 (inv_temp = 1/T_KD).
+ *
+ *   h           [M, d]  dtype
+ *   W_lm        [V, d]  dtype
+ *   tok         [M]     int32
+ *   zmax        [M]     fp32 or NULL: the maximal logit
+ *   logsoftmax  [M, V]  fp32 or NULL
+ * Row r = i*B + k of a block: k >= 1 holds draft d_k of sequence i.
+ * ---------------------------------------------------------------------- */
+HDF_API size_t hdf_lm_head_workspace_size(int64_t M, int d, int64_t V, int dtype);
+HDF_API int hdf_lm_head_argmax(const void* h, int dtype, int64_t M, int d,
+                       const void* W_lm, int64_t V, float inv_temp,
+                       int32_t* tok, float* zmax, float* logsoftmax,
+                       void* ws, size_t ws_bytes, hdf_stream_t stream);
+
+/* ------------------------------------------------------------------------
+ * (4) Block verification — greedy acceptance (Sec. 1, Sec. 3.4):
+ *   accept[i] = max{ n <= n_draft : draft[i][k] == target[i][k] for k < n }
+ * draft row i starts at draft + i*draft_stride (elements), likewise target,
+ * so the drafts can be read straight out of hdf_lm_head_argmax's tok
+ * (draft = tok + 1, draft_stride = B).  tau = mean(accept + 1) counts the
+ * bonus token (Table 2 prints tau above the number of drafted steps).
+ * ---------------------------------------------------------------------- */
+HDF_API int hdf_accept_len(const int32_t* draft, int64_t draft_stride,
+                   const int32_t* target, int64_t target_stride,
+                   int batch, int n_draft, int32_t* accept, hdf_stream_t stream);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* HDF_H */

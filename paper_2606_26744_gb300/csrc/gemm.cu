@@ -1,0 +1,468 @@
+// tcgen05 / TMEM GEMM for the dense contractions of the draft step:
+// the conditioning projection (context K/V), the block Q/K/V/O projections,
+// the SwiGLU MLP and the LM head (Sec. 2.1-2.3 of the HyperDFlash paper as
+// read for the drafter), plus the generic fc reducer of Table 1.
+//
+//   D[M, N] = A[M, K] * B[N, K]^T      (both operands K-major)
+//
+// One CTA of 4 warps computes a 128 x BN tile (optionally one K-split of it):
+//   warp 0 / lane 0  TMA producer: A as two 64-row boxes, B as one BN-row box,
+//                    128-byte swizzle, into a STAGES-deep shared-memory ring
+//   warp 1 / lane 0  MMA issuer: tcgen05.mma.cta_group::1 (kind::f16 for bf16,
+//                    kind::tf32 for fp32), 4 MMAs of K=16 (bf16) per stage,
+//                    fp32 accumulator in TMEM, tcgen05.commit frees the stage
+//   warp 2           TMEM allocation / release
+//   all 4 warps      epilogue: tcgen05.ld 32x32b (thread i <-> TMEM lane i =
+//                    tile row i), fused RoPE / residual add / SwiGLU / LM-head
+//                    argmax + sum-exp partials, direct global stores.
+// Split-K writes fp32 partial tiles; the last CTA of a tile to arrive (atomic
+// ticket, no waiting) sums them in a fixed order and runs the epilogue.
+#include <algorithm>
+#include <climits>
+
+#include "common.cuh"
+#include "kernels.h"
+
+namespace hdf {
+namespace {
+
+constexpr int BM = 128;
+constexpr int ROW_BYTES = 128;  // one 128-byte swizzle row per tile row and stage
+
+template <typename T> struct GT;
+template <> struct GT<__nv_bfloat16> {
+  static constexpr int BK = 64;
+  static constexpr uint32_t FMT = 1;  // bf16
+};
+template <> struct GT<float> {
+  static constexpr int BK = 32;
+  static constexpr uint32_t FMT = 2;  // tf32
+};
+
+constexpr int stages_for(int bn) { return bn >= 256 ? 4 : (bn >= 128 ? 3 : (bn >= 64 ? 4 : 5)); }
+constexpr int smem_for(int bn) { return stages_for(bn) * (BM + bn) * ROW_BYTES + 1024; }
+
+__device__ __forceinline__ void operand_rows(const Operand& op, int tile_row0, int half, int tile_idx,
+                                             const CUtensorMap** map, int* row) {
+  if (op.mode == kPair64) {
+    *map = &op.map[half];
+    *row = tile_idx * 64;
+  } else {
+    const int r = tile_row0 + half * 64;
+    const int mi = r / op.rows_per_map;
+    *map = &op.map[mi];
+    *row = r - mi * op.rows_per_map;
+  }
+}
+
+__device__ __forceinline__ int ctx_position(const int* cu, int batch, long long t) {
+  int lo = 0, hi = batch;  // find b with cu[b] <= t < cu[b+1]
+  while (hi - lo > 1) {
+    const int mid = (lo + hi) >> 1;
+    if (__ldg(cu + mid) <= t) lo = mid; else hi = mid;
+  }
+  return (int)(t - __ldg(cu + lo));
+}
+__device__ __forceinline__ int block_position(const int* cu, int block, int j) {
+  const int b = j / block;
+  return (__ldg(cu + b + 1) - __ldg(cu + b)) + (j - b * block);
+}
+
+template <typename T>
+__device__ __forceinline__ void store16(T* dst, const float* v);
+template <>
+__device__ __forceinline__ void store16<__nv_bfloat16>(__nv_bfloat16* dst, const float* v) {
+  uint4* p = reinterpret_cast<uint4*>(dst);
+  p[0] = V16<__nv_bfloat16>::pack(v);
+  p[1] = V16<__nv_bfloat16>::pack(v + 8);
+}
+template <>
+__device__ __forceinline__ void store16<float>(float* dst, const float* v) {
+  float4* p = reinterpret_cast<float4*>(dst);
+#pragma unroll
+  for (int i = 0; i < 4; ++i) p[i] = make_float4(v[4 * i], v[4 * i + 1], v[4 * i + 2], v[4 * i + 3]);
+}
+
+// Epilogue for one 16-column chunk of the tile.  Called by all 128 threads
+// with identical (tile, c0) so that shuffles and barriers are uniform.
+template <typename T, int BN>
+__device__ __forceinline__ void epilogue_chunk(const GemmArgs& g, int tile_m, int tile_n, int c0,
+                                               float* v, uint8_t* smem) {
+  const Epilogue& E = g.epi;
+  const int row = threadIdx.x;
+  const int lane = row & 31, warp = row >> 5;
+  switch (E.kind) {
+    case kEpiStore: {  // rows = tokens, columns = output features
+      const long long t = (long long)tile_m * BM + row;
+      const int col0 = tile_n * BN + c0;
+      if (t >= g.M || col0 >= g.N) return;
+      const int seg = col0 / E.seg_width;
+      const int fl = col0 - seg * E.seg_width;
+      if ((E.rope_mask >> seg) & 1) {
+        const int pos = (int)min((long long)ctx_position(E.cu_ctx, E.batch, t), E.rope_rows - 1);
+        const int hh = E.head_dim >> 1;
+        const float* cs = E.rope_cos + (size_t)pos * hh;
+        const float* sn = E.rope_sin + (size_t)pos * hh;
+#pragma unroll
+        for (int i = 0; i < 8; ++i) {
+          const int pi = ((fl + 2 * i) % E.head_dim) >> 1;
+          const float c = __ldg(cs + pi), s = __ldg(sn + pi);
+          const float x0 = v[2 * i], x1 = v[2 * i + 1];
+          v[2 * i] = x0 * c - x1 * s;
+          v[2 * i + 1] = x0 * s + x1 * c;
+        }
+      }
+      store16<T>(reinterpret_cast<T*>(E.out[seg]) + t * E.ld + fl, v);
+      return;
+    }
+    case kEpiStoreT: {  // rows = output features, columns = tokens
+      const int f = tile_m * BM + row;
+      const int seg = f / E.seg_width;
+      const int fl = f - seg * E.seg_width;
+      const int jb = tile_n * BN + c0;
+      if ((E.rope_mask >> seg) & 1) {  // pair (2i, 2i+1) lives in lanes (l, l^1)
+        const bool even = (fl & 1) == 0;
+        const int hh = E.head_dim >> 1;
+        const int pi = (fl % E.head_dim) >> 1;
+#pragma unroll
+        for (int k = 0; k < 16; ++k) {
+          const float pv = __shfl_xor_sync(0xffffffffu, v[k], 1);
+          const int j = jb + k;
+          if (j < g.N) {
+            const int pos = (int)min((long long)block_position(E.cu_ctx, E.block, j), E.rope_rows - 1);
+            const float c = __ldg(E.rope_cos + (size_t)pos * hh + pi);
+            const float s = __ldg(E.rope_sin + (size_t)pos * hh + pi);
+            v[k] = even ? (v[k] * c - pv * s) : (pv * s + v[k] * c);
+          }
+        }
+      }
+      if (f >= g.M) return;
+      T* out = reinterpret_cast<T*>(E.out[seg]);
+#pragma unroll
+      for (int k = 0; k < 16; ++k) {
+        const int j = jb + k;
+        if (j < g.N) out[(long long)j * E.ld + fl] = from_f32<T>(v[k]);
+      }
+      return;
+    }
+    case kEpiResidT: {
+      const int f = tile_m * BM + row;
+      if (f >= g.M) return;
+      const int jb = tile_n * BN + c0;
+#pragma unroll
+      for (int k = 0; k < 16; ++k) {
+        const int j = jb + k;
+        if (j < g.N) {
+          float* p = E.resid + (long long)j * E.ld + f;
+          *p = *p + v[k];
+        }
+      }
+      return;
+    }
+    case kEpiSwigluT: {  // rows 0..63: gate g_f, rows 64..127: up u_f (same f)
+      float* xbuf = reinterpret_cast<float*>(smem);  // [64][17]
+      if (row >= 64) {
+#pragma unroll
+        for (int k = 0; k < 16; ++k) xbuf[(row - 64) * 17 + k] = v[k];
+      }
+      __syncthreads();
+      if (row < 64) {
+        const int f = tile_m * 64 + row;
+        const int jb = tile_n * BN + c0;
+        T* act = reinterpret_cast<T*>(E.out[0]);
+        if (f < E.seg_width) {
+#pragma unroll
+          for (int k = 0; k < 16; ++k) {
+            const int j = jb + k;
+            if (j < g.N) {
+              const float gv = v[k];
+              const float u = xbuf[row * 17 + k];
+              act[(long long)j * E.ld + f] = from_f32<T>(gv / (1.0f + expf(-gv)) * u);
+            }
+          }
+        }
+      }
+      __syncthreads();
+      return;
+    }
+    case kEpiLmHeadT: {  // rows = vocabulary entries, columns = tokens
+      float* rmax = reinterpret_cast<float*>(smem);  // [4][16]
+      int* rarg = reinterpret_cast<int*>(smem + 256);
+      float* rsum = reinterpret_cast<float*>(smem + 512);
+      const long long V = g.M;
+      const long long vr = (long long)tile_m * BM + row;
+      const bool valid = vr < V;
+      const int jb = tile_n * BN + c0;
+      if (E.logsoftmax && valid) {
+#pragma unroll
+        for (int k = 0; k < 16; ++k)
+          if (jb + k < g.N) E.logsoftmax[(long long)(jb + k) * V + vr] = v[k] * E.inv_temp;
+      }
+      float bv[16];
+      int bi[16];
+#pragma unroll
+      for (int k = 0; k < 16; ++k) {
+        bv[k] = valid ? v[k] : -INFINITY;
+        bi[k] = valid ? (int)vr : INT_MAX;
+      }
+#pragma unroll
+      for (int o = 16; o >= 1; o >>= 1) {
+#pragma unroll
+        for (int k = 0; k < 16; ++k) {
+          const float ov = __shfl_xor_sync(0xffffffffu, bv[k], o);
+          const int oi = __shfl_xor_sync(0xffffffffu, bi[k], o);
+          if (ov > bv[k] || (ov == bv[k] && oi < bi[k])) { bv[k] = ov; bi[k] = oi; }
+        }
+      }
+#pragma unroll
+      for (int k = 0; k < 16; ++k) {
+        float e = valid ? expf((v[k] - bv[k]) * E.inv_temp) : 0.f;
+        e = warp_sum(e);
+        if (lane == k) {
+          rmax[warp * 16 + k] = bv[k];
+          rarg[warp * 16 + k] = bi[k];
+          rsum[warp * 16 + k] = e;
+        }
+      }
+      __syncthreads();
+      if (row < 16) {
+        const int k = row, j = jb + k;
+        float m = rmax[k];
+        int a = rarg[k];
+        for (int w = 1; w < 4; ++w) {
+          const float mw = rmax[w * 16 + k];
+          const int aw = rarg[w * 16 + k];
+          if (mw > m || (mw == m && aw < a)) { m = mw; a = aw; }
+        }
+        float s = 0.f;
+        for (int w = 0; w < 4; ++w) {
+          const float mw = rmax[w * 16 + k];
+          if (mw != -INFINITY) s += rsum[w * 16 + k] * expf((mw - m) * E.inv_temp);
+        }
+        if (j < g.N) {
+          const size_t o = (size_t)tile_m * g.N + j;
+          E.part_max[o] = m;
+          E.part_arg[o] = a;
+          E.part_sum[o] = s;
+        }
+      }
+      __syncthreads();
+      return;
+    }
+  }
+}
+
+template <typename T, int BN>
+__global__ void __launch_bounds__(128, 1) gemm_kernel(const __grid_constant__ GemmArgs g) {
+  constexpr int STAGES = stages_for(BN);
+  constexpr int BK = GT<T>::BK;
+  constexpr int A_BYTES = BM * ROW_BYTES;
+  constexpr int B_BYTES = BN * ROW_BYTES;
+  constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
+  constexpr uint32_t TMEM_COLS = BN < 32 ? 32 : BN;
+  constexpr uint32_t IDESC = umma_idesc(BM, BN, GT<T>::FMT);
+
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                             ~static_cast<uintptr_t>(1023));
+  __shared__ __align__(8) uint64_t full_bar[STAGES];
+  __shared__ __align__(8) uint64_t empty_bar[STAGES];
+  __shared__ __align__(8) uint64_t acc_bar;
+  __shared__ uint32_t tmem_slot;
+  __shared__ volatile int abort_flag;
+  __shared__ int last_flag;
+
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int tiles_m = (g.M + BM - 1) / BM;
+  const int tiles_n = (g.N + BN - 1) / BN;
+  int bid = blockIdx.x;
+  const int split = bid % g.k_splits;
+  bid /= g.k_splits;
+  const int GN = g.group_n < 1 ? 1 : g.group_n;
+  const int per_group = tiles_m * GN;
+  const int grp = bid / per_group;
+  const int rem = bid - grp * per_group;
+  const int n0 = grp * GN;
+  const int gw = min(GN, tiles_n - n0);
+  const int tile_m = rem / gw;
+  const int tile_n = n0 + rem % gw;
+
+  const int num_kb = (g.K + BK - 1) / BK;
+  const int kb_per = (num_kb + g.k_splits - 1) / g.k_splits;
+  const int kb0 = split * kb_per;
+  const int kb1 = min(num_kb, kb0 + kb_per);
+
+  if (tid == 0) {
+    for (int s = 0; s < STAGES; ++s) {
+      mbar_init(smem_u32(&full_bar[s]), 1);
+      mbar_init(smem_u32(&empty_bar[s]), 1);
+    }
+    mbar_init(smem_u32(&acc_bar), 1);
+    abort_flag = 0;
+    fence_mbar_init();
+  }
+  if (warp == 2) tmem_alloc(smem_u32(&tmem_slot), TMEM_COLS);
+  if (warp == 3 && lane == 0) {
+    prefetch_tmap(&g.A.map[0]);
+    prefetch_tmap(&g.B.map[0]);
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = tmem_slot;
+
+  if (warp == 0 && lane == 0) {
+    // ------------------------------------------------ TMA producer
+    int s = 0;
+    uint32_t ph = 0;
+    int issued = 0;
+    for (int kb = kb0; kb < kb1; ++kb) {
+      if (!mbar_wait(smem_u32(&empty_bar[s]), ph ^ 1, g.status)) { abort_flag = 1; break; }
+      if (abort_flag) break;
+      const uint32_t fb = smem_u32(&full_bar[s]);
+      mbar_arrive_expect_tx(fb, STAGE_BYTES);
+      const uint32_t sa = smem_u32(smem + s * STAGE_BYTES);
+      const uint32_t sb = sa + A_BYTES;
+      const CUtensorMap* map;
+      int row;
+#pragma unroll
+      for (int h = 0; h < 2; ++h) {
+        operand_rows(g.A, tile_m * BM, h, tile_m, &map, &row);
+        tma_load_2d(sa + h * (64 * ROW_BYTES), map, kb * BK, row, fb);
+      }
+      operand_rows(g.B, tile_n * BN, 0, tile_n, &map, &row);
+      tma_load_2d(sb, map, kb * BK, row, fb);
+      ++issued;
+      if (++s == STAGES) { s = 0; ph ^= 1; }
+    }
+    if (abort_flag) {
+      // let copies already in flight land before shared memory is released
+      int ss = s;
+      uint32_t pp = ph;
+      for (int i = 0; i < min(issued, STAGES); ++i) {
+        if (--ss < 0) { ss = STAGES - 1; pp ^= 1; }
+        mbar_wait(smem_u32(&full_bar[ss]), pp, nullptr);
+      }
+    }
+  } else if (warp == 1 && lane == 0) {
+    // ------------------------------------------------ MMA issuer
+    int s = 0;
+    uint32_t ph = 0;
+    for (int kb = kb0; kb < kb1; ++kb) {
+      if (!mbar_wait(smem_u32(&full_bar[s]), ph, g.status)) { abort_flag = 1; break; }
+      if (abort_flag) break;
+      tc_fence_after();
+      const uint32_t sa = smem_u32(smem + s * STAGE_BYTES);
+      const uint64_t ad = umma_desc_sw128(sa);
+      const uint64_t bd = umma_desc_sw128(sa + A_BYTES);
+#pragma unroll
+      for (int k = 0; k < 4; ++k)  // 4 x 32 bytes of K per 128-byte row
+        if (sizeof(T) == 2)
+          mma_bf16(tmem, ad + 2 * k, bd + 2 * k, IDESC, (kb > kb0 || k > 0) ? 1u : 0u);
+        else
+          mma_tf32(tmem, ad + 2 * k, bd + 2 * k, IDESC, (kb > kb0 || k > 0) ? 1u : 0u);
+      mma_commit(smem_u32(&empty_bar[s]));
+      if (++s == STAGES) { s = 0; ph ^= 1; }
+    }
+    mma_commit(smem_u32(&acc_bar));  // also drains every MMA issued above
+  }
+  __syncwarp();
+
+  // ------------------------------------------------------ epilogue
+  if (!mbar_wait(smem_u32(&acc_bar), 0, g.status)) abort_flag = 1;
+  tc_fence_after();
+  __syncthreads();
+  const bool aborted = abort_flag != 0;
+  const uint32_t taddr = tmem + ((uint32_t)(warp * 32) << 16);
+  if (!aborted && kb1 > kb0) {
+    if (g.k_splits == 1) {
+#pragma unroll 1
+      for (int c0 = 0; c0 < BN; c0 += 16) {
+        float v[16];
+        tmem_ld16(taddr + c0, v);
+        epilogue_chunk<T, BN>(g, tile_m, tile_n, c0, v, smem);
+      }
+    } else {
+      const int tile = tile_m * tiles_n + tile_n;
+      float* mine = g.ws_partial + ((size_t)(tile * g.k_splits + split) * BM + tid) * BN;
+#pragma unroll 1
+      for (int c0 = 0; c0 < BN; c0 += 16) {
+        float v[16];
+        tmem_ld16(taddr + c0, v);
+        float4* p = reinterpret_cast<float4*>(mine + c0);
+#pragma unroll
+        for (int i = 0; i < 4; ++i) __stcg(p + i, make_float4(v[4 * i], v[4 * i + 1], v[4 * i + 2], v[4 * i + 3]));
+      }
+      __threadfence();
+      __syncthreads();
+      if (tid == 0) last_flag = (atomicAdd(g.counters + tile, 1) == g.k_splits - 1);
+      __syncthreads();
+      if (last_flag) {
+        __threadfence();
+        const float* base = g.ws_partial + ((size_t)tile * g.k_splits * BM + tid) * BN;
+#pragma unroll 1
+        for (int c0 = 0; c0 < BN; c0 += 16) {
+          float v[16];
+#pragma unroll
+          for (int i = 0; i < 16; ++i) v[i] = 0.f;
+          for (int sp = 0; sp < g.k_splits; ++sp) {
+            const float4* p = reinterpret_cast<const float4*>(base + (size_t)sp * BM * BN + c0);
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+              const float4 q = __ldcg(p + i);
+              v[4 * i] += q.x; v[4 * i + 1] += q.y; v[4 * i + 2] += q.z; v[4 * i + 3] += q.w;
+            }
+          }
+          epilogue_chunk<T, BN>(g, tile_m, tile_n, c0, v, smem);
+        }
+        if (tid == 0) g.counters[tile] = 0;
+      }
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 2) {
+    tc_fence_after();
+    tmem_dealloc(tmem, TMEM_COLS);
+  }
+}
+
+template <typename T, int BN>
+cudaError_t launch_bn(const GemmArgs& g, cudaStream_t s) {
+  auto k = gemm_kernel<T, BN>;
+  const int smem = smem_for(BN);
+  static bool attr_set = false;  // per instantiation; set once per process
+  cudaError_t e;
+  if (!attr_set) {
+    if ((e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, smem)) != cudaSuccess)
+      return e;
+    attr_set = true;
+  }
+  const long long tiles = (long long)((g.M + BM - 1) / BM) * ((g.N + BN - 1) / BN) * g.k_splits;
+  k<<<(unsigned)tiles, 128, smem, s>>>(g);
+  return cudaGetLastError();
+}
+
+template <typename T>
+cudaError_t launch_t(const GemmArgs& g, cudaStream_t s) {
+  switch (g.bn) {
+    case 16: return launch_bn<T, 16>(g, s);
+    case 32: return launch_bn<T, 32>(g, s);
+    case 64: return launch_bn<T, 64>(g, s);
+    case 128: return launch_bn<T, 128>(g, s);
+    case 256: return launch_bn<T, 256>(g, s);
+    default: return cudaErrorInvalidValue;
+  }
+}
+
+}  // namespace
+
+int gemm_stages(int, int bn) { return stages_for(bn); }
+size_t gemm_smem_bytes(int, int bn) { return (size_t)smem_for(bn); }
+
+cudaError_t launch_gemm(const GemmArgs& g, cudaStream_t s) {
+  if (g.M <= 0 || g.N <= 0) return cudaSuccess;
+  return g.dtype == HDF_BF16 ? launch_t<__nv_bfloat16>(g, s) : launch_t<float>(g, s);
+}
+
+}  // namespace hdf

@@ -1,0 +1,642 @@
+// C ABI of libhdf (declared in include/hdf.h): host-side validation,
+// workspace layout, TMA tensor-map encoding and the launch sequence of one
+// block-drafting step.  Every computation runs in the CUDA kernels of this
+// library; nothing here touches tensor data on the host.
+#include <cudaTypedefs.h>
+
+#include <algorithm>
+#include <cmath>
+#include <cstdarg>
+#include <cstdio>
+#include <cstring>
+#include <string>
+
+#include "common.cuh"
+#include "kernels.h"
+
+using namespace hdf;
+
+namespace {
+
+thread_local std::string g_err;
+
+__device__ int g_device_status;  // HDF_ERR_DEVICE_CHECK after a bounded wait ran out
+
+int fail(int code, const char* fmt, ...) {
+  char buf[512];
+  va_list ap;
+  va_start(ap, fmt);
+  vsnprintf(buf, sizeof buf, fmt, ap);
+  va_end(ap);
+  g_err = buf;
+  return code;
+}
+int cuda_fail(cudaError_t e, const char* where) {
+  return fail(HDF_ERR_CUDA, "%s: %s", where, cudaGetErrorString(e));
+}
+#define CK(call, where)                              \
+  do {                                               \
+    cudaError_t e_ = (call);                         \
+    if (e_ != cudaSuccess) return cuda_fail(e_, where); \
+  } while (0)
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+size_t esize(int dtype) { return dtype == HDF_BF16 ? 2 : 4; }
+size_t up256(size_t x) { return (x + 255) & ~size_t(255); }
+
+int* device_status_ptr() {
+  static int* ptr[64] = {nullptr};
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return nullptr;
+  if (!ptr[dev]) {
+    void* p = nullptr;
+    if (cudaGetSymbolAddress(&p, g_device_status) != cudaSuccess) return nullptr;
+    ptr[dev] = static_cast<int*>(p);
+  }
+  return ptr[dev];
+}
+
+int num_sms() {
+  static int cache[64] = {0};
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return 148;
+  if (!cache[dev]) {
+    int n = 0;
+    cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev);
+    cache[dev] = n > 0 ? n : 148;
+  }
+  return cache[dev];
+}
+
+PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
+  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+  if (!fn) {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) ==
+            cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
+  }
+  return fn;
+}
+
+// 2-D K-major map over a [rows, cols] row-major tensor (row stride ld
+// elements), box {128 bytes of columns, box_rows}, 128-byte swizzle,
+// zero fill outside the tensor.
+int make_map(CUtensorMap* m, const void* ptr, int dtype, long long rows, long long cols, long long ld,
+             int box_rows) {
+  auto fn = encode_fn();
+  if (!fn) return fail(HDF_ERR_CUDA, "cuTensorMapEncodeTiled unavailable");
+  const size_t es = esize(dtype);
+  cuuint64_t dims[2] = {(cuuint64_t)cols, (cuuint64_t)std::max<long long>(rows, 1)};
+  cuuint64_t strides[1] = {(cuuint64_t)(ld * es)};
+  cuuint32_t box[2] = {(cuuint32_t)(128 / es), (cuuint32_t)box_rows};
+  cuuint32_t estr[2] = {1, 1};
+  CUresult r = fn(m, dtype == HDF_BF16 ? CU_TENSOR_MAP_DATA_TYPE_BFLOAT16 : CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 2,
+                  const_cast<void*>(ptr), dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                  CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  if (r != CUDA_SUCCESS)
+    return fail(HDF_ERR_CUDA, "cuTensorMapEncodeTiled failed (%d) rows=%lld cols=%lld box_rows=%d", (int)r, rows,
+                cols, box_rows);
+  return HDF_OK;
+}
+
+// ------------------------------------------------------------ GEMM plans
+int pick_bn(long long n) {
+  if (n <= 16) return 16;
+  if (n <= 32) return 32;
+  if (n <= 64) return 64;
+  if (n <= 128) return 128;
+  return 256;
+}
+
+struct SplitPlan {
+  int bn, k_splits, tiles;
+};
+
+// Weights-as-A GEMM (rows = output features, columns = tokens): K-split so
+// that about two CTAs per SM stream weights, each over >= 4 k-blocks.
+SplitPlan plan_swap(int dtype, long long M, long long N, long long K) {
+  SplitPlan p;
+  p.bn = pick_bn(N);
+  const int bk = dtype == HDF_BF16 ? 64 : 32;
+  p.tiles = (int)(((M + 127) / 128) * ((N + p.bn - 1) / p.bn));
+  const int num_kb = (int)((K + bk - 1) / bk);
+  const int target = 2 * num_sms();
+  int splits = std::max(1, (target + p.tiles - 1) / p.tiles);
+  splits = std::min(splits, std::max(1, num_kb / 4));
+  const int kb_per = (num_kb + splits - 1) / splits;
+  p.k_splits = (num_kb + kb_per - 1) / kb_per;
+  return p;
+}
+size_t split_ws_bytes(const SplitPlan& p) {
+  return p.k_splits > 1 ? (size_t)p.tiles * p.k_splits * 128 * p.bn * 4 : 0;
+}
+
+void init_gemm(GemmArgs& g, int dtype, long long M, long long N, long long K, const SplitPlan& p) {
+  std::memset(&g, 0, sizeof g);
+  g.M = (int)M;
+  g.N = (int)N;
+  g.K = (int)K;
+  g.dtype = dtype;
+  g.bn = p.bn;
+  g.k_splits = p.k_splits;
+  g.group_n = 1;
+  g.status = device_status_ptr();
+  g.A.rows_per_map = 1 << 30;
+  g.B.rows_per_map = 1 << 30;
+}
+
+// ---------------------------------------------------- draft-block layout
+struct DraftLayout {
+  size_t c, kc, vc, h, x, q, kb, vb, o, act, part_o, part_ml, split, counters, total;
+  int chunk, n_chunks;
+  SplitPlan qkv, oproj, gu, down;
+};
+
+int attn_chunk(const hdf_draft_shape* sh, int* n_chunks) {
+  const int per = std::max(1, (2 * num_sms() + sh->batch * sh->n_heads - 1) / (sh->batch * sh->n_heads));
+  int chunk = (sh->max_ctx + per - 1) / per;
+  chunk = std::max(256, ((chunk + 63) / 64) * 64);
+  *n_chunks = std::max(1, (sh->max_ctx + chunk - 1) / chunk);
+  return chunk;
+}
+
+DraftLayout draft_layout(const hdf_draft_shape* sh) {
+  DraftLayout L;
+  const size_t es = esize(sh->dtype);
+  const long long M = (long long)sh->batch * sh->block;
+  const long long d = sh->d, F = sh->ffn;
+  size_t off = 0;
+  auto take = [&](size_t bytes) {
+    const size_t o = off;
+    off += up256(bytes);
+    return o;
+  };
+  L.c = take(sh->n_ctx * d * es);
+  L.kc = take(sh->n_ctx * d * es);
+  L.vc = take(sh->n_ctx * d * es);
+  L.h = take(M * d * 4);
+  L.x = take(M * d * es);
+  L.q = take(M * d * es);
+  L.kb = take(M * d * es);
+  L.vb = take(M * d * es);
+  L.o = take(M * d * es);
+  L.act = take(M * F * es);
+  L.chunk = attn_chunk(sh, &L.n_chunks);
+  const size_t np = (size_t)sh->batch * sh->n_heads * L.n_chunks * sh->block;
+  L.part_o = take(np * sh->head_dim * 4);
+  L.part_ml = take(np * 2 * 4);
+  L.qkv = plan_swap(sh->dtype, 3 * d, M, d);
+  L.oproj = plan_swap(sh->dtype, d, M, d);
+  L.gu = plan_swap(sh->dtype, 2 * F, M, d);
+  L.down = plan_swap(sh->dtype, d, M, F);
+  size_t split = std::max(std::max(split_ws_bytes(L.qkv), split_ws_bytes(L.oproj)),
+                          std::max(split_ws_bytes(L.gu), split_ws_bytes(L.down)));
+  L.split = take(split);
+  const int tiles = std::max(std::max(L.qkv.tiles, L.oproj.tiles), std::max(L.gu.tiles, L.down.tiles));
+  L.counters = take((size_t)tiles * 4);
+  L.total = off;
+  return L;
+}
+
+int check_draft_shape(const hdf_draft_shape* sh) {
+  if (!sh) return fail(HDF_ERR_INVALID_ARG, "shape is NULL");
+  if (sh->dtype != HDF_BF16 && sh->dtype != HDF_F32) return fail(HDF_ERR_DTYPE, "dtype %d", sh->dtype);
+  if (sh->batch < 0 || sh->block < 2 || sh->block > 16)
+    return fail(HDF_ERR_SHAPE, "batch %d / block %d (need block in 2..16)", sh->batch, sh->block);
+  if (sh->d <= 0 || sh->d % 128) return fail(HDF_ERR_SHAPE, "d=%d must be a positive multiple of 128", sh->d);
+  if (sh->head_dim != 64 && sh->head_dim != 128) return fail(HDF_ERR_SHAPE, "head_dim %d", sh->head_dim);
+  if ((long long)sh->n_heads * sh->head_dim != sh->d) return fail(HDF_ERR_SHAPE, "n_heads*head_dim != d");
+  if (sh->ffn <= 0 || sh->ffn % 64) return fail(HDF_ERR_SHAPE, "ffn=%d must be a multiple of 64", sh->ffn);
+  if (sh->vocab <= 0 || sh->n_layers < 1) return fail(HDF_ERR_SHAPE, "vocab/n_layers");
+  if (sh->n_ctx < 0 || sh->max_ctx < 0 || sh->n_ctx > 0x7fffffffLL)
+    return fail(HDF_ERR_SHAPE, "n_ctx/max_ctx");
+  if ((long long)sh->batch * sh->block > 4096) return fail(HDF_ERR_UNSUPPORTED, "batch*block > 4096");
+  if (!(sh->norm_eps >= 0.f)) return fail(HDF_ERR_INVALID_ARG, "norm_eps");
+  return HDF_OK;
+}
+
+}  // namespace
+
+// =====================================================================
+extern "C" {
+
+int hdf_version(void) { return 100; }
+
+const char* hdf_status_str(int s) {
+  switch (s) {
+    case HDF_OK: return "ok";
+    case HDF_ERR_INVALID_ARG: return "invalid argument";
+    case HDF_ERR_SHAPE: return "unsupported or inconsistent shape";
+    case HDF_ERR_DTYPE: return "unknown dtype";
+    case HDF_ERR_ALIGNMENT: return "pointer not 16-byte aligned";
+    case HDF_ERR_WORKSPACE: return "workspace missing, misaligned or too small";
+    case HDF_ERR_CUDA: return "CUDA error";
+    case HDF_ERR_UNSUPPORTED: return "unsupported configuration";
+    case HDF_ERR_DEVICE_CHECK: return "device-side bounded wait expired";
+    default: return "unknown status";
+  }
+}
+
+const char* hdf_last_error(void) { return g_err.c_str(); }
+
+int hdf_device_status(int reset) {
+  CK(cudaDeviceSynchronize(), "cudaDeviceSynchronize");
+  int v = 0;
+  CK(cudaMemcpyFromSymbol(&v, g_device_status, sizeof v), "cudaMemcpyFromSymbol");
+  if (reset) {
+    const int z = 0;
+    CK(cudaMemcpyToSymbol(g_device_status, &z, sizeof z), "cudaMemcpyToSymbol");
+  }
+  return v;
+}
+
+// ------------------------------------------------------------- reducer
+int hdf_gated_reduce(const void* H, int dtype, int64_t n_tokens, int m, int d, const void* Wf, const float* b,
+                     float rms_eps, float gate_scale, float gate_offset, const void* path_norm_w,
+                     float path_norm_eps, const float* alpha_override, void* y, float* alpha_out,
+                     hdf_stream_t stream) {
+  g_err.clear();
+  if (dtype != HDF_BF16 && dtype != HDF_F32) return fail(HDF_ERR_DTYPE, "dtype %d", dtype);
+  if (n_tokens < 0) return fail(HDF_ERR_SHAPE, "n_tokens < 0");
+  if (!(m == 1 || m == 2 || m == 3 || m == 4 || m == 8)) return fail(HDF_ERR_UNSUPPORTED, "m=%d", m);
+  const int vec = dtype == HDF_BF16 ? 8 : 4;
+  if (d <= 0 || d % vec || d > 16384) return fail(HDF_ERR_SHAPE, "d=%d (multiple of %d, <= 16384)", d, vec);
+  if (n_tokens == 0) return HDF_OK;
+  if (!H || !y) return fail(HDF_ERR_INVALID_ARG, "H and y are required");
+  if (!alpha_override && (!Wf || !b)) return fail(HDF_ERR_INVALID_ARG, "Wf and b are required without override");
+  if (!aligned16(H) || !aligned16(y) || (Wf && !aligned16(Wf)) || (path_norm_w && !aligned16(path_norm_w)))
+    return fail(HDF_ERR_ALIGNMENT, "H, Wf, path_norm_w and y must be 16-byte aligned");
+  if (!std::isfinite(rms_eps) || !std::isfinite(gate_scale) || !std::isfinite(gate_offset) ||
+      !std::isfinite(path_norm_eps) || rms_eps < 0 || path_norm_eps < 0)
+    return fail(HDF_ERR_INVALID_ARG, "non-finite or negative scalar");
+  ReduceArgs a;
+  a.H = H;
+  a.Wf = Wf;
+  a.b = b;
+  a.path_norm_w = path_norm_w;
+  a.alpha_override = alpha_override;
+  a.y = y;
+  a.alpha_out = alpha_out;
+  a.n_tokens = n_tokens;
+  a.m = m;
+  a.d = d;
+  a.rms_eps = rms_eps;
+  a.gate_scale = gate_scale;
+  a.gate_offset = gate_offset;
+  a.path_norm_eps = path_norm_eps;
+  a.status = device_status_ptr();
+  CK(launch_gated_reduce(a, dtype, (cudaStream_t)stream), "gated_reduce launch");
+  return HDF_OK;
+}
+
+// -------------------------------------------------------- fc comparison
+size_t hdf_fc_reduce_workspace_size(int64_t, int, int, int) { return 0; }
+
+int hdf_fc_reduce(const void* H, int dtype, int64_t n_tokens, int m, int d, const void* W_fc, void* y, void*,
+                  size_t, hdf_stream_t stream) {
+  g_err.clear();
+  if (dtype != HDF_BF16 && dtype != HDF_F32) return fail(HDF_ERR_DTYPE, "dtype %d", dtype);
+  if (n_tokens < 0 || m < 1 || d <= 0 || d % 128) return fail(HDF_ERR_SHAPE, "need d %% 128 == 0");
+  if ((long long)m * d * esize(dtype) % 16) return fail(HDF_ERR_SHAPE, "row stride");
+  if (n_tokens == 0) return HDF_OK;
+  if (!H || !W_fc || !y) return fail(HDF_ERR_INVALID_ARG, "null pointer");
+  if (!aligned16(H) || !aligned16(W_fc) || !aligned16(y)) return fail(HDF_ERR_ALIGNMENT, "alignment");
+  if (n_tokens > 0x7fffffffLL) return fail(HDF_ERR_SHAPE, "n_tokens too large");
+  const long long K = (long long)m * d;
+  SplitPlan p{d % 256 == 0 ? 256 : 128, 1, 0};
+  GemmArgs g;
+  init_gemm(g, dtype, n_tokens, d, K, p);
+  g.group_n = 8;
+  int rc;
+  if ((rc = make_map(&g.A.map[0], H, dtype, n_tokens, K, K, 64))) return rc;
+  if ((rc = make_map(&g.B.map[0], W_fc, dtype, d, K, K, p.bn))) return rc;
+  g.epi.kind = kEpiStore;
+  g.epi.out[0] = y;
+  g.epi.seg_width = d;
+  g.epi.ld = d;
+  CK(launch_gemm(g, (cudaStream_t)stream), "fc gemm launch");
+  return HDF_OK;
+}
+
+// --------------------------------------------------------------- RoPE
+int hdf_rope_table(double theta, int head_dim, int64_t max_pos, float* cos_out, float* sin_out,
+                   hdf_stream_t stream) {
+  g_err.clear();
+  if (!(theta > 0) || head_dim <= 0 || head_dim % 2 || max_pos < 0)
+    return fail(HDF_ERR_INVALID_ARG, "theta/head_dim/max_pos");
+  if (max_pos == 0) return HDF_OK;
+  if (!cos_out || !sin_out) return fail(HDF_ERR_INVALID_ARG, "null output");
+  CK(launch_rope_table(theta, head_dim, max_pos, cos_out, sin_out, (cudaStream_t)stream), "rope launch");
+  return HDF_OK;
+}
+
+// --------------------------------------------------------- draft block
+size_t hdf_draft_block_workspace_size(const hdf_draft_shape* shape) {
+  if (check_draft_shape(shape) != HDF_OK) return 0;
+  return draft_layout(shape).total;
+}
+
+int hdf_draft_block(const hdf_drafter_weights* w, const hdf_draft_shape* sh, const void* ctx,
+                    const int32_t* cu_ctx, const int32_t* anchor, void* h_out, void* ws, size_t ws_bytes,
+                    const hdf_trace* trace, hdf_stream_t stream) {
+  g_err.clear();
+  int rc = check_draft_shape(sh);
+  if (rc) return rc;
+  if (!w || !w->layers) return fail(HDF_ERR_INVALID_ARG, "weights / layers NULL");
+  const int dt = sh->dtype;
+  const long long M = (long long)sh->batch * sh->block;
+  const long long d = sh->d, F = sh->ffn;
+  if (M == 0) return HDF_OK;
+  if (!cu_ctx || !anchor || !h_out || (sh->n_ctx > 0 && !ctx)) return fail(HDF_ERR_INVALID_ARG, "null input");
+  if (!w->embed || !w->mask_vec || !w->ctx_norm || !w->final_norm || !w->rope_cos || !w->rope_sin)
+    return fail(HDF_ERR_INVALID_ARG, "null weight");
+  if (w->rope_max_pos < (long long)sh->max_ctx + sh->block)
+    return fail(HDF_ERR_SHAPE, "rope_max_pos %lld < max_ctx + block", (long long)w->rope_max_pos);
+  const void* ptrs[] = {ctx, h_out, w->embed, w->mask_vec, w->ctx_norm, w->final_norm};
+  for (const void* p : ptrs)
+    if (p && !aligned16(p)) return fail(HDF_ERR_ALIGNMENT, "tensor not 16-byte aligned");
+  for (int l = 0; l < sh->n_layers; ++l) {
+    const hdf_layer_weights& L = w->layers[l];
+    const void* lp[] = {L.attn_norm, L.wq, L.wk, L.wv, L.wo, L.mlp_norm, L.wg, L.wu, L.wd};
+    for (const void* p : lp) {
+      if (!p) return fail(HDF_ERR_INVALID_ARG, "layer %d weight NULL", l);
+      if (!aligned16(p)) return fail(HDF_ERR_ALIGNMENT, "layer %d weight misaligned", l);
+    }
+  }
+  const DraftLayout Lo = draft_layout(sh);
+  if (!ws || ws_bytes < Lo.total || (reinterpret_cast<uintptr_t>(ws) & 255))
+    return fail(HDF_ERR_WORKSPACE, "workspace %zu bytes (need %zu, 256-byte aligned)", ws_bytes, Lo.total);
+  cudaStream_t s = (cudaStream_t)stream;
+  char* W = static_cast<char*>(ws);
+  void* c = W + Lo.c;
+  void* kc = W + Lo.kc;
+  void* vc = W + Lo.vc;
+  float* h = reinterpret_cast<float*>(W + Lo.h);
+  void* x = W + Lo.x;
+  void* q = W + Lo.q;
+  void* kbk = W + Lo.kb;
+  void* vbk = W + Lo.vb;
+  void* o = W + Lo.o;
+  void* act = W + Lo.act;
+  float* split = reinterpret_cast<float*>(W + Lo.split);
+  int* counters = reinterpret_cast<int*>(W + Lo.counters);
+
+  const int n_ev = trace ? trace->n_events : 0;
+  const int want_ev = 3 + HDF_DRAFT_STAGES_PER_LAYER * sh->n_layers;
+  if (trace && (!trace->events || n_ev != want_ev)) return fail(HDF_ERR_INVALID_ARG, "trace needs %d events", want_ev);
+  int ev_i = 0;
+  auto mark = [&]() -> int {
+    if (trace) CK(cudaEventRecord((cudaEvent_t)trace->events[ev_i++], s), "cudaEventRecord");
+    return HDF_OK;
+  };
+
+  CK(cudaMemsetAsync(counters, 0, up256((size_t)std::max({Lo.qkv.tiles, Lo.oproj.tiles, Lo.gu.tiles, Lo.down.tiles}) * 4), s),
+     "memset counters");
+  // ---- context RMSNorm
+  if ((rc = mark())) return rc;
+  CK(launch_rmsnorm(ctx, 0, w->ctx_norm, c, dt, sh->n_ctx, (int)d, sh->norm_eps, s), "ctx norm");
+
+  for (int l = 0; l < sh->n_layers; ++l) {
+    const hdf_layer_weights& Lw = w->layers[l];
+    // ---- conditioning projection: [K_c | V_c] = c [W_k; W_v]^T, RoPE on K_c
+    if ((rc = mark())) return rc;
+    if (sh->n_ctx > 0) {
+      SplitPlan p{d % 256 == 0 ? 256 : 128, 1, 0};
+      GemmArgs g;
+      init_gemm(g, dt, sh->n_ctx, 2 * d, d, p);
+      g.group_n = 8;
+      if ((rc = make_map(&g.A.map[0], c, dt, sh->n_ctx, d, d, 64))) return rc;
+      if ((rc = make_map(&g.B.map[0], Lw.wk, dt, d, d, d, p.bn))) return rc;
+      if ((rc = make_map(&g.B.map[1], Lw.wv, dt, d, d, d, p.bn))) return rc;
+      g.B.rows_per_map = (int)d;
+      g.epi.kind = kEpiStore;
+      g.epi.out[0] = kc;
+      g.epi.out[1] = vc;
+      g.epi.seg_width = (int)d;
+      g.epi.ld = d;
+      g.epi.rope_mask = 1;
+      g.epi.rope_cos = w->rope_cos;
+      g.epi.rope_sin = w->rope_sin;
+      g.epi.rope_rows = w->rope_max_pos;
+      g.epi.head_dim = sh->head_dim;
+      g.epi.cu_ctx = cu_ctx;
+      g.epi.batch = sh->batch;
+      g.epi.block = sh->block;
+      g.epi.pos_mode = 1;
+      CK(launch_gemm(g, s), "ctx kv gemm");
+    }
+    // ---- block input / attention norm
+    if ((rc = mark())) return rc;
+    if (l == 0)
+      CK(launch_embed_norm(w->embed, w->mask_vec, anchor, Lw.attn_norm, h, x, dt, sh->batch, sh->block, (int)d,
+                           sh->vocab, sh->norm_eps, s),
+         "embed norm");
+    else
+      CK(launch_rmsnorm(h, 1, Lw.attn_norm, x, dt, M, (int)d, sh->norm_eps, s), "attn norm");
+    // ---- Q / K_b / V_b with RoPE at block positions
+    if ((rc = mark())) return rc;
+    {
+      GemmArgs g;
+      init_gemm(g, dt, 3 * d, M, d, Lo.qkv);
+      if ((rc = make_map(&g.A.map[0], Lw.wq, dt, d, d, d, 64))) return rc;
+      if ((rc = make_map(&g.A.map[1], Lw.wk, dt, d, d, d, 64))) return rc;
+      if ((rc = make_map(&g.A.map[2], Lw.wv, dt, d, d, d, 64))) return rc;
+      g.A.rows_per_map = (int)d;
+      if ((rc = make_map(&g.B.map[0], x, dt, M, d, d, Lo.qkv.bn))) return rc;
+      g.ws_partial = split;
+      g.counters = counters;
+      g.epi.kind = kEpiStoreT;
+      g.epi.out[0] = q;
+      g.epi.out[1] = kbk;
+      g.epi.out[2] = vbk;
+      g.epi.seg_width = (int)d;
+      g.epi.ld = d;
+      g.epi.rope_mask = 3;
+      g.epi.rope_cos = w->rope_cos;
+      g.epi.rope_sin = w->rope_sin;
+      g.epi.rope_rows = w->rope_max_pos;
+      g.epi.head_dim = sh->head_dim;
+      g.epi.cu_ctx = cu_ctx;
+      g.epi.batch = sh->batch;
+      g.epi.block = sh->block;
+      g.epi.pos_mode = 2;
+      CK(launch_gemm(g, s), "qkv gemm");
+    }
+    // ---- attention over [K_c; K_b]
+    if ((rc = mark())) return rc;
+    {
+      AttnArgs a;
+      std::memset(&a, 0, sizeof a);
+      a.q = q;
+      a.kb = kbk;
+      a.vb = vbk;
+      a.kc = kc;
+      a.vc = vc;
+      a.cu_ctx = cu_ctx;
+      a.out = o;
+      a.part_o = reinterpret_cast<float*>(W + Lo.part_o);
+      a.part_ml = reinterpret_cast<float*>(W + Lo.part_ml);
+      a.batch = sh->batch;
+      a.block = sh->block;
+      a.n_heads = sh->n_heads;
+      a.head_dim = sh->head_dim;
+      a.d = (int)d;
+      a.n_ctx = sh->n_ctx;
+      a.chunk = Lo.chunk;
+      a.n_chunks = Lo.n_chunks;
+      a.status = device_status_ptr();
+      AttnTmaps tm;
+      if (dt == HDF_BF16) {
+        const void* kc_src = sh->n_ctx > 0 ? kc : kbk;
+        const void* vc_src = sh->n_ctx > 0 ? vc : vbk;
+        const long long rows = sh->n_ctx > 0 ? sh->n_ctx : M;
+        if ((rc = make_map(&tm.k, kc_src, dt, rows, d, d, 64))) return rc;
+        if ((rc = make_map(&tm.v, vc_src, dt, rows, d, d, 64))) return rc;
+        if ((rc = make_map(&tm.kb, kbk, dt, M, d, d, 64))) return rc;
+        if ((rc = make_map(&tm.vb, vbk, dt, M, d, d, 64))) return rc;
+      }
+      CK(launch_attention(a, &tm, dt, s), "attention");
+    }
+    // ---- h += O W_o^T
+    if ((rc = mark())) return rc;
+    {
+      GemmArgs g;
+      init_gemm(g, dt, d, M, d, Lo.oproj);
+      if ((rc = make_map(&g.A.map[0], Lw.wo, dt, d, d, d, 64))) return rc;
+      if ((rc = make_map(&g.B.map[0], o, dt, M, d, d, Lo.oproj.bn))) return rc;
+      g.ws_partial = split;
+      g.counters = counters;
+      g.epi.kind = kEpiResidT;
+      g.epi.resid = h;
+      g.epi.ld = d;
+      CK(launch_gemm(g, s), "o gemm");
+    }
+    // ---- MLP norm
+    if ((rc = mark())) return rc;
+    CK(launch_rmsnorm(h, 1, Lw.mlp_norm, x, dt, M, (int)d, sh->norm_eps, s), "mlp norm");
+    // ---- act = silu(x W_g^T) * (x W_u^T)
+    if ((rc = mark())) return rc;
+    {
+      GemmArgs g;
+      init_gemm(g, dt, 2 * F, M, d, Lo.gu);
+      if ((rc = make_map(&g.A.map[0], Lw.wg, dt, F, d, d, 64))) return rc;
+      if ((rc = make_map(&g.A.map[1], Lw.wu, dt, F, d, d, 64))) return rc;
+      g.A.mode = kPair64;
+      if ((rc = make_map(&g.B.map[0], x, dt, M, d, d, Lo.gu.bn))) return rc;
+      g.ws_partial = split;
+      g.counters = counters;
+      g.epi.kind = kEpiSwigluT;
+      g.epi.out[0] = act;
+      g.epi.seg_width = (int)F;
+      g.epi.ld = F;
+      CK(launch_gemm(g, s), "gate/up gemm");
+    }
+    // ---- h += act W_d^T
+    if ((rc = mark())) return rc;
+    {
+      GemmArgs g;
+      init_gemm(g, dt, d, M, F, Lo.down);
+      if ((rc = make_map(&g.A.map[0], Lw.wd, dt, d, F, F, 64))) return rc;
+      if ((rc = make_map(&g.B.map[0], act, dt, M, F, F, Lo.down.bn))) return rc;
+      g.ws_partial = split;
+      g.counters = counters;
+      g.epi.kind = kEpiResidT;
+      g.epi.resid = h;
+      g.epi.ld = d;
+      CK(launch_gemm(g, s), "down gemm");
+    }
+  }
+  // ---- final norm
+  if ((rc = mark())) return rc;
+  CK(launch_rmsnorm(h, 1, w->final_norm, h_out, dt, M, (int)d, sh->norm_eps, s), "final norm");
+  if ((rc = mark())) return rc;
+  return HDF_OK;
+}
+
+// -------------------------------------------------------------- LM head
+namespace {
+struct LmLayout {
+  SplitPlan p;
+  int tiles_m;
+  size_t pmax, parg, psum, split, counters, total;
+};
+LmLayout lm_layout(int64_t M, int64_t V, int dtype, int d) {
+  LmLayout L;
+  L.p = plan_swap(dtype, V, M, d);
+  L.tiles_m = (int)((V + 127) / 128);
+  size_t off = 0;
+  auto take = [&](size_t b) {
+    const size_t o = off;
+    off += up256(b);
+    return o;
+  };
+  L.pmax = take((size_t)L.tiles_m * M * 4);
+  L.parg = take((size_t)L.tiles_m * M * 4);
+  L.psum = take((size_t)L.tiles_m * M * 4);
+  L.split = take(split_ws_bytes(L.p));
+  L.counters = take((size_t)L.p.tiles * 4);
+  L.total = off;
+  return L;
+}
+}  // namespace
+
+size_t hdf_lm_head_workspace_size(int64_t M, int d, int64_t V, int dtype) {
+  if (M <= 0 || V <= 0 || d <= 0) return 0;
+  return lm_layout(M, V, dtype, d).total;
+}
+
+int hdf_lm_head_argmax(const void* h, int dtype, int64_t M, int d, const void* W_lm, int64_t V, float inv_temp,
+                       int32_t* tok, float* zmax, float* logsoftmax, void* ws, size_t ws_bytes,
+                       hdf_stream_t stream) {
+  g_err.clear();
+  if (dtype != HDF_BF16 && dtype != HDF_F32) return fail(HDF_ERR_DTYPE, "dtype %d", dtype);
+  if (M < 0 || V <= 0 || d <= 0 || d > 65536 || V > 0x7fffffffLL || M > 0x7fffffffLL)
+    return fail(HDF_ERR_SHAPE, "M/V/d");
+  if ((d * esize(dtype)) % 16) return fail(HDF_ERR_SHAPE, "d row stride must be a multiple of 16 bytes");
+  if (!(inv_temp > 0) || !std::isfinite(inv_temp)) return fail(HDF_ERR_INVALID_ARG, "inv_temp must be > 0");
+  if (M == 0) return HDF_OK;
+  if (!h || !W_lm || !tok) return fail(HDF_ERR_INVALID_ARG, "null pointer");
+  if (!aligned16(h) || !aligned16(W_lm)) return fail(HDF_ERR_ALIGNMENT, "h / W_lm alignment");
+  const LmLayout L = lm_layout(M, V, dtype, d);
+  if (!ws || ws_bytes < L.total || (reinterpret_cast<uintptr_t>(ws) & 255))
+    return fail(HDF_ERR_WORKSPACE, "workspace %zu bytes (need %zu, 256-byte aligned)", ws_bytes, L.total);
+  cudaStream_t s = (cudaStream_t)stream;
+  char* W = static_cast<char*>(ws);
+  GemmArgs g;
+  init_gemm(g, dtype, V, M, d, L.p);
+  int rc;
+  if ((rc = make_map(&g.A.map[0], W_lm, dtype, V, d, d, 64))) return rc;
+  if ((rc = make_map(&g.B.map[0], h, dtype, M, d, d, L.p.bn))) return rc;
+  g.ws_partial = reinterpret_cast<float*>(W + L.split);
+  g.counters = reinterpret_cast<int*>(W + L.counters);
+  g.epi.kind = kEpiLmHeadT;
+  g.epi.inv_temp = inv_temp;
+  g.epi.logsoftmax = logsoftmax;
+  g.epi.part_max = reinterpret_cast<float*>(W + L.pmax);
+  g.epi.part_arg = reinterpret_cast<int*>(W + L.parg);
+  g.epi.part_sum = reinterpret_cast<float*>(W + L.psum);
+  CK(cudaMemsetAsync(g.counters, 0, (size_t)L.p.tiles * 4, s), "memset counters");
+  CK(launch_gemm(g, s), "lm head gemm");
+  CK(launch_lm_reduce(g.epi.part_max, g.epi.part_arg, g.epi.part_sum, L.tiles_m, M, V, inv_temp, tok, zmax,
+                      logsoftmax, s),
+     "lm reduce");
+  return HDF_OK;
+}
+
+// -------------------------------------------------------------- verify
+int hdf_accept_len(const int32_t* draft, int64_t draft_stride, const int32_t* target, int64_t target_stride,
+                   int batch, int n_draft, int32_t* accept, hdf_stream_t stream) {
+  g_err.clear();
+  if (batch < 0 || n_draft < 0) return fail(HDF_ERR_SHAPE, "batch/n_draft");
+  if (batch == 0) return HDF_OK;
+  if (!draft || !target || !accept) return fail(HDF_ERR_INVALID_ARG, "null pointer");
+  if (draft_stride < n_draft || target_stride < n_draft) return fail(HDF_ERR_SHAPE, "stride < n_draft");
+  CK(launch_accept(draft, draft_stride, target, target_stride, batch, n_draft, accept, (cudaStream_t)stream),
+     "accept launch");
+  return HDF_OK;
+}
+
+}  // extern "C"

@@ -1,0 +1,126 @@
+// Host-side launch interfaces of the CUDA kernels (internal to libhdf).
+#pragma once
+
+#include <cuda.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+namespace hdf {
+
+// ------------------------------------------------------------ reducer ----
+struct ReduceArgs {
+  const void* H;
+  const void* Wf;
+  const float* b;
+  const void* path_norm_w;
+  const float* alpha_override;
+  void* y;
+  float* alpha_out;
+  long long n_tokens;
+  int m, d;
+  float rms_eps, gate_scale, gate_offset, path_norm_eps;
+  int* status;
+};
+cudaError_t launch_gated_reduce(const ReduceArgs& a, int dtype, cudaStream_t s);
+
+// --------------------------------------------------------------- GEMM ----
+// D[M, N] = A[M, K] * B[N, K]^T, both operands K-major, loaded by TMA with
+// 128-byte swizzle.  An operand may be the row-concatenation of up to three
+// tensors (one tensor map each), or (A only) a "pair" whose 64-row halves of
+// each 128-row tile come from two tensors at the same row offset.
+enum OperandMode { kConcat = 0, kPair64 = 1 };
+
+struct Operand {
+  CUtensorMap map[3];
+  int rows_per_map;  // kConcat: rows covered by each map (tile-aligned)
+  int mode;
+};
+
+enum EpiKind {
+  kEpiStore = 0,    // rows = tokens, cols = features -> out[seg][row, col]
+  kEpiStoreT = 1,   // rows = features, cols = tokens -> out[seg][col, row]
+  kEpiResidT = 2,   // resid[col, row] += D  (fp32 residual)
+  kEpiSwigluT = 3,  // pair tile: act[col, f] = silu(g) * u
+  kEpiLmHeadT = 4,  // rows = vocab, cols = tokens: argmax / sum-exp partials
+};
+
+struct Epilogue {
+  int kind;
+  void* out[3];         // segment outputs (dtype of the GEMM)
+  int seg_width;        // features per segment
+  long long ld;         // row stride of out[] / resid / act, elements
+  int rope_mask;        // bit s: RoPE on segment s
+  const float* rope_cos;
+  const float* rope_sin;
+  long long rope_rows;  // positions >= rope_rows are clamped (contract violation)
+  int head_dim;
+  const int* cu_ctx;    // positions: context rows -> t - cu[b]
+  int batch;
+  int block;            // block rows: pos = T_b + (j % block)
+  int pos_mode;         // 0 none, 1 context rows, 2 block rows
+  float* resid;         // kEpiResidT
+  // kEpiLmHeadT
+  float inv_temp;
+  float* logsoftmax;    // [N, M] fp32 or null (stored transposed: token-major)
+  float* part_max;      // [tiles_m, N]
+  int* part_arg;
+  float* part_sum;
+};
+
+struct GemmArgs {
+  Operand A, B;
+  int M, N, K;
+  int dtype;            // HDF_BF16 or HDF_F32 (tf32)
+  int bn;               // tile width along N: 16, 32, 64, 128 or 256
+  int k_splits;         // >= 1; >1 needs ws_partial / counters
+  float* ws_partial;    // [tiles, k_splits, 128, bn] fp32
+  int* counters;        // [tiles], zero on entry, left zero on exit
+  int group_n;          // raster: n-tiles swept together
+  Epilogue epi;
+  int* status;
+};
+cudaError_t launch_gemm(const GemmArgs& g, cudaStream_t s);
+int gemm_stages(int dtype, int bn);
+size_t gemm_smem_bytes(int dtype, int bn);
+
+// ----------------------------------------------------- small kernels ----
+cudaError_t launch_rope_table(double theta, int head_dim, long long max_pos, float* c, float* s,
+                              cudaStream_t st);
+// y[r] = RMSNorm_w(x[r]) for rows r; x fp32 or dtype, y dtype.
+cudaError_t launch_rmsnorm(const void* x, int x_is_f32, const void* w, void* y, int dtype,
+                           long long rows, int d, float eps, cudaStream_t s);
+// h[i*B + 0] = embed[anchor[i]], h[i*B + k] = mask_vec; x = RMSNorm(h).
+cudaError_t launch_embed_norm(const void* embed, const void* mask_vec, const int* anchor,
+                              const void* norm_w, float* h, void* x, int dtype, int batch,
+                              int block, int d, int vocab, float eps, cudaStream_t s);
+cudaError_t launch_accept(const int* draft, long long ds, const int* target, long long ts,
+                          int batch, int nd, int* accept, cudaStream_t s);
+cudaError_t launch_lm_reduce(const float* part_max, const int* part_arg, const float* part_sum,
+                             int tiles, long long M, long long V, float inv_temp, int* tok,
+                             float* zmax, float* logsoftmax, cudaStream_t s);
+
+// -------------------------------------------------------- attention ----
+struct AttnArgs {
+  const void* q;       // [M, d]  block queries (M = batch * block)
+  const void* kb;      // [M, d]  block keys
+  const void* vb;      // [M, d]
+  const void* kc;      // [n_ctx, d] context keys
+  const void* vc;      // [n_ctx, d]
+  const int* cu_ctx;   // [batch + 1]
+  void* out;           // [M, d]
+  float* part_o;       // [batch, heads, chunks, block, hd]
+  float* part_ml;      // [batch, heads, chunks, block, 2]
+  int batch, block, n_heads, head_dim, d;
+  long long n_ctx;
+  int chunk;           // context keys per split
+  int n_chunks;        // splits per (sequence, head) = ceil(max_ctx / chunk) (>= 1)
+  int* status;
+};
+// bf16 path: TMA maps over context K/V and block K/V, box {64 cols, 64 rows}
+struct AttnTmaps {
+  CUtensorMap k, v, kb, vb;
+};
+cudaError_t launch_attention(const AttnArgs& a, const AttnTmaps* tm, int dtype, cudaStream_t s);
+size_t attention_smem_bytes(int head_dim);
+
+}  // namespace hdf

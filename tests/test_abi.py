@@ -1,0 +1,72 @@
+"""The C-ABI library loads without a GPU, exports every entry point that
+include/hdf.h declares, and rejects bad arguments on the host before any
+CUDA call (these calls return before touching the device)."""
+import ctypes
+
+import pytest
+
+from paper_2606_26744_gb300 import build, hdf
+
+
+@pytest.fixture(scope="module")
+def lib():
+    build.build()
+    return hdf.load()
+
+
+def test_every_declared_symbol_is_exported(lib):
+    names = hdf.declared_functions()
+    assert len(names) >= 13
+    for n in ("hdf_gated_reduce", "hdf_draft_block", "hdf_lm_head_argmax", "hdf_accept_len"):
+        assert n in names
+    for n in names:
+        assert hasattr(lib, n), n
+    # the binding declares exactly the header's functions
+    assert set(hdf._SIGS) == set(names)
+
+
+def test_status_strings(lib):
+    assert lib.hdf_version() == 100
+    assert lib.hdf_status_str(0) == b"ok"
+    assert b"aligned" in lib.hdf_status_str(4)
+
+
+def _reduce(lib, **kw):
+    a = dict(H=16, dtype=1, n=4, m=4, d=64, Wf=16, b=16, y=16)
+    a.update(kw)
+    p = lambda v: None if v is None else ctypes.c_void_p(v)
+    return lib.hdf_gated_reduce(p(a["H"]), a["dtype"], a["n"], a["m"], a["d"], p(a["Wf"]), p(a["b"]),
+                                1e-6, 1.0, 0.0, None, 1e-6, None, p(a["y"]), None, None)
+
+
+def test_reduce_host_validation(lib):
+    assert _reduce(lib, dtype=7) == 3                 # HDF_ERR_DTYPE
+    assert _reduce(lib, m=5) == 7                     # HDF_ERR_UNSUPPORTED
+    assert _reduce(lib, d=60) == 2                    # d % 8 for bf16
+    assert _reduce(lib, n=-1) == 2
+    assert _reduce(lib, n=0) == 0                     # empty: nothing launched
+    assert _reduce(lib, H=None) == 1                  # HDF_ERR_INVALID_ARG
+    assert _reduce(lib, Wf=None) == 1                 # gate weight required without override
+    assert _reduce(lib, H=24) == 4                    # HDF_ERR_ALIGNMENT
+    assert b"aligned" in lib.hdf_last_error()
+
+
+def test_lm_head_and_accept_host_validation(lib):
+    v = ctypes.c_void_p
+    assert lib.hdf_lm_head_argmax(v(16), 9, 4, 64, v(16), 100, 1.0, v(16), None, None, v(256), 1 << 20, None) == 3
+    assert lib.hdf_lm_head_argmax(v(16), 1, 4, 64, v(16), 100, 0.0, v(16), None, None, v(256), 1 << 20, None) == 1
+    assert lib.hdf_lm_head_argmax(v(16), 1, 4, 60, v(16), 100, 1.0, v(16), None, None, v(256), 1 << 20, None) == 2
+    assert lib.hdf_accept_len(v(16), 3, v(16), 7, 2, 7, v(16), None) == 2   # stride < n_draft
+    assert lib.hdf_accept_len(None, 7, v(16), 7, 2, 7, v(16), None) == 1
+    assert lib.hdf_accept_len(None, 7, None, 7, 0, 7, None, None) == 0      # empty batch
+
+
+def test_draft_block_host_validation(lib):
+    sh = hdf.DraftShape(1, 1, 16, 2048, 16, 128, 8192, 32768, 1, 2048, 2048, 1e-6)
+    w = hdf.DrafterWeights()
+    bad = hdf.DraftShape(1, 1, 40, 2048, 16, 128, 8192, 32768, 1, 2048, 2048, 1e-6)   # block > 16
+    assert lib.hdf_draft_block(ctypes.byref(w), ctypes.byref(bad), None, None, None, None, None, 0, None, None) == 2
+    bad2 = hdf.DraftShape(1, 1, 16, 2000, 16, 125, 8192, 32768, 1, 2048, 2048, 1e-6)  # d % 128
+    assert lib.hdf_draft_block(ctypes.byref(w), ctypes.byref(bad2), None, None, None, None, None, 0, None, None) == 2
+    assert lib.hdf_draft_block(None, ctypes.byref(sh), None, None, None, None, None, 0, None, None) == 1
+    assert lib.hdf_draft_block_workspace_size(ctypes.byref(bad)) == 0

@@ -1,0 +1,122 @@
+"""End-to-end parity of one block-drafting step with the fp64 oracle:
+gated reduce (Eq. 1) -> drafter block -> LM head argmax -> accepted length.
+
+The decode workload (m4 d2048 T2048 B16, 16x128 heads, F8192, V32768) is the
+one bench.py times and is checked in full.  The wider workloads run with
+their full model widths but short ragged contexts, so the oracle finishes
+in seconds; their full-context kernels are covered by the sampled-row tests
+of the reducer, GEMM and LM head."""
+import numpy as np
+import pytest
+import torch
+
+import oracle as O
+from paper_2606_26744_gb300 import hdf
+from paper_2606_26744_gb300 import workloads as W
+from _util import TOL_BF16, TOL_F32_REDUCE, TOL_F32_TF32, check_tokens, rowwise_rel, to64
+
+pytestmark = pytest.mark.gpu
+
+
+def _weights64(w):
+    out = {k: to64(v) for k, v in w.items() if k != "layers"}
+    out["layers"] = [{k: to64(v) for k, v in lw.items()} for lw in w["layers"]]
+    return out
+
+
+def _to_cuda(w):
+    out = {k: v.cuda() for k, v in w.items() if k != "layers"}
+    out["layers"] = [{k: v.cuda() for k, v in lw.items()} for lw in w["layers"]]
+    return out
+
+
+def run_step(cfg, seed, ctx_lens=None):
+    if ctx_lens is not None:
+        cfg = W.scaled(cfg, batch=len(ctx_lens), ctx_len=max(ctx_lens) if ctx_lens else 0)
+    inp = W.make_draft_inputs(cfg, seed)
+    if ctx_lens is not None:  # explicit ragged lengths for this case
+        cu = np.concatenate([[0], np.cumsum(ctx_lens)]).astype(np.int32)
+        inp = dict(inp)
+        inp["ctx_lens"] = list(ctx_lens)
+        inp["cu_ctx"] = torch.tensor(cu)
+        red = W.make_reduce_inputs(int(cu[-1]), cfg.m, cfg.d, cfg.dtype, cfg.wf_std, seed=seed)
+        inp.update(red)
+    lens = inp["ctx_lens"]
+    max_ctx = max(lens) if lens else 0
+    act = cfg.dtype
+
+    # ---------------- GPU path (C ABI through the binding)
+    wc = _to_cuda(inp["weights"])
+    drafter = hdf.Drafter(wc, n_heads=cfg.n_heads, head_dim=cfg.head_dim, rope_theta=cfg.rope_theta,
+                          rope_max_pos=max_ctx + cfg.block, norm_eps=cfg.norm_eps)
+    H = inp["H"].cuda()
+    y = hdf.hdf_gated_reduce(H, inp["Wf"].cuda(), inp["b"].cuda())
+    cu = inp["cu_ctx"].cuda()
+    anchor = inp["anchor"].cuda()
+    h = drafter.hdf_draft_block(y, cu, anchor, block=cfg.block, max_ctx=max_ctx)
+    tok, zmax, ls = hdf.hdf_lm_head_argmax(h, wc["lm_head"], logsoftmax=cfg.logsoftmax)
+    torch.cuda.synchronize()
+    assert hdf.device_status() == 0
+
+    # ---------------- oracle
+    w64 = _weights64(inp["weights"])
+    y_ref, _ = O.gated_reduce(to64(inp["H"]), to64(inp["Wf"]), to64(inp["b"]), out_dtype=act)
+    h_ref = O.draft_block(w64, y_ref, inp["cu_ctx"].tolist(), inp["anchor"].tolist(), block=cfg.block,
+                          n_heads=cfg.n_heads, head_dim=cfg.head_dim, rope_theta=cfg.rope_theta,
+                          norm_eps=cfg.norm_eps, act_dtype=act)
+    lm = O.lm_head(h_ref, w64["lm_head"], logsoftmax=cfg.logsoftmax)
+
+    tol_red = TOL_F32_REDUCE if act == "f32" else TOL_BF16
+    tol = TOL_F32_TF32 if act == "f32" else TOL_BF16
+    if y_ref.shape[0]:
+        assert rowwise_rel(to64(y), y_ref) <= tol_red
+    err_h = rowwise_rel(to64(h), h_ref)
+    assert err_h <= tol, f"h_out row-normwise error {err_h}"
+    ties = check_tokens(tok.cpu().numpy(), lm["z"])
+    if cfg.logsoftmax:
+        assert rowwise_rel(to64(ls), lm["logsoftmax"]) <= tol
+
+    # ---------------- verification against targets built from the oracle drafts
+    B = cfg.block
+    batch = cfg.batch
+    plan = W.accept_plan(cfg, seed)
+    d_ref = O.draft_tokens(lm["tok"], batch, B)
+    tgt = W.make_targets(torch.from_numpy(d_ref), plan, cfg.vocab, seed)
+    acc = hdf.hdf_accept_len(tok[1:], tgt.cuda(), n_draft=B - 1, draft_stride=B, batch=batch)
+    d_gpu = tok.cpu().numpy().reshape(batch, B)[:, 1:]
+    assert np.array_equal(acc.cpu().numpy(), O.accept_len(d_gpu, tgt.numpy()))
+    assert np.array_equal(O.accept_len(d_ref, tgt.numpy()), np.array(plan))
+    if ties == 0:
+        assert np.array_equal(acc.cpu().numpy(), np.array(plan))
+    return err_h, ties
+
+
+def test_tiny_workload_fp32():
+    run_step(W.CONFIGS["tiny"], seed=1000)
+
+
+def test_decode_workload_full():
+    """The decode workload exactly as bench.py runs it."""
+    run_step(W.CONFIGS["decode"], seed=1001)
+
+
+def test_ragged_multisequence_two_layers():
+    cfg = W.DraftConfig("ragged", m=4, d=512, block=16, n_layers=2, n_heads=4, head_dim=128, ffn=1024,
+                        vocab=4096, batch=5, ctx_len=300)
+    run_step(cfg, seed=7, ctx_lens=[0, 1, 63, 65, 300])
+
+
+def test_head_dim_64_short_block():
+    cfg = W.DraftConfig("hd64", m=4, d=256, block=8, n_layers=1, n_heads=4, head_dim=64, ffn=512,
+                        vocab=2048, batch=3, ctx_len=257)
+    run_step(cfg, seed=8, ctx_lens=[10, 130, 257])
+
+
+def test_serve_widths_short_ragged_context():
+    cfg = W.scaled(W.CONFIGS["serve"], vocab=8192, ctx_len_range=None)
+    run_step(cfg, seed=9, ctx_lens=[512, 700, 33, 1024])
+
+
+def test_large_widths_short_context():
+    cfg = W.scaled(W.CONFIGS["large"], vocab=8192, n_layers=1)
+    run_step(cfg, seed=10, ctx_lens=[300, 129])

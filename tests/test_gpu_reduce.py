@@ -1,0 +1,99 @@
+"""Parity of the gated reducer (Eq. 1) kernel with the fp64 oracle."""
+import numpy as np
+import pytest
+import torch
+
+import oracle as O
+from paper_2606_26744_gb300 import hdf
+from paper_2606_26744_gb300 import workloads as W
+from _util import TOL_BF16, TOL_F32_REDUCE, exact_fraction, rowwise_rel, to64
+
+pytestmark = pytest.mark.gpu
+
+
+def _run(inp, **kw):
+    H = inp["H"].cuda()
+    N, m, d = H.shape
+    a = torch.full((N, m), -7.0, device="cuda")
+    y = hdf.hdf_gated_reduce(H, inp["Wf"].cuda(), inp["b"].cuda(), alpha_out=a, **kw)
+    torch.cuda.synchronize()
+    assert hdf.device_status() == 0
+    return y.cpu(), a.cpu()
+
+
+@pytest.mark.parametrize("N,m,d,dtype,std", [
+    (64, 4, 256, "f32", 0.02),      # tiny workload
+    (37, 4, 2048, "bf16", 0.1),     # decode width, ragged token count
+    (5, 4, 7168, "bf16", 0.1),      # large width: W_f read through L1
+    (130, 2, 512, "bf16", 0.1),
+    (9, 8, 256, "bf16", 0.1),
+    (7, 3, 128, "f32", 0.1),
+    (1, 4, 4096, "bf16", 0.1),
+    (3, 1, 64, "bf16", 0.1),
+])
+def test_reduce_parity(N, m, d, dtype, std):
+    inp = W.make_reduce_inputs(N, m, d, dtype, std, seed=N * 131 + d)
+    y, a = _run(inp)
+    y_ref, a_ref = O.gated_reduce(to64(inp["H"]), to64(inp["Wf"]), to64(inp["b"]), out_dtype=dtype)
+    tol = TOL_F32_REDUCE if dtype == "f32" else TOL_BF16
+    assert rowwise_rel(to64(y), y_ref) <= tol
+    np.testing.assert_allclose(to64(a), a_ref, rtol=0, atol=1e-4)
+    if dtype == "bf16":
+        assert exact_fraction(to64(y), y_ref) >= 0.99
+
+
+def test_reduce_scale_offset_and_path_norm():
+    N, m, d = 33, 4, 1024
+    inp = W.make_reduce_inputs(N, m, d, "bf16", 0.1, seed=5)
+    g = torch.Generator().manual_seed(9)
+    pnw = (1 + 0.1 * torch.randn(m, d, generator=g)).to(torch.bfloat16)
+    y, a = _run(inp, gate_scale=0.7, gate_offset=0.05, rms_eps=1e-3, path_norm_w=pnw.cuda(),
+                path_norm_eps=1e-5)
+    y_ref, a_ref = O.gated_reduce(to64(inp["H"]), to64(inp["Wf"]), to64(inp["b"]), rms_eps=1e-3,
+                                  gate_scale=0.7, gate_offset=0.05, path_norm_w=to64(pnw),
+                                  path_norm_eps=1e-5, out_dtype="bf16")
+    assert rowwise_rel(to64(y), y_ref) <= TOL_BF16
+    np.testing.assert_allclose(to64(a), a_ref, atol=1e-4)
+
+
+def test_reduce_m1_identity_bit_exact():
+    inp = W.make_reduce_inputs(19, 1, 512, "bf16", 0.1, seed=3)
+    H = inp["H"].cuda()
+    y = hdf.hdf_gated_reduce(H, None, None, alpha_override=torch.ones(19, 1, device="cuda"))
+    assert torch.equal(y, H[:, 0, :])
+
+
+def test_reduce_one_hot_selects_path_bit_exact():
+    inp = W.make_reduce_inputs(21, 4, 2048, "bf16", 0.1, seed=4)
+    H = inp["H"].cuda()
+    for j in range(4):
+        a = torch.zeros(21, 4, device="cuda")
+        a[:, j] = 1
+        y = hdf.hdf_gated_reduce(H, inp["Wf"].cuda(), inp["b"].cuda(), alpha_override=a)
+        assert torch.equal(y, H[:, j, :])
+
+
+def test_reduce_mean_pool_matches_oracle():
+    inp = W.make_reduce_inputs(16, 4, 256, "f32", 0.02, seed=8)
+    H = inp["H"].cuda()
+    y = hdf.hdf_gated_reduce(H, None, None, alpha_override=torch.full((16, 4), 0.25, device="cuda"))
+    np.testing.assert_allclose(to64(y), to64(inp["H"]).mean(axis=1), rtol=0, atol=1e-6)
+
+
+def test_reduce_empty_is_noop():
+    y = hdf.hdf_gated_reduce(torch.empty(0, 4, 256, device="cuda"), torch.empty(4, 1024, device="cuda"),
+                             torch.zeros(4, device="cuda"))
+    assert y.shape == (0, 256)
+
+
+def test_reduce_sweep_width_sampled_rows():
+    # reducer-only workload width (m=4, d=7168) at 65536 tokens, checked on sampled tokens
+    N, m, d = 65536, 4, 7168
+    inp = W.make_reduce_inputs(N, m, d, "bf16", 0.1, seed=11, device="cuda")
+    y = hdf.hdf_gated_reduce(inp["H"], inp["Wf"], inp["b"])
+    torch.cuda.synchronize()
+    rows = torch.cat([torch.tensor([0, 1, 2, N - 2, N - 1]), torch.randperm(N, generator=torch.Generator().manual_seed(0))[:59]])
+    Hs = to64(inp["H"][rows.cuda()])
+    y_ref, _ = O.gated_reduce(Hs, to64(inp["Wf"]), to64(inp["b"]), out_dtype="bf16")
+    assert rowwise_rel(to64(y[rows.cuda()]), y_ref) <= TOL_BF16
+    assert exact_fraction(to64(y[rows.cuda()]), y_ref) >= 0.99
