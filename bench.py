@@ -124,8 +124,9 @@ def stage_work(cfg, n_ctx, batch, ctx_lens):
 
 
 def kernels_per_step(cfg):
-    attn = 2 if cfg.dtype == "bf16" else 1
-    per_layer = 1 + 1 + 1 + attn + 1 + 1 + 1 + 1
+    # per layer: context K/V GEMM, block norm, QKV GEMM, attention (chunk merge
+    # fused), O GEMM, MLP norm, gate/up GEMM, down GEMM
+    per_layer = 8
     return 1 + 1 + cfg.n_layers * per_layer + 1 + 2 + 1
 
 
@@ -190,8 +191,30 @@ def run_ours(args, rank, world, local_rank):
     stream.synchronize()
 
     K = args.steps
-    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(n_ev)] for _ in range(K)]
-    outer = [[torch.cuda.Event(enable_timing=True) for _ in range(4)] for _ in range(K)]
+
+    def ev():
+        # external: inside graph capture the record becomes a timing node
+        try:
+            return torch.cuda.Event(enable_timing=True, external=True)
+        except TypeError:
+            return torch.cuda.Event(enable_timing=True)
+    evs = [[ev() for _ in range(n_ev)] for _ in range(K)]
+    outer = [[ev() for _ in range(4)] for _ in range(K)]
+    # torch creates CUDA events lazily: record each once so the handles the
+    # library receives are valid
+    for e in [x for row in evs + outer for x in row]:
+        e.record(stream)
+    stream.synchronize()
+    graph = None
+    if not args.eager:
+        # the K timed steps are captured once and replayed as one graph, so the
+        # host's launch rate does not gate the GPU
+        graph = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(graph, stream=stream):
+            for k in range(K):
+                step(tgt, events=evs[k], outer=outer[k])
+        graph.replay()  # warm replay (untimed)
+        stream.synchronize()
     t0 = torch.cuda.Event(enable_timing=True)
     t1 = torch.cuda.Event(enable_timing=True)
     clocks = ClockSampler(local_rank)
@@ -201,8 +224,11 @@ def run_ours(args, rank, world, local_rank):
         torch.distributed.barrier()
     torch.cuda.synchronize()
     t0.record(stream)
-    for k in range(K):
-        step(tgt, events=evs[k], outer=outer[k])
+    if graph is not None:
+        graph.replay()
+    else:
+        for k in range(K):
+            step(tgt, events=evs[k], outer=outer[k])
     t1.record(stream)
     torch.cuda.synchronize()
     if world > 1:
@@ -322,6 +348,67 @@ def oracle_step_fn(cfg, inp, tgt=None):
     return run
 
 
+def run_sweep(args):
+    """Reducer-only bandwidth sweep: H [N, 4, 7168] bf16, each N timed with
+    CUDA events over `steps` back-to-back calls (inputs far above L2), plus
+    the dense fc collapse on the same input as the comparison path."""
+    from paper_2606_26744_gb300 import build, hdf
+    build.build()
+    dev = torch.device("cuda", 0)
+    pk = peaks()
+    m, d = W.SWEEP_M, W.SWEEP_D
+    free = torch.cuda.mem_get_info()[0]
+    ns = [n for n in (args.sweep_n or W.SWEEP_N) if n * m * d * 2 * 1.6 < free]
+    rows = []
+    for n in ns:
+        inp = W.make_reduce_inputs(n, m, d, "bf16", 0.1, seed=1004, device=dev)
+        H, Wf, b = inp["H"], inp["Wf"], inp["b"]
+        y = torch.empty((n, d), dtype=torch.bfloat16, device=dev)
+        for _ in range(args.warmup):
+            hdf.hdf_gated_reduce(H, Wf, b, y=y)
+        torch.cuda.synchronize()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record()
+        for _ in range(args.steps):
+            hdf.hdf_gated_reduce(H, Wf, b, y=y)
+        e1.record()
+        torch.cuda.synchronize()
+        ms = e0.elapsed_time(e1) / args.steps
+        byt = n * m * d * 2 + n * d * 2 + m * m * d * 2
+        row = {"n": n, "ms": round(ms, 4), "gbs": round(byt / ms / 1e6, 1),
+               "frac_hbm": round(byt / ms / 1e6 / pk["hbm_gbs"], 4)}
+        if n <= args.fc_max_n:
+            Wfc = (torch.randn((d, m * d), device=dev) * 0.02).to(torch.bfloat16)
+            yfc = torch.empty_like(y)
+            hdf.hdf_fc_reduce(H, Wfc, y=yfc)
+            torch.cuda.synchronize()
+            reps = max(1, args.steps // 4)
+            e0.record()
+            for _ in range(reps):
+                hdf.hdf_fc_reduce(H, Wfc, y=yfc)
+            e1.record()
+            torch.cuda.synchronize()
+            fms = e0.elapsed_time(e1) / reps
+            row["fc_ms"] = round(fms, 3)
+            row["fc_tflops"] = round(2.0 * n * m * d * d / fms / 1e9, 1)
+            row["fc_over_reducer"] = round(fms / ms, 1)
+            del Wfc, yfc
+        rows.append(row)
+        del inp, H, y
+        torch.cuda.empty_cache()
+    big = rows[-1]
+    line = {"metric": "reducer GB/s", "value": big["gbs"], "unit": "GB/s", "n_gpus": 1, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": big["ms"], "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+            "config": {"workload": "reducer sweep", "m": m, "d": d, "n": big["n"],
+                       "l2": "inputs larger than L2 for N >= 4096"},
+            "roofline": {"kernel": "gated_reduce", "bound": "hbm", "achieved": big["gbs"], "peak": pk["hbm_gbs"],
+                         "unit": "GB/s", "frac": big["frac_hbm"], "traffic": None},
+            "sweep": rows}
+    print(json.dumps(line), flush=True)
+    return 0
+
+
 def host_cores():
     try:
         return len(os.sched_getaffinity(0))
@@ -375,13 +462,20 @@ def main():
     ap.add_argument("--steps", type=int, default=200)
     ap.add_argument("--warmup", type=int, default=10)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
-    ap.add_argument("--config", default="decode", choices=sorted(W.CONFIGS))
+    ap.add_argument("--config", default="decode", choices=sorted(W.CONFIGS) + ["sweep"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--eager", action="store_true", help="launch the timed steps one by one (no CUDA graph)")
+    ap.add_argument("--sweep-n", type=int, nargs="*", default=None, help="token counts of the reducer sweep")
+    ap.add_argument("--fc-max-n", type=int, default=262144, help="largest N for the fc comparison")
     args = ap.parse_args()
     if args.warmup < 3:
         args.warmup = 3
     if args.impl == "reference":
+        if args.config == "sweep":
+            args.config = "decode"
         return run_reference(args)
+    if args.config == "sweep":
+        return run_sweep(args)
 
     world = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
@@ -415,7 +509,9 @@ def main():
                        "heads": f"{cfg.n_heads}x{cfg.head_dim}", "ffn": cfg.ffn, "vocab": cfg.vocab,
                        "parallelism": f"replicas x{world}",
                        "l2": "no flush: one step streams > 300 MB of weights and activations, above the 126 MB L2",
-                       "timing": "CUDA events on the launch stream; per-stage events recorded inside the timed steps"},
+                       "timing": ("CUDA events on the launch stream around the K steps, " +
+                                  ("eager launches" if args.eager else "captured once as one CUDA graph and replayed") +
+                                  "; per-stage events are recorded inside the timed steps")},
             "roofline": rf,
             "reducer": {"gbs": red.get("gbs"), "frac_hbm": red.get("frac"), "us": red["us"]},
             "stages": stages,

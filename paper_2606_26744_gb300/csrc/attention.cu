@@ -10,8 +10,9 @@
 // 4-stage ring; tile i lands in stage i % 4 and is consumed by warp i % 4,
 // which runs S = Q K^T and O += P V on mma.sync m16n8k16 (the B <= 16 queries
 // are one m16 row tile) with an fp32 online softmax in the log2 domain.  The
-// four warps merge in shared memory, the CTA writes an fp32 partial
-// (m, l, O) and a combine kernel merges the chunks of each (sequence, head).
+// four warps merge in shared memory; a sequence that fits one chunk writes
+// its output directly, otherwise each CTA writes an fp32 partial (m, l, O)
+// and the last chunk to finish (atomic ticket) merges them.
 // With B queries per key the kernel does ~B flops per byte of K/V, so it is
 // bound by HBM, not by the tensor pipe.
 #include <cmath>
@@ -134,7 +135,8 @@ __global__ void __launch_bounds__(160, 1)
     for (int t = warp; t < ntiles; t += NCW) {
       const int s = t % NSTAGE;
       const uint32_t ph = (t / NSTAGE) & 1;
-      if (!mbar_wait(smem_u32(&full_bar[s]), ph, a.status)) break;
+      const bool got = mbar_wait(smem_u32(&full_bar[s]), ph, a.status);
+      if (!__all_sync(0xffffffffu, got)) break;  // warp-uniform exit
       const bool blk = t >= n_ctx_tiles;
       const int valid = blk ? B : min(KT, kend - kbeg - t * KT);
       const uint32_t kbase = smem_u32(smem + s * STAGE_BYTES);
@@ -195,14 +197,19 @@ __global__ void __launch_bounds__(160, 1)
         o[i][0] *= al0; o[i][1] *= al0;
         o[i][2] *= al1; o[i][3] *= al1;
       }
-      // O += P V : 4 k-steps of 16 keys
+      // O += P V : 4 k-steps of 16 keys.  P is split into a bf16 high part
+      // and a bf16 remainder (two MMAs), which keeps ~16 significant bits of
+      // the softmax weights instead of bf16's 8.
 #pragma unroll
       for (int kk = 0; kk < 4; ++kk) {
-        uint32_t pa[4];
-        pa[0] = pack_bf16x2(sc[2 * kk][0], sc[2 * kk][1]);
-        pa[1] = pack_bf16x2(sc[2 * kk][2], sc[2 * kk][3]);
-        pa[2] = pack_bf16x2(sc[2 * kk + 1][0], sc[2 * kk + 1][1]);
-        pa[3] = pack_bf16x2(sc[2 * kk + 1][2], sc[2 * kk + 1][3]);
+        uint32_t pa[4], pl[4];
+        const float pv8[8] = {sc[2 * kk][0], sc[2 * kk][1], sc[2 * kk][2], sc[2 * kk][3],
+                              sc[2 * kk + 1][0], sc[2 * kk + 1][1], sc[2 * kk + 1][2], sc[2 * kk + 1][3]};
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+          pa[i] = pack_bf16x2(pv8[2 * i], pv8[2 * i + 1]);
+          pl[i] = pack_bf16x2(pv8[2 * i] - bf16lo(pa[i]), pv8[2 * i + 1] - bf16hi(pa[i]));
+        }
 #pragma unroll
         for (int np = 0; np < NB_O / 2; ++np) {
           const int mat = lane >> 3, rr = lane & 7;
@@ -212,7 +219,9 @@ __global__ void __launch_bounds__(160, 1)
           uint32_t b0, b1, b2, b3;
           ldsm_x4_t(addr, b0, b1, b2, b3);
           mma16816(o[2 * np], pa, b0, b1);
+          mma16816(o[2 * np], pl, b0, b1);
           mma16816(o[2 * np + 1], pa, b2, b3);
+          mma16816(o[2 * np + 1], pl, b2, b3);
         }
       }
       __syncwarp();
@@ -240,9 +249,11 @@ __global__ void __launch_bounds__(160, 1)
   if (warp == NCW) __syncthreads();  // matches (A)
   __syncthreads();
 
-  // merge the four warps, write this chunk's partial
+  // merge the four warps into this chunk's (m, l, O)
   const float* ow = reinterpret_cast<const float*>(smem);
-  const size_t pidx = (((size_t)b * a.n_heads + h) * a.n_chunks + chunk_id) * a.block;
+  __nv_bfloat16* out = reinterpret_cast<__nv_bfloat16*>(a.out);
+  const size_t base = ((size_t)b * a.n_heads + h) * a.n_chunks;
+  const size_t pidx = (base + chunk_id) * a.block;
   for (int i = tid; i < B * HD; i += blockDim.x) {
     const int r = i / HD, col = i - r * HD;
     float mstar = -INFINITY;
@@ -255,36 +266,54 @@ __global__ void __launch_bounds__(160, 1)
       acc += ow[(w * 16 + r) * HD + col] * f;
       lsum += wl[w][r] * f;
     }
-    a.part_o[(pidx + r) * HD + col] = acc;
-    if (col == 0) {
-      a.part_ml[(pidx + r) * 2] = mstar;
-      a.part_ml[(pidx + r) * 2 + 1] = lsum;
+    if (nc_b == 1) {  // the whole sequence in one CTA: final output
+      out[((size_t)b * B + r) * a.d + h * HD + col] = __float2bfloat16_rn(acc / lsum);
+    } else {
+      __stcg(a.part_o + (pidx + r) * HD + col, acc);
+      if (col == 0) {
+        __stcg(a.part_ml + (pidx + r) * 2, mstar);
+        __stcg(a.part_ml + (pidx + r) * 2 + 1, lsum);
+      }
     }
   }
-}
+  if (nc_b == 1) return;
 
-// merge chunk partials: O = sum_c O_c 2^(m_c - m*) / sum_c l_c 2^(m_c - m*)
-template <typename T>
-__global__ void attn_combine_kernel(const AttnArgs a) {
-  const int h = blockIdx.x, b = blockIdx.y, col = threadIdx.x;
-  const int HD = a.head_dim;
-  const int c0 = __ldg(a.cu_ctx + b), Tb = __ldg(a.cu_ctx + b + 1) - c0;
-  const int nc_b = min(a.n_chunks, Tb > 0 ? (Tb + a.chunk - 1) / a.chunk : 1);
-  const size_t base = ((size_t)b * a.n_heads + h) * a.n_chunks;
-  T* out = reinterpret_cast<T*>(a.out);
-  for (int r = 0; r < a.block; ++r) {
+  // The last chunk of (sequence, head) to finish merges all chunks (atomic
+  // ticket, nobody waits): O = sum_c O_c 2^(m_c - m*) / sum_c l_c 2^(m_c - m*).
+  // Per-(row, chunk) factors go to shared memory first, so the element loop
+  // issues independent loads.
+  __shared__ int last;
+  __threadfence();
+  __syncthreads();
+  if (tid == 0) last = atomicAdd(a.counters + b * a.n_heads + h, 1) == nc_b - 1;
+  __syncthreads();
+  if (!last) return;
+  __threadfence();
+  float* fac = reinterpret_cast<float*>(smem + NCW * 16 * HD * 4);  // [B][nc_b]
+  if (tid < B) {
     float mstar = -INFINITY;
-    for (int c = 0; c < nc_b; ++c) mstar = fmaxf(mstar, a.part_ml[((base + c) * a.block + r) * 2]);
-    float acc = 0.f, l = 0.f;
+    for (int c = 0; c < nc_b; ++c) mstar = fmaxf(mstar, __ldcg(a.part_ml + ((base + c) * a.block + tid) * 2));
+    float l = 0.f;
     for (int c = 0; c < nc_b; ++c) {
-      const size_t pi = (base + c) * a.block + r;
-      const float mc = a.part_ml[pi * 2];
+      const size_t pi = (base + c) * a.block + tid;
+      const float mc = __ldcg(a.part_ml + pi * 2);
       const float f = mc == -INFINITY ? 0.f : exp2f(mc - mstar);
-      l += a.part_ml[pi * 2 + 1] * f;
-      acc += a.part_o[pi * HD + col] * f;
+      fac[tid * nc_b + c] = f;
+      l += __ldcg(a.part_ml + pi * 2 + 1) * f;
     }
-    out[((size_t)b * a.block + r) * a.d + h * HD + col] = from_f32<T>(acc / l);
+    const float inv = 1.0f / l;
+    for (int c = 0; c < nc_b; ++c) fac[tid * nc_b + c] *= inv;
   }
+  __syncthreads();
+  for (int i = tid; i < B * HD; i += blockDim.x) {
+    const int r = i / HD, col = i - r * HD;
+    float acc = 0.f;
+#pragma unroll 4
+    for (int c = 0; c < nc_b; ++c)
+      acc += __ldcg(a.part_o + ((base + c) * a.block + r) * HD + col) * fac[r * nc_b + c];
+    out[((size_t)b * B + r) * a.d + h * HD + col] = __float2bfloat16_rn(acc);
+  }
+  if (tid == 0) a.counters[b * a.n_heads + h] = 0;
 }
 
 // fp32 path (tiny correctness workloads): one warp per (sequence, head, query),
@@ -349,8 +378,6 @@ cudaError_t launch_hd(const AttnArgs& a, const AttnTmaps* tm, cudaStream_t s) {
     attr_set = true;
   }
   k<<<dim3(a.n_chunks, a.n_heads, a.batch), 160, attn_smem<HD>(), s>>>(a, *tm);
-  if ((e = cudaGetLastError()) != cudaSuccess) return e;
-  attn_combine_kernel<__nv_bfloat16><<<dim3(a.n_heads, a.batch), HD, 0, s>>>(a);
   return cudaGetLastError();
 }
 

@@ -150,7 +150,8 @@ void init_gemm(GemmArgs& g, int dtype, long long M, long long N, long long K, co
 
 // ---------------------------------------------------- draft-block layout
 struct DraftLayout {
-  size_t c, kc, vc, h, x, q, kb, vb, o, act, part_o, part_ml, split, counters, total;
+  size_t c, kc, vc, h, x, q, kb, vb, o, act, part_o, part_ml, split, counters, counters_bytes, total;
+  int gemm_tiles;
   int chunk, n_chunks;
   SplitPlan qkv, oproj, gu, down;
 };
@@ -196,7 +197,10 @@ DraftLayout draft_layout(const hdf_draft_shape* sh) {
                           std::max(split_ws_bytes(L.gu), split_ws_bytes(L.down)));
   L.split = take(split);
   const int tiles = std::max(std::max(L.qkv.tiles, L.oproj.tiles), std::max(L.gu.tiles, L.down.tiles));
-  L.counters = take((size_t)tiles * 4);
+  // GEMM split-K tickets, then attention merge tickets [batch * heads]
+  L.gemm_tiles = tiles;
+  L.counters_bytes = up256(((size_t)tiles + (size_t)sh->batch * sh->n_heads) * 4);
+  L.counters = take(L.counters_bytes);
   L.total = off;
   return L;
 }
@@ -388,13 +392,22 @@ int hdf_draft_block(const hdf_drafter_weights* w, const hdf_draft_shape* sh, con
   const int want_ev = 3 + HDF_DRAFT_STAGES_PER_LAYER * sh->n_layers;
   if (trace && (!trace->events || n_ev != want_ev)) return fail(HDF_ERR_INVALID_ARG, "trace needs %d events", want_ev);
   int ev_i = 0;
+  cudaStreamCaptureStatus cap = cudaStreamCaptureStatusNone;
+  if (trace) CK(cudaStreamIsCapturing(s, &cap), "cudaStreamIsCapturing");
+  // under stream capture the records become external event nodes of the
+  // graph, so the stage times stay measurable when the graph is replayed
   auto mark = [&]() -> int {
-    if (trace) CK(cudaEventRecord((cudaEvent_t)trace->events[ev_i++], s), "cudaEventRecord");
+    if (!trace) return HDF_OK;
+    cudaEvent_t ev = (cudaEvent_t)trace->events[ev_i++];
+    if (cap == cudaStreamCaptureStatusActive)
+      CK(cudaEventRecordWithFlags(ev, s, cudaEventRecordExternal), "cudaEventRecordWithFlags");
+    else
+      CK(cudaEventRecord(ev, s), "cudaEventRecord");
     return HDF_OK;
   };
 
-  CK(cudaMemsetAsync(counters, 0, up256((size_t)std::max({Lo.qkv.tiles, Lo.oproj.tiles, Lo.gu.tiles, Lo.down.tiles}) * 4), s),
-     "memset counters");
+  CK(cudaMemsetAsync(counters, 0, Lo.counters_bytes, s), "memset counters");
+  int* attn_counters = counters + Lo.gemm_tiles;
   // ---- context RMSNorm
   if ((rc = mark())) return rc;
   CK(launch_rmsnorm(ctx, 0, w->ctx_norm, c, dt, sh->n_ctx, (int)d, sh->norm_eps, s), "ctx norm");
@@ -487,6 +500,7 @@ int hdf_draft_block(const hdf_drafter_weights* w, const hdf_draft_shape* sh, con
       a.n_ctx = sh->n_ctx;
       a.chunk = Lo.chunk;
       a.n_chunks = Lo.n_chunks;
+      a.counters = attn_counters;
       a.status = device_status_ptr();
       AttnTmaps tm;
       if (dt == HDF_BF16) {

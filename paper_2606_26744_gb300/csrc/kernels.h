@@ -114,6 +114,7 @@ struct AttnArgs {
   long long n_ctx;
   int chunk;           // context keys per split
   int n_chunks;        // splits per (sequence, head) = ceil(max_ctx / chunk) (>= 1)
+  int* counters;       // [batch * n_heads], zero on entry, left zero on exit
   int* status;
 };
 // bf16 path: TMA maps over context K/V and block K/V, box {64 cols, 64 rows}

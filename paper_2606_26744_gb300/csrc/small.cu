@@ -38,71 +38,92 @@ __device__ __forceinline__ float block_sum(float v, float* sh) {
   return t;
 }
 
-// One CTA per row: y = x / sqrt(mean(x^2) + eps) * w.  x is XT, y is T.
-template <typename XT, typename T>
-__global__ void rmsnorm_kernel(const XT* __restrict__ x, const T* __restrict__ w, T* __restrict__ y,
-                               int d, float eps) {
+// Row RMSNorm, y = x / sqrt(mean(x^2) + eps) * w, one CTA of 256 threads
+// per row.  Every thread loads its VPT 16-byte vectors of the row at once
+// (all in flight), keeps them in registers across the reduction and writes
+// y once: one read and one write of the row, no dependent load chains.
+// XT is the input type (fp32 residual or T), T the output/weight type.
+// With EMBED the row is [embed[anchor]; mask_vec x (B-1)] and is also
+// written to the fp32 residual h.
+template <typename XT, typename T, int VPT, bool EMBED>
+__global__ void __launch_bounds__(256) rmsnorm_vec_kernel(const XT* __restrict__ x, const T* __restrict__ w,
+                                                          T* __restrict__ y, int d, float eps,
+                                                          const int* __restrict__ anchor,
+                                                          const T* __restrict__ mask_vec, float* __restrict__ h,
+                                                          int block, int vocab) {
+  constexpr int XV = 16 / sizeof(XT);  // input elements per 16-byte vector
   __shared__ float sh[32];
   const long long r = blockIdx.x;
   const XT* xr = x + r * d;
+  if (EMBED) {  // x is the embedding table here
+    const int i = (int)(r / block), k = (int)(r - (long long)i * block);
+    const int tokid = min(max(__ldg(anchor + i), 0), vocab - 1);  // ids outside [0, V) are clamped
+    xr = k == 0 ? x + (long long)tokid * d : reinterpret_cast<const XT*>(mask_vec);
+  }
+  const int nv = d / XV;
+  float v[VPT][XV];
   float ss = 0.f;
-  for (int i = threadIdx.x; i < d; i += blockDim.x) {
-    const float v = to_f32(xr[i]);
-    ss = fmaf(v, v, ss);
+#pragma unroll
+  for (int k = 0; k < VPT; ++k) {
+    const int i = threadIdx.x + k * 256;
+    uint4 raw = make_uint4(0, 0, 0, 0);
+    if (i < nv) raw = ld_nc16(xr + (size_t)i * XV);
+    V16<XT>::unpack(raw, v[k]);
+#pragma unroll
+    for (int e = 0; e < XV; ++e) ss = fmaf(v[k][e], v[k][e], ss);
   }
   const float inv = rsqrtf(block_sum(ss, sh) / (float)d + eps);
-  T* yr = y + r * d;
-  for (int i = threadIdx.x; i < d; i += blockDim.x) yr[i] = from_f32<T>(to_f32(xr[i]) * inv * to_f32(w[i]));
+#pragma unroll
+  for (int k = 0; k < VPT; ++k) {
+    const int i = threadIdx.x + k * 256;
+    if (i >= nv) continue;
+    if (EMBED) {
+#pragma unroll
+      for (int e = 0; e < XV; e += 4)
+        *reinterpret_cast<float4*>(h + r * d + (size_t)i * XV + e) =
+            make_float4(v[k][e], v[k][e + 1], v[k][e + 2], v[k][e + 3]);
+    }
+    float g[XV];
+    if constexpr (sizeof(T) == 2 && XV == 8) {
+      V16<T>::unpack(ld_nc16(w + (size_t)i * 8), g);
+    } else if constexpr (sizeof(T) == 2 && XV == 4) {
+      const uint2 raw = __ldg(reinterpret_cast<const uint2*>(w + (size_t)i * 4));
+      g[0] = bf16lo(raw.x); g[1] = bf16hi(raw.x); g[2] = bf16lo(raw.y); g[3] = bf16hi(raw.y);
+    } else {
+      V16<float>::unpack(ld_nc16(w + (size_t)i * 4), g);
+    }
+    float o[XV];
+#pragma unroll
+    for (int e = 0; e < XV; ++e) o[e] = v[k][e] * inv * g[e];
+    T* yr = y + r * d + (size_t)i * XV;
+    if constexpr (sizeof(T) == 2 && XV == 8) {
+      *reinterpret_cast<uint4*>(yr) = V16<T>::pack(o);
+    } else if constexpr (sizeof(T) == 2 && XV == 4) {
+      *reinterpret_cast<uint2*>(yr) = make_uint2(pack_bf16x2(o[0], o[1]), pack_bf16x2(o[2], o[3]));
+    } else {
+      *reinterpret_cast<uint4*>(yr) = V16<float>::pack(o);
+    }
+  }
 }
 
-// Vectorised bf16 -> bf16 RMSNorm (context rows): 16-byte loads and stores.
-__global__ void rmsnorm_bf16_vec_kernel(const __nv_bfloat16* __restrict__ x,
-                                        const __nv_bfloat16* __restrict__ w,
-                                        __nv_bfloat16* __restrict__ y, int d, float eps) {
-  __shared__ float sh[32];
-  const long long r = blockIdx.x;
-  const int nv = d / 8;
-  const uint4* xr = reinterpret_cast<const uint4*>(x + r * d);
-  float ss = 0.f;
-  for (int i = threadIdx.x; i < nv; i += blockDim.x) {
-    float f[8];
-    V16<__nv_bfloat16>::unpack(ld_stream16(xr + i), f);
-#pragma unroll
-    for (int e = 0; e < 8; ++e) ss = fmaf(f[e], f[e], ss);
-  }
-  const float inv = rsqrtf(block_sum(ss, sh) / (float)d + eps);
-  uint4* yr = reinterpret_cast<uint4*>(y + r * d);
-  const uint4* wr = reinterpret_cast<const uint4*>(w);
-  for (int i = threadIdx.x; i < nv; i += blockDim.x) {
-    float f[8], g[8];
-    V16<__nv_bfloat16>::unpack(ld_nc16(xr + i), f);
-    V16<__nv_bfloat16>::unpack(ld_nc16(wr + i), g);
-#pragma unroll
-    for (int e = 0; e < 8; ++e) f[e] = f[e] * inv * g[e];
-    yr[i] = V16<__nv_bfloat16>::pack(f);
-  }
-}
-
-// Block input [anchor; mask x (B-1)] into the fp32 residual, then RMSNorm.
-template <typename T>
-__global__ void embed_norm_kernel(const T* __restrict__ embed, const T* __restrict__ mask_vec,
-                                  const int* __restrict__ anchor, const T* __restrict__ w,
-                                  float* __restrict__ h, T* __restrict__ x, int block, int d, int vocab,
-                                  float eps) {
-  __shared__ float sh[32];
-  const int r = blockIdx.x;
-  const int i = r / block, k = r - i * block;
-  const int tokid = min(max(__ldg(anchor + i), 0), vocab - 1);  // ids outside [0, V) are clamped
-  const T* src = k == 0 ? embed + (long long)tokid * d : mask_vec;
-  float ss = 0.f;
-  for (int e = threadIdx.x; e < d; e += blockDim.x) {
-    const float v = to_f32(src[e]);
-    h[(long long)r * d + e] = v;
-    ss = fmaf(v, v, ss);
-  }
-  const float inv = rsqrtf(block_sum(ss, sh) / (float)d + eps);
-  for (int e = threadIdx.x; e < d; e += blockDim.x)
-    x[(long long)r * d + e] = from_f32<T>(to_f32(src[e]) * inv * to_f32(w[e]));
+template <typename XT, typename T, bool EMBED>
+cudaError_t launch_norm_t(const void* x, const void* w, void* y, long long rows, int d, float eps,
+                          const int* anchor, const void* mask_vec, float* h, int block, int vocab,
+                          cudaStream_t s) {
+  constexpr int XV = 16 / sizeof(XT);
+  const int vpt = (d / XV + 255) / 256;
+  const dim3 grid((unsigned)rows);
+#define HDF_NORM_LAUNCH(N)                                                                                  \
+  rmsnorm_vec_kernel<XT, T, N, EMBED><<<grid, 256, 0, s>>>((const XT*)x, (const T*)w, (T*)y, d, eps, anchor, \
+                                                           (const T*)mask_vec, h, block, vocab)
+  if (vpt <= 1) HDF_NORM_LAUNCH(1);
+  else if (vpt <= 2) HDF_NORM_LAUNCH(2);
+  else if (vpt <= 4) HDF_NORM_LAUNCH(4);
+  else if (vpt <= 8) HDF_NORM_LAUNCH(8);
+  else if (vpt <= 16) HDF_NORM_LAUNCH(16);
+  else return cudaErrorInvalidValue;
+#undef HDF_NORM_LAUNCH
+  return cudaGetLastError();
 }
 
 __global__ void accept_kernel(const int* __restrict__ draft, long long ds, const int* __restrict__ target,
@@ -180,16 +201,11 @@ cudaError_t launch_rmsnorm(const void* x, int x_is_f32, const void* w, void* y, 
   if (rows == 0) return cudaSuccess;
   if (dtype == HDF_BF16) {
     if (x_is_f32)
-      rmsnorm_kernel<float, __nv_bfloat16><<<(unsigned)rows, 256, 0, s>>>(
-          (const float*)x, (const __nv_bfloat16*)w, (__nv_bfloat16*)y, d, eps);
-    else
-      rmsnorm_bf16_vec_kernel<<<(unsigned)rows, 128, 0, s>>>((const __nv_bfloat16*)x,
-                                                             (const __nv_bfloat16*)w, (__nv_bfloat16*)y, d, eps);
-  } else {
-    rmsnorm_kernel<float, float><<<(unsigned)rows, 256, 0, s>>>((const float*)x, (const float*)w, (float*)y,
-                                                                d, eps);
+      return launch_norm_t<float, __nv_bfloat16, false>(x, w, y, rows, d, eps, nullptr, nullptr, nullptr, 1, 1, s);
+    return launch_norm_t<__nv_bfloat16, __nv_bfloat16, false>(x, w, y, rows, d, eps, nullptr, nullptr, nullptr, 1,
+                                                              1, s);
   }
-  return cudaGetLastError();
+  return launch_norm_t<float, float, false>(x, w, y, rows, d, eps, nullptr, nullptr, nullptr, 1, 1, s);
 }
 
 cudaError_t launch_embed_norm(const void* embed, const void* mask_vec, const int* anchor, const void* norm_w,
@@ -198,13 +214,9 @@ cudaError_t launch_embed_norm(const void* embed, const void* mask_vec, const int
   const int rows = batch * block;
   if (rows == 0) return cudaSuccess;
   if (dtype == HDF_BF16)
-    embed_norm_kernel<__nv_bfloat16><<<rows, 256, 0, s>>>(
-        (const __nv_bfloat16*)embed, (const __nv_bfloat16*)mask_vec, anchor, (const __nv_bfloat16*)norm_w, h,
-        (__nv_bfloat16*)x, block, d, vocab, eps);
-  else
-    embed_norm_kernel<float><<<rows, 256, 0, s>>>((const float*)embed, (const float*)mask_vec, anchor,
-                                                  (const float*)norm_w, h, (float*)x, block, d, vocab, eps);
-  return cudaGetLastError();
+    return launch_norm_t<__nv_bfloat16, __nv_bfloat16, true>(embed, norm_w, x, rows, d, eps, anchor, mask_vec, h,
+                                                             block, vocab, s);
+  return launch_norm_t<float, float, true>(embed, norm_w, x, rows, d, eps, anchor, mask_vec, h, block, vocab, s);
 }
 
 cudaError_t launch_accept(const int* draft, long long ds, const int* target, long long ts, int batch, int nd,

@@ -72,9 +72,23 @@ def run_step(cfg, seed, ctx_lens=None):
         assert rowwise_rel(to64(y), y_ref) <= tol_red
     err_h = rowwise_rel(to64(h), h_ref)
     assert err_h <= tol, f"h_out row-normwise error {err_h}"
-    ties = check_tokens(tok.cpu().numpy(), lm["z"])
+    # LM head stage: the oracle's logits of the GPU's own h_out (exact bf16
+    # values); the only difference left is fp32 vs fp64 accumulation, so the
+    # drafts must match bit-exactly outside the 1e-3 tie band.
+    lm_stage = O.lm_head(to64(h), w64["lm_head"], logsoftmax=cfg.logsoftmax)
+    check_tokens(tok.cpu().numpy(), lm_stage["z"])
     if cfg.logsoftmax:
-        assert rowwise_rel(to64(ls), lm["logsoftmax"]) <= tol
+        assert rowwise_rel(to64(ls), lm_stage["logsoftmax"]) <= tol
+    # End to end: drafts against the oracle run from the same inputs.  bf16
+    # storage re-rounds at every storage point, so h_out differs from the
+    # oracle's by about one ulp in a few percent of entries and the logits by
+    # a noise sigma that grows with d; drafts may differ only where the
+    # oracle's top-2 gap is within 6 sigma (and 1e-3) -- those are reported.
+    sigma = float(np.sqrt(np.mean((lm_stage["z"] - lm["z"]) ** 2)))
+    band = max(1e-3, 6 * sigma)
+    ties = check_tokens(tok.cpu().numpy(), lm["z"], band=band)
+    print(f"[{cfg.name}] h_out err {err_h:.2e}, logit noise sigma {sigma:.2e}, e2e tie band {band:.2e}, "
+          f"rows in band {ties}/{lm['z'].shape[0]}")
 
     # ---------------- verification against targets built from the oracle drafts
     B = cfg.block
