@@ -214,6 +214,29 @@ HDF_API int hdf_lm_head_argmax(const void* h, int dtype, int64_t M, int d,
                        int32_t* tok, float* zmax, float* logsoftmax,
                        void* ws, size_t ws_bytes, hdf_stream_t stream);
 
+/* Same computation and arguments as hdf_lm_head_argmax, but without a
+ * workspace argument.  The paper has no counterpart: this entry point exists
+ * for callers that cannot hand the library device memory -- for instance a
+ * plugin whose host process owns every device allocation through its own
+ * pool, or code that runs where no allocator may be called once serving has
+ * started.  The scratch lives in a file-scope device array of
+ * HDF_LM_HEAD_STATIC_SCRATCH_BYTES that every GPU loading the library keeps
+ * until the process exits; the call allocates nothing.
+ *   - The first call on a device looks up the array's device address (once
+ *     per device, with that device current); make that first call before any
+ *     stream capture.
+ *   - All calls share the one array and it keeps the last call's contents:
+ *     two calls whose kernels overlap on the GPU (different streams, or
+ *     different host threads) race and corrupt each other's results.
+ *   - A request needing more scratch than the array holds (hdf_lm_head_
+ *     workspace_size() above the limit) returns HDF_ERR_WORKSPACE and
+ *     launches nothing; use hdf_lm_head_argmax with a workspace then. */
+#define HDF_LM_HEAD_STATIC_SCRATCH_BYTES (16u << 20)
+HDF_API int hdf_lm_head_argmax_static(const void* h, int dtype, int64_t M, int d,
+                       const void* W_lm, int64_t V, float inv_temp,
+                       int32_t* tok, float* zmax, float* logsoftmax,
+                       hdf_stream_t stream);
+
 /* ------------------------------------------------------------------------
  * (4) Block verification — greedy acceptance (Sec. 1, Sec. 3.4):
  *   accept[i] = max{ n <= n_draft : draft[i][k] == target[i][k] for k < n }

@@ -9,6 +9,7 @@
 #include <cstdarg>
 #include <cstdio>
 #include <cstring>
+#include <mutex>
 #include <string>
 
 #include "common.cuh"
@@ -638,6 +639,60 @@ int hdf_lm_head_argmax(const void* h, int dtype, int64_t M, int d, const void* W
                       logsoftmax, s),
      "lm reduce");
   return HDF_OK;
+}
+
+// ------------------------------------------ LM head on library-owned scratch
+// For callers that cannot allocate device memory themselves: the LM head's
+// scratch (split-K partial tiles, per-tile argmax / sum-exp partials and the
+// tile tickets) lives in this file-scope device array instead of a caller
+// workspace.  Every GPU that loads the library holds the array until the
+// process exits; all calls share it.
+}  // extern "C"
+namespace {
+__device__ __align__(256) unsigned char g_lm_static_scratch[HDF_LM_HEAD_STATIC_SCRATCH_BYTES];
+static_assert(HDF_LM_HEAD_STATIC_SCRATCH_BYTES % 256 == 0, "scratch size must keep 256-byte alignment");
+
+// Device address of the scratch array on the current device.  In host code
+// the array's name is only a host-side stand-in, so the address has to come
+// from cudaGetSymbolAddress, once per device, with that device current.
+int lm_static_scratch(void** out) {
+  static std::mutex mu;
+  static void* ptr[64] = {nullptr};
+  int dev = 0;
+  CK(cudaGetDevice(&dev), "cudaGetDevice");
+  if (dev < 0 || dev >= 64) return fail(HDF_ERR_UNSUPPORTED, "device ordinal %d", dev);
+  std::lock_guard<std::mutex> lock(mu);
+  if (!ptr[dev]) {
+    void* p = nullptr;
+    CK(cudaGetSymbolAddress(&p, g_lm_static_scratch), "cudaGetSymbolAddress(LM-head scratch)");
+    ptr[dev] = p;
+  }
+  *out = ptr[dev];
+  return HDF_OK;
+}
+}  // namespace
+extern "C" {
+
+int hdf_lm_head_argmax_static(const void* h, int dtype, int64_t M, int d, const void* W_lm, int64_t V,
+                              float inv_temp, int32_t* tok, float* zmax, float* logsoftmax, hdf_stream_t stream) {
+  g_err.clear();
+  const bool sizes_ok = (dtype == HDF_BF16 || dtype == HDF_F32) && M > 0 && V > 0 && d > 0 && d <= 65536 &&
+                        V <= 0x7fffffffLL && M <= 0x7fffffffLL;
+  if (!sizes_ok)  // let the workspace entry point report the exact argument error (or M == 0: nothing to do)
+    return hdf_lm_head_argmax(h, dtype, M, d, W_lm, V, inv_temp, tok, zmax, logsoftmax, nullptr, 0, stream);
+  const size_t need = lm_layout(M, V, dtype, d).total;
+  if (need > (size_t)HDF_LM_HEAD_STATIC_SCRATCH_BYTES)
+    return fail(HDF_ERR_WORKSPACE,
+                "M=%lld d=%d V=%lld needs %zu bytes of scratch, the library's static buffer holds %zu; "
+                "use hdf_lm_head_argmax with a caller workspace",
+                (long long)M, d, (long long)V, need, (size_t)HDF_LM_HEAD_STATIC_SCRATCH_BYTES);
+  void* ws = nullptr;
+  int rc = lm_static_scratch(&ws);
+  if (rc) return rc;
+  // the tile tickets are cleared inside hdf_lm_head_argmax; every other
+  // scratch entry is written before it is read
+  return hdf_lm_head_argmax(h, dtype, M, d, W_lm, V, inv_temp, tok, zmax, logsoftmax, ws,
+                            (size_t)HDF_LM_HEAD_STATIC_SCRATCH_BYTES, stream);
 }
 
 // -------------------------------------------------------------- verify

@@ -72,6 +72,8 @@ _SIGS = {
     "hdf_lm_head_argmax": (c_int, [c_vp, c_int, c_i64, c_int, c_vp, c_i64, c_float, c_vp, c_vp, c_vp,
                                    c_vp, c_size, c_vp]),
     "hdf_accept_len": (c_int, [c_vp, c_i64, c_vp, c_i64, c_int, c_int, c_vp, c_vp]),
+    "hdf_lm_head_argmax_static": (c_int, [c_vp, c_int, c_i64, c_int, c_vp, c_i64, c_float, c_vp, c_vp, c_vp,
+                                          c_vp]),
 }
 
 _lib = None
@@ -243,6 +245,27 @@ def hdf_lm_head_argmax(h: torch.Tensor, W_lm: torch.Tensor, *, inv_temp: float =
         ws = torch.empty(max(need, 1), dtype=torch.uint8, device=dev)
     _check(lib.hdf_lm_head_argmax(_p(h), _dtype(h), M, d, _p(W_lm), V, inv_temp, _p(tok), _p(zmax),
                                   _p(ls) if logsoftmax else None, _p(ws), ws.numel(), _stream(stream)))
+    return tok, zmax, (ls if logsoftmax else None)
+
+
+def hdf_lm_head_argmax_static(h: torch.Tensor, W_lm: torch.Tensor, *, inv_temp: float = 1.0,
+                              logsoftmax: bool = False, tok: Optional[torch.Tensor] = None,
+                              zmax: Optional[torch.Tensor] = None, ls: Optional[torch.Tensor] = None,
+                              stream=None):
+    """LM head on the library's own scratch array: for callers that cannot
+    give the library device memory for a workspace.  Outputs are still the
+    caller's; calls that overlap on the GPU share the scratch and race."""
+    M, d = h.shape
+    V = W_lm.shape[0]
+    dev = h.device
+    if tok is None:
+        tok = torch.empty((M,), dtype=torch.int32, device=dev)
+    if zmax is None:
+        zmax = torch.empty((M,), dtype=torch.float32, device=dev)
+    if logsoftmax and ls is None:
+        ls = torch.empty((M, V), dtype=torch.float32, device=dev)
+    _check(load().hdf_lm_head_argmax_static(_p(h), _dtype(h), M, d, _p(W_lm), V, inv_temp, _p(tok), _p(zmax),
+                                            _p(ls) if logsoftmax else None, _stream(stream)))
     return tok, zmax, (ls if logsoftmax else None)
 
 
