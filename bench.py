@@ -292,6 +292,17 @@ def run_ours(args, rank, world, local_rank):
                 h2d=h2d, d2h=d2h, acc_mean=acc_mean, tok=tok, y=y, inputs=inp, tgt=tgt)
 
 
+# DRAM bytes (read + write) per launch from the ncu captures summarised in
+# profiles/*_decode.md, decode workload only; an entry must be removed when
+# its kernel changes.
+NCU_DRAM_BYTES_DECODE = {
+    "L0.ctx_kv_gemm": 26285568 + 256,
+    "lm_head": 134415104 + 3586560,
+    "L0.attention": 17013504,
+    "gated_reduce": 33692416,
+}
+
+
 def roofline_of(cfg, res, pk):
     work = stage_work(cfg, res["n_ctx"], res["batch"], res["lens"])
     dom = max(res["dur"], key=lambda n: res["dur"][n])
@@ -318,6 +329,9 @@ def roofline_of(cfg, res, pk):
         ach = byt / t / 1e9
         rf = {"kernel": dom, "bound": "hbm", "achieved": round(ach, 1), "peak": pk["hbm_gbs"], "unit": "GB/s",
               "frac": round(ach / pk["hbm_gbs"], 4), "traffic": None, "peak_source": pk["source"] + " hbm copy"}
+    if cfg.name == "decode" and dom in NCU_DRAM_BYTES_DECODE:
+        rf["traffic"] = NCU_DRAM_BYTES_DECODE[dom]
+        rf["algorithmic_bytes"] = byt
     return rf, stages
 
 
