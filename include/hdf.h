@@ -100,6 +100,19 @@ HDF_API int hdf_gated_reduce(const void* H, int dtype, int64_t n_tokens, int m, 
                      const float* alpha_override,
                      void* y, float* alpha_out, hdf_stream_t stream);
 
+/* Kernel choice of hdf_gated_reduce; both compute Eq. 1 and agree within
+ * fp32 summation order.  HDF_REDUCE_GENERAL: one CTA streams whole tokens and
+ * re-reads them from L2 for the weighted sum (every dtype and option).
+ * HDF_REDUCE_CLUSTER: 8-CTA clusters split d, keep W_f slices in shared
+ * memory and exchange the gate partials over distributed shared memory
+ * (bf16, m in {1,2,4}, d % 512 == 0, no alpha_override or path_norm_w; the
+ * general kernel runs otherwise).  HDF_REDUCE_AUTO (the default) takes the
+ * cluster kernel for m >= 2 and n_tokens >= 8192, where it is faster.
+ * Process-wide; returns HDF_ERR_INVALID_ARG for another value.  The paper
+ * has no counterpart: it is a tuning and test hook. */
+enum { HDF_REDUCE_AUTO = 0, HDF_REDUCE_GENERAL = 1, HDF_REDUCE_CLUSTER = 2 };
+HDF_API int hdf_set_reduce_path(int path);
+
 /* Generic fc reducer of vanilla DFlash (Sec. 2.2, Table 1 "generic fc"),
  * kept as the comparison path and the fallback the paper names:
  *   y_t = W_fc vec(H_t),   W_fc [d, m*d] dtype, y [n_tokens, d] dtype.

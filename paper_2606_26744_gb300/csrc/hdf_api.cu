@@ -9,6 +9,7 @@
 #include <cstdarg>
 #include <cstdio>
 #include <cstring>
+#include <atomic>
 #include <mutex>
 #include <string>
 
@@ -259,6 +260,16 @@ int hdf_device_status(int reset) {
 }
 
 // ------------------------------------------------------------- reducer
+static std::atomic<int> g_reduce_path{HDF_REDUCE_AUTO};
+
+int hdf_set_reduce_path(int path) {
+  g_err.clear();
+  if (path != HDF_REDUCE_AUTO && path != HDF_REDUCE_GENERAL && path != HDF_REDUCE_CLUSTER)
+    return fail(HDF_ERR_INVALID_ARG, "reduce path %d", path);
+  g_reduce_path.store(path);
+  return HDF_OK;
+}
+
 int hdf_gated_reduce(const void* H, int dtype, int64_t n_tokens, int m, int d, const void* Wf, const float* b,
                      float rms_eps, float gate_scale, float gate_offset, const void* path_norm_w,
                      float path_norm_eps, const float* alpha_override, void* y, float* alpha_out,
@@ -293,6 +304,26 @@ int hdf_gated_reduce(const void* H, int dtype, int64_t n_tokens, int m, int d, c
   a.gate_offset = gate_offset;
   a.path_norm_eps = path_norm_eps;
   a.status = device_status_ptr();
+  unsigned box[3];
+  const int path = g_reduce_path.load();
+  const bool cluster_wanted =
+      path == HDF_REDUCE_CLUSTER || (path == HDF_REDUCE_AUTO && m >= 2 && n_tokens >= 8192);
+  if (cluster_wanted && reduce_cluster_box(a, dtype, box)) {
+    // 3-D view of H: {64 elements, tokens, 128-byte chunks of a token row}
+    auto fn = encode_fn();
+    if (!fn) return fail(HDF_ERR_CUDA, "cuTensorMapEncodeTiled unavailable");
+    CUtensorMap hm;
+    cuuint64_t dims[3] = {64, (cuuint64_t)n_tokens, (cuuint64_t)((long long)m * d / 64)};
+    cuuint64_t strides[2] = {(cuuint64_t)((long long)m * d * 2), 128};
+    cuuint32_t bx[3] = {box[0], box[1], box[2]};
+    cuuint32_t estr[3] = {1, 1, 1};
+    CUresult r = fn(&hm, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(H), dims, strides, bx, estr,
+                    CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_NONE,
+                    CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    if (r != CUDA_SUCCESS) return fail(HDF_ERR_CUDA, "cuTensorMapEncodeTiled (3-D view of H) failed (%d)", (int)r);
+    CK(launch_gated_reduce_cluster(a, &hm, (cudaStream_t)stream), "gated_reduce cluster launch");
+    return HDF_OK;
+  }
   CK(launch_gated_reduce(a, dtype, (cudaStream_t)stream), "gated_reduce launch");
   return HDF_OK;
 }

@@ -22,6 +22,11 @@ struct ReduceArgs {
   int* status;
 };
 cudaError_t launch_gated_reduce(const ReduceArgs& a, int dtype, cudaStream_t s);
+// bf16 cluster path: box {64, rb, E/64} of the 3-D view {64 elements, tokens,
+// 128-byte chunks} of H (128-byte swizzle) that the caller encodes; false
+// when the shape or options need the general kernel above.
+bool reduce_cluster_box(const ReduceArgs& a, int dtype, unsigned box[3]);
+cudaError_t launch_gated_reduce_cluster(const ReduceArgs& a, const CUtensorMap* h_map, cudaStream_t s);
 
 // --------------------------------------------------------------- GEMM ----
 // D[M, N] = A[M, K] * B[N, K]^T, both operands K-major, loaded by TMA with

@@ -225,4 +225,619 @@ cudaError_t launch_gated_reduce(const ReduceArgs& a, int dtype, cudaStream_t s) 
   return dtype == HDF_BF16 ? launch_t<__nv_bfloat16>(a, s) : launch_t<float>(a, s);
 }
 
+// ===========================================================================
+// bf16 cluster path (the hot path of Eq. 1).
+//
+// A cluster of 8 CTAs shares every token: CTA rank c owns elements
+// [c*E, (c+1)*E) of each of the m paths (E = d/8), so its slice of W_f
+// (m x m*E, 28 KB at d = 7168) stays in shared memory for the whole run.
+// Tokens move in batches of RB (8, or 4 when the slice is wide).  The warps
+// of a CTA have fixed roles and meet only at mbarriers:
+//   producer warp   one TMA box per path per batch from the 3-D view
+//                   {64 elements, tokens, 128-byte chunks} of H, which lands
+//                   as [chunk][token][64 elements] rows of 128 bytes with the
+//                   128-byte swizzle, so ldmatrix reads any 8 of them without
+//                   bank conflicts
+//   NGW gate warps  split every batch's tiles; each warp owns the same tiles
+//                   in every batch, so its W_f fragments and shared-memory
+//                   offsets stay in registers.  On the tensor cores
+//                   (mma.sync m16n8k16) the 16 rows of a tile are (token,
+//                   k-range) pairs, RB tokens x KR = 16/RB k-ranges of 16
+//                   elements; the 8 columns are (gate, k-range) pairs of W_f,
+//                   and only the blocks whose k-ranges agree are kept.  The
+//                   sums of squares come from the same A fragments on the
+//                   FP32 pipe.  Pairs of gate warps combine their partials and
+//                   send them to every rank with st.async, which completes the
+//                   receiver's exchange mbarrier on bytes.  A slot goes back
+//                   to the producer as soon as the gate warps are done with
+//                   it, so most of the ring is always loading.
+//   alpha warp      sums every batch's partials over all senders in a fixed
+//                   order (the same on every rank, so every rank gets the same
+//                   alpha) and publishes alpha for the batch
+//   NWW weighted    take whole batches in turn and write the y slice, reading
+//   warps           H again: the batch was streamed a few microseconds before
+//                   and is still in L2
+// Gate warps run at most LA batches ahead of the alpha warp, which bounds how
+// far any rank can run ahead in the exchange.  H comes from HBM once, W_f once
+// per CTA.
+namespace {
+
+constexpr int RC = 8;              // CTAs per cluster
+constexpr int NGW = 8;             // gate warps
+constexpr int GGRP = 2;            // gate warps whose partials are combined before they are sent
+constexpr int MAXT = 8;            // tiles per gate warp and batch (fragments held in registers)
+constexpr int NWW = 6;             // weighted warps
+constexpr int NAB = NWW + 2;       // published alpha buffers
+constexpr int NTHR = 32 * (2 + NGW + NWW);  // + producer warp + alpha warp
+constexpr int LA = 4;              // gate warps run at most this many batches ahead
+constexpr int NXCH = 2 * LA + 2;   // exchange buffers (a rank sends batch j only after this rank used j - 2*LA)
+constexpr int NSRC = RC * NGW / GGRP;  // partial senders per batch: (rank, gate warp group), one per lane
+
+struct RedGeo {
+  int E;       // elements per path in a CTA slice
+  int rb;      // tokens per batch (4 or 8)
+  int ws;      // W_f slice row stride (bytes): m*E*2 + 16
+  int box;     // bytes of one path's box: E * rb * 2
+  int preg;    // path region stride in a slot: box rounded up to 1024 bytes
+  int slot;    // bytes per batch slot: m * preg
+  int ring;    // batch slots
+  int xbuf;    // bytes of one exchange buffer: NSRC rows of rb * (m+1) partials
+  long long nbatch;
+};
+
+__device__ __forceinline__ uint32_t cluster_rank() {
+  uint32_t r;
+  asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+  return r;
+}
+__device__ __forceinline__ uint32_t cluster_id_x() {
+  uint32_t r;
+  asm volatile("mov.u32 %0, %%clusterid.x;" : "=r"(r));
+  return r;
+}
+__device__ __forceinline__ uint32_t n_clusters_x() {
+  uint32_t r;
+  asm volatile("mov.u32 %0, %%nclusterid.x;" : "=r"(r));
+  return r;
+}
+__device__ __forceinline__ uint32_t map_rank(uint32_t local, uint32_t rank) {
+  uint32_t r;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(local), "r"(rank));
+  return r;
+}
+__device__ __forceinline__ void cluster_sync_all() {
+  asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
+__device__ __forceinline__ bool mbar_try_wait_cluster(uint32_t bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n .reg .pred p;\n mbarrier.try_wait.parity.acquire.cluster.shared::cta.b64 p, [%1], %2;\n"
+      " selp.u32 %0, 1, 0, p;\n}\n"
+      : "=r"(ok)
+      : "r"(bar), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+__device__ __forceinline__ bool mbar_wait_cluster(uint32_t bar, uint32_t parity, int* status) {
+  if (mbar_try_wait_cluster(bar, parity)) return true;
+  const unsigned long long t0 = globaltimer_ns();
+  while (true) {
+#pragma unroll 1
+    for (int i = 0; i < 32; ++i)
+      if (mbar_try_wait_cluster(bar, parity)) return true;
+    if (globaltimer_ns() - t0 > kWaitLimitNs) {
+      record_device_error(status);
+      return false;
+    }
+  }
+}
+__device__ __forceinline__ void ldsm_x2(uint32_t addr, uint32_t& r0, uint32_t& r1) {
+  asm volatile("ldmatrix.sync.aligned.m8n8.x2.shared.b16 {%0,%1}, [%2];" : "=r"(r0), "=r"(r1) : "r"(addr));
+}
+__device__ __forceinline__ void ldsm_x4(uint32_t addr, uint32_t& r0, uint32_t& r1, uint32_t& r2, uint32_t& r3) {
+  asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0,%1,%2,%3}, [%4];"
+               : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
+               : "r"(addr));
+}
+__device__ __forceinline__ void mma16816(float* d, const uint32_t* a, uint32_t b0, uint32_t b1) {
+  asm volatile(
+      "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, "
+      "{%0,%1,%2,%3};"
+      : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
+      : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
+}
+__device__ __forceinline__ void tma_load_3d(uint32_t dst, const CUtensorMap* map, int x, int y, int z, uint32_t bar) {
+  asm volatile(
+      "cp.async.bulk.tensor.3d.shared::cluster.global.mbarrier::complete_tx::bytes"
+      " [%0], [%1, {%2, %3, %4}], [%5];" ::"r"(dst),
+      "l"((uint64_t)map), "r"(x), "r"(y), "r"(z), "r"(bar)
+      : "memory");
+}
+
+// acc.{x,y} += (bf16 pair of w)^2, both halves at once
+__device__ __forceinline__ void sq_acc2(unsigned long long& acc, uint32_t w) {
+  const unsigned long long v = ((unsigned long long)(w & 0xffff0000u) << 32) | (unsigned long long)(w << 16);
+  asm("fma.rn.f32x2 %0, %1, %1, %0;" : "+l"(acc) : "l"(v));
+}
+__device__ __forceinline__ float sum2(unsigned long long v) {
+  return __uint_as_float((uint32_t)v) + __uint_as_float((uint32_t)(v >> 32));
+}
+
+// k-step (16 elements of a path slice) that k-range kr of tile step s covers.
+// Every k-step is covered once.  The order keeps the W_f rows one B fragment
+// reads, (gate, k-range) pairs, in distinct bank groups: k-ranges that share
+// an 8-column tile sit 2 k-steps (64 bytes) apart.
+template <int KR>
+__device__ __forceinline__ int kstep_of(int s, int kr) {
+  if (KR == 4) return 4 * s + ((kr & 1) << 1) + (kr >> 1);  // 0, 2, 1, 3
+  return 4 * (s >> 1) + 2 * kr + (s & 1);                   // KR == 2
+}
+
+template <int M, int RB>
+__global__ void __launch_bounds__(NTHR, 1)
+    gated_reduce_cluster_kernel(const ReduceArgs a, const RedGeo geo, const __grid_constant__ CUtensorMap hmap) {
+  constexpr int KR = 16 / RB;          // k-ranges per tile
+  constexpr int NCOL = M * KR;         // (gate, k-range) columns
+  constexpr int NT = (NCOL + 7) / 8;   // 8-column tiles (2 only for m = 4, RB = 4)
+  constexpr int NV = M + 1;            // partials per token: m gate dots, sum of squares
+  constexpr int XV = RB * NV;          // partials per sender
+  constexpr int U = M == 1 ? 8 : 16 / M;  // weighted outputs per lane and round (8-16 loads in flight)
+  constexpr uint32_t kXchBytes = NSRC * XV * 4;  // one batch's partials from all senders
+  static_assert(RB * M <= 32, "one lane per alpha");
+  static_assert(NSRC == 32 && XV % 4 == 0 && XV <= 64, "one sender per lane; rows are read as float4");
+
+  extern __shared__ __align__(128) uint8_t sm[];
+  __shared__ __align__(8) uint64_t full_bar[16];
+  __shared__ __align__(8) uint64_t empty_bar[16];
+  __shared__ __align__(8) uint64_t xfull[NXCH];
+  __shared__ __align__(8) uint64_t xdone[NXCH];        // the alpha warp has read an exchange buffer
+  __shared__ __align__(8) uint64_t alpha_ready[NAB];
+  __shared__ __align__(8) uint64_t alpha_free[NAB];
+  __shared__ float red[NGW][16][NV];    // per gate warp: tile row (token, k-range) x partial
+  __shared__ float alpha_s[NAB][RB][M];
+  __shared__ float bias_s[M];
+  __shared__ volatile int abort_flag;
+  __shared__ volatile int group_abort[NGW / GGRP];  // written and read by one gate warp group only
+
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const uint32_t rank = cluster_rank(), cid = cluster_id_x(), ncl = n_clusters_x();
+  const int d = a.d, E = geo.E, e0 = (int)rank * E;
+  const long long n = a.n_tokens;
+  uint8_t* wsm = sm;  // [M gates][ws bytes]
+  // TMA destinations start on a 128-byte boundary: the ring starts on the
+  // next 1024-byte boundary after the W_f slice (the launch adds the slack)
+  const uint32_t sm0 = smem_u32(sm);
+  uint8_t* ring = sm + (((sm0 + M * geo.ws + 1023u) & ~1023u) - sm0);  // [ring][m paths][chunk][RB][128 B]
+  float* xch = reinterpret_cast<float*>(ring + (size_t)geo.ring * geo.slot);  // [NXCH][NSRC][XV]
+
+  // W_f slice: row j = gate j, flat slice index k = p*E + e
+  {
+    const int per_row16 = M * E / 8;
+    const __nv_bfloat16* Wf = reinterpret_cast<const __nv_bfloat16*>(a.Wf);
+    for (int i = tid; i < M * per_row16; i += blockDim.x) {
+      const int j = i / per_row16, r = i - j * per_row16;
+      const int p = (r * 8) / E, e = r * 8 - p * E;
+      *reinterpret_cast<uint4*>(wsm + j * geo.ws + r * 16) =
+          __ldg(reinterpret_cast<const uint4*>(Wf + (size_t)j * M * d + (size_t)p * d + e0 + e));
+    }
+  }
+  const long long nl = geo.nbatch > (long long)cid ? (geo.nbatch - cid + ncl - 1) / ncl : 0;
+  if (tid < M) bias_s[tid] = a.b[tid];
+  if (tid == 0) {
+    for (int s = 0; s < geo.ring; ++s) {
+      mbar_init(smem_u32(&full_bar[s]), 1);
+      mbar_init(smem_u32(&empty_bar[s]), NGW);
+    }
+    // exchange barriers complete on bytes: every rank's st.async signals them
+    for (int b = 0; b < NXCH; ++b) {
+      mbar_init(smem_u32(&xfull[b]), 1);
+      mbar_init(smem_u32(&xdone[b]), 1);
+    }
+    for (int b = 0; b < NAB; ++b) {
+      mbar_init(smem_u32(&alpha_ready[b]), 1);
+      mbar_init(smem_u32(&alpha_free[b]), 1);
+    }
+    abort_flag = 0;
+    for (int gg = 0; gg < NGW / GGRP; ++gg) group_abort[gg] = 0;
+    fence_mbar_init();
+    for (int b = 0; b < NXCH && b < nl; ++b) mbar_arrive_expect_tx(smem_u32(&xfull[b]), kXchBytes);
+  }
+  __syncthreads();
+  cluster_sync_all();  // every rank's barriers exist (and are armed) before anyone signals them remotely
+
+  // a wait that every lane of the warp takes; false (for the whole warp) on
+  // time-out or when another warp has given up
+  auto warp_wait = [&](uint32_t bar, uint32_t parity, bool cluster_scope) -> bool {
+    bool got = cluster_scope ? mbar_wait_cluster(bar, parity, a.status) : mbar_wait(bar, parity, a.status);
+    got = __all_sync(0xffffffffu, got) && !__any_sync(0xffffffffu, abort_flag != 0);
+    if (!got && lane == 0) abort_flag = 1;
+    return got;
+  };
+  auto arrive = [&](uint64_t* bar) {
+    if (lane == 0) asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(bar)) : "memory");
+  };
+
+  if (warp == 0) {
+    if (lane == 0) {  // ---------------------------------------------- producer
+      prefetch_tmap(&hmap);
+      long long issued = 0;
+      for (long long i = 0; i < nl && !abort_flag; ++i) {
+        const int slot = (int)(i % geo.ring);
+        const uint32_t ph = (uint32_t)((i / geo.ring) & 1);
+        if (!mbar_wait(smem_u32(&empty_bar[slot]), ph ^ 1, a.status)) { abort_flag = 1; break; }
+        const long long t0 = ((long long)cid + i * ncl) * RB;
+        const uint32_t fb = smem_u32(&full_bar[slot]);
+        mbar_arrive_expect_tx(fb, (uint32_t)(M * geo.box));
+        const uint32_t dst = smem_u32(ring + (size_t)slot * geo.slot);
+#pragma unroll
+        for (int p = 0; p < M; ++p)
+          tma_load_3d(dst + p * geo.preg, &hmap, 0, (int)t0, (p * d + e0) / 64, fb);
+        issued = i + 1;
+      }
+      // no copy may still be landing when the CTA exits: wait for the last
+      // batch of every slot (already complete on the normal path)
+      for (long long i = issued > geo.ring ? issued - geo.ring : 0; i < issued; ++i)
+        if (!mbar_wait(smem_u32(&full_bar[i % geo.ring]), (uint32_t)((i / geo.ring) & 1), a.status)) break;
+    }
+    __syncwarp();
+  } else if (warp <= NGW) {
+    // ------------------------------------------------------------ gate warps
+    const int gw = warp - 1, grp = gw / GGRP;
+    const int g = lane >> 2, q = lane & 3;
+    // Tiles go in units of two tile steps (s = 2*sp, 2*sp+1) of one path;
+    // unit u = gw + NGW*k belongs to this warp, its tiles are k = 2*(u/NGW) + c.
+    const int SP = E / (16 * KR);  // tile steps per path
+    const int NP = (SP + 1) / 2;   // units per path
+    // A operand, ldmatrix.x4: lane -> matrix mi (rows 0-7 / 8-15, k 0-7 / 8-15), row R
+    const int mi = lane >> 3, Ra = (lane & 7) + 8 * (mi & 1), khA = mi >> 1;
+    const int tA = Ra % RB, krA = Ra / RB;
+    // B operand (W_f), ldmatrix.x2 / x4: lane -> column n = (gate, k-range), k half
+    const int nB = 8 * (lane >> 4) + (lane & 7), khB = (lane >> 3) & 1;
+    const int jB = nB < NCOL ? nB % M : 0, krB = nB < NCOL ? nB / M : 0;
+    uint32_t aoff[MAXT], bf[MAXT][NT][2];
+    unsigned valid = 0;  // the same for every lane
+    {
+      int p = 0, sp = gw;
+      while (sp >= NP) { sp -= NP; ++p; }
+#pragma unroll
+      for (int k = 0; k < MAXT; ++k) {
+        if (k > 0 && (k & 1) == 0) {
+          sp += NGW;
+          while (sp >= NP) { sp -= NP; ++p; }
+        }
+        const int s = 2 * sp + (k & 1);
+        const bool v = p < M && s < SP;
+        if (v) valid |= 1u << k;
+        const int pv = v ? p : 0, sv = v ? s : 0;
+        const int ka = kstep_of<KR>(sv, krA);
+        const int row = (ka >> 2) * RB + tA, un = ((ka & 3) << 1) | khA;
+        aoff[k] = pv * geo.preg + row * 128 + ((un ^ (row & 7)) << 4);
+        const uint32_t baddr =
+            smem_u32(wsm + jB * geo.ws + khB * 16) + (uint32_t)(pv * E + 16 * kstep_of<KR>(sv, krB)) * 2;
+        if (NT == 2)
+          ldsm_x4(baddr, bf[k][0][0], bf[k][0][1], bf[k][NT - 1][0], bf[k][NT - 1][1]);
+        else
+          ldsm_x2(baddr, bf[k][0][0], bf[k][0][1]);
+      }
+    }
+    // the warps of a group meet at a named barrier (ids 1..NGW/GGRP)
+    auto group_sync = [&]() {
+      if (GGRP > 1) asm volatile("bar.sync %0, %1;" ::"r"(1 + grp), "r"(32 * GGRP) : "memory");
+    };
+    for (long long i = 0; i < nl; ++i) {
+      bool w_ok = true;
+      if (i >= LA) {  // credit: the alpha warp has read the partials of batch i - LA
+        const long long c = i - LA;
+        w_ok = warp_wait(smem_u32(&xdone[c % NXCH]), (uint32_t)((c / NXCH) & 1), false);
+      }
+      const int slot = (int)(i % geo.ring);
+      if (w_ok) w_ok = warp_wait(smem_u32(&full_bar[slot]), (uint32_t)((i / geo.ring) & 1), false);
+      if (GGRP > 1) {
+        // one decision for the whole group: a flag written before the
+        // barrier, read after it, never by anyone else
+        if (!w_ok && lane == 0) group_abort[grp] = 1;
+        group_sync();
+        if (group_abort[grp]) break;
+      } else if (!w_ok) {
+        break;
+      }
+      const uint32_t sbase = smem_u32(ring + (size_t)slot * geo.slot);
+      uint32_t av[MAXT][4];
+#pragma unroll
+      for (int k = 0; k < MAXT; ++k)
+        if (valid >> k & 1) ldsm_x4(sbase + aoff[k], av[k][0], av[k][1], av[k][2], av[k][3]);
+      __syncwarp();  // this warp is done with the slot
+      arrive(&empty_bar[slot]);
+      float dg[2][NT][4];  // chain: tile parity
+      unsigned long long sl[2] = {0ull, 0ull}, sh[2] = {0ull, 0ull};  // sums of squares, rows g and g + 8
+#pragma unroll
+      for (int c = 0; c < 2; ++c)
+#pragma unroll
+        for (int t = 0; t < NT; ++t) dg[c][t][0] = dg[c][t][1] = dg[c][t][2] = dg[c][t][3] = 0.f;
+#pragma unroll
+      for (int k = 0; k < MAXT; ++k) {
+        if (valid >> k & 1) {
+#pragma unroll
+          for (int t = 0; t < NT; ++t) mma16816(dg[k & 1][t], av[k], bf[k][t][0], bf[k][t][1]);
+          sq_acc2(sl[k & 1], av[k][0]);
+          sq_acc2(sl[k & 1], av[k][2]);
+          sq_acc2(sh[k & 1], av[k][1]);
+          sq_acc2(sh[k & 1], av[k][3]);
+        }
+      }
+      // keep the blocks whose k-ranges agree, and the sums of squares
+#pragma unroll
+      for (int t = 0; t < NT; ++t) {
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+          const int R = g + 8 * (e >> 1), ncol = 8 * t + 2 * q + (e & 1);
+          if (ncol < NCOL && ncol / M == R / RB) red[gw][R][ncol % M] = dg[0][t][e] + dg[1][t][e];
+        }
+      }
+      {
+        float lo = sum2(sl[0]) + sum2(sl[1]), hi = sum2(sh[0]) + sum2(sh[1]);
+        lo += __shfl_xor_sync(0xffffffffu, lo, 1);
+        hi += __shfl_xor_sync(0xffffffffu, hi, 1);
+        lo += __shfl_xor_sync(0xffffffffu, lo, 2);
+        hi += __shfl_xor_sync(0xffffffffu, hi, 2);
+        if (q == 0) {
+          red[gw][g][M] = lo;
+          red[gw][g + 8][M] = hi;
+        }
+      }
+      __syncwarp();
+      group_sync();  // the group's partials are complete
+      // the group's first warp sends; red is rewritten only after the next
+      // batch's group barrier, which that warp reaches after its sends
+      for (int x = lane; x < XV && gw % GGRP == 0; x += 32) {
+        const int tk = x / NV, k = x - tk * NV;
+        float v = 0.f;
+#pragma unroll
+        for (int h = 0; h < GGRP; ++h)
+#pragma unroll
+          for (int kr = 0; kr < KR; ++kr) v += red[gw + h][kr * RB + tk][k];
+        const int b = (int)(i % NXCH);
+        const uint32_t lx = smem_u32(xch + ((size_t)b * NSRC + rank * (NGW / GGRP) + grp) * XV + x);
+        const uint32_t lb = smem_u32(&xfull[b]);
+#pragma unroll
+        for (uint32_t r = 0; r < RC; ++r)
+          asm volatile("st.async.shared::cluster.mbarrier::complete_tx::bytes.f32 [%0], %1, [%2];" ::"r"(
+                           map_rank(lx, r)),
+                       "f"(v), "r"(map_rank(lb, r))
+                       : "memory");
+      }
+      __syncwarp();
+    }
+  } else if (warp == NGW + 1) {
+    // ------------------------------------------------------------ alpha warp
+    long long consumed = 0;
+    bool ok = true;
+    for (long long i = 0; i < nl; ++i) {
+      consumed = i;
+      const int b = (int)(i % NXCH);
+      if (!warp_wait(smem_u32(&xfull[b]), (uint32_t)((i / NXCH) & 1), true)) {
+        ok = false;
+        break;
+      }
+      // buffer b is complete: arm it for batch i + NXCH (no rank sends that
+      // batch before this warp has read batch i + 2)
+      if (lane == 0 && i + NXCH < nl) mbar_arrive_expect_tx(smem_u32(&xfull[b]), kXchBytes);
+      // lane L holds sender L's partials; a transposed butterfly sums them
+      // over the 32 senders in a fixed order and leaves partial x on lane x
+      // (and on lane x - 32 for x >= 32)
+      constexpr int XP = XV <= 32 ? 32 : 64;  // padded
+      float v[XP];
+      const float4* row = reinterpret_cast<const float4*>(xch + ((size_t)b * NSRC + lane) * XV);
+#pragma unroll
+      for (int k = 0; k < XP / 4; ++k) {
+        const float4 f = k < XV / 4 ? row[k] : make_float4(0.f, 0.f, 0.f, 0.f);
+        v[4 * k] = f.x;
+        v[4 * k + 1] = f.y;
+        v[4 * k + 2] = f.z;
+        v[4 * k + 3] = f.w;
+      }
+      __syncwarp();
+      arrive(&xdone[b]);
+#pragma unroll
+      for (int h = 0; h < XP / 32; ++h) {
+        float* w = v + 32 * h;
+#pragma unroll
+        for (int o = 16; o >= 1; o >>= 1) {
+          const bool upper = (lane & o) != 0;
+#pragma unroll
+          for (int k = 0; k < o; ++k) {
+            const float send = upper ? w[k] : w[k + o];
+            const float keep = upper ? w[k + o] : w[k];
+            w[k] = keep + __shfl_xor_sync(0xffffffffu, send, o);
+          }
+        }
+      }
+      const int tk = lane / M, j = lane - tk * M;
+      const int xg = tk * NV + j, xs = tk * NV + M;
+      const float g0 = __shfl_sync(0xffffffffu, v[0], xg & 31), s0 = __shfl_sync(0xffffffffu, v[0], xs & 31);
+      float gl = g0, ssum = s0;
+      if (XP == 64) {
+        const float g1 = __shfl_sync(0xffffffffu, v[XP == 64 ? 32 : 0], xg & 31);
+        const float s1 = __shfl_sync(0xffffffffu, v[XP == 64 ? 32 : 0], xs & 31);
+        gl = xg >= 32 ? g1 : g0;
+        ssum = xs >= 32 ? s1 : s0;
+      }
+      const int ab = (int)(i % NAB);
+      if (i >= NAB && !warp_wait(smem_u32(&alpha_free[ab]), (uint32_t)(((i / NAB) - 1) & 1), false)) {
+        ok = false;
+        break;
+      }
+      const long long t0 = ((long long)cid + i * ncl) * RB;
+      const int nv = (int)min((long long)RB, n - t0);
+      if (lane < RB * M) {
+        const float rr = rsqrtf(ssum / (float)(M * d) + a.rms_eps);
+        const float al = 1.0f / (1.0f + expf(-(a.gate_scale * rr * gl + bias_s[j]))) + a.gate_offset;
+        alpha_s[ab][tk][j] = al;
+        if (a.alpha_out && rank == 0 && tk < nv) a.alpha_out[(t0 + tk) * M + j] = al;
+      }
+      __syncwarp();
+      arrive(&alpha_ready[ab]);
+    }
+    if (!ok && lane == 0) {
+      // abort: let the other ranks' partials already on their way land
+      // before the cluster exits (one shared time limit for all of them)
+      const unsigned long long t0 = globaltimer_ns();
+      for (long long j = consumed; j < nl && j < consumed + NXCH; ++j) {
+        const uint32_t bar = smem_u32(&xfull[j % NXCH]), par = (uint32_t)((j / NXCH) & 1);
+        while (!mbar_try_wait_cluster(bar, par) && globaltimer_ns() - t0 < kWaitLimitNs) {
+        }
+      }
+    }
+  } else {
+    // -------------------------------------------------------- weighted warps
+    const int ww = warp - NGW - 2;
+    const int nitems = (E / 64) * RB * 8;  // 16-byte output units of a batch's slice
+    const __nv_bfloat16* H = reinterpret_cast<const __nv_bfloat16*>(a.H);
+    __nv_bfloat16* y = reinterpret_cast<__nv_bfloat16*>(a.y);
+    for (long long i = ww; i < nl; i += NWW) {
+      const int ab = (int)(i % NAB);
+      if (!warp_wait(smem_u32(&alpha_ready[ab]), (uint32_t)((i / NAB) & 1), false)) break;
+      const long long t0 = ((long long)cid + i * ncl) * RB;
+      const int nv = (int)min((long long)RB, n - t0);
+      for (int w0 = lane; w0 < nitems; w0 += 32 * U) {
+        // U outputs per lane, all U*m loads issued first (H comes from L2);
+        // eight lanes cover one 128-byte run of a token row
+        uint4 h[U][M];
+        int tk[U], col[U];
+#pragma unroll
+        for (int r = 0; r < U; ++r) {
+          const int wr = w0 + 32 * r;
+          const int u = wr & 7, row = wr >> 3, z = row / RB;
+          tk[r] = row - z * RB;
+          col[r] = e0 + z * 64 + u * 8;
+          const bool live = wr < nitems && tk[r] < nv;
+          if (!live) tk[r] = -1;
+#pragma unroll
+          for (int p = 0; p < M; ++p)
+            h[r][p] = live ? ld_stream16(H + ((t0 + tk[r]) * M + p) * d + col[r]) : make_uint4(0, 0, 0, 0);
+        }
+#pragma unroll
+        for (int r = 0; r < U; ++r) {
+          if (tk[r] < 0) continue;
+          float out[8];
+#pragma unroll
+          for (int e = 0; e < 8; ++e) out[e] = 0.f;
+#pragma unroll
+          for (int p = 0; p < M; ++p) {
+            float x[8];
+            V16<__nv_bfloat16>::unpack(h[r][p], x);
+            const float al = alpha_s[ab][tk[r]][p];
+#pragma unroll
+            for (int e = 0; e < 8; ++e) out[e] = fmaf(al, x[e], out[e]);
+          }
+          *reinterpret_cast<uint4*>(y + (t0 + tk[r]) * d + col[r]) = V16<__nv_bfloat16>::pack(out);
+        }
+      }
+      __syncwarp();  // alpha_s[ab] is free once every lane is past it
+      arrive(&alpha_free[ab]);
+    }
+  }
+  __syncthreads();
+  cluster_sync_all();  // no rank still writes into this CTA's shared memory
+}
+
+bool cluster_geometry(const ReduceArgs& a, int dtype, RedGeo* geo, size_t* smem) {
+  if (dtype != HDF_BF16 || a.alpha_override || a.path_norm_w) return false;
+  if (a.n_tokens <= 0 || a.n_tokens > (1ll << 31) - 64) return false;  // TMA coordinates are 32-bit
+  if (!(a.m == 1 || a.m == 2 || a.m == 4) || a.d % (RC * 64)) return false;
+  geo->E = a.d / RC;
+  if (geo->E / 64 > 256) return false;  // TMA box dimension limit
+
+  geo->ws = a.m * geo->E * 2 + 16;
+  const size_t budget = 219 * 1024;
+  // batch size: the one that keeps more bytes loading (ring - 1 slots), 8 on a tie
+  long long best = -1;
+  for (int rb = 8; rb >= 4; rb /= 2) {
+    // the gate warps' tiles must fit their registers: m * units per path <= NGW * MAXT / 2
+    if (a.m * ((geo->E / (16 * (16 / rb)) + 1) / 2) > NGW * MAXT / 2) continue;
+    RedGeo g = *geo;
+    g.rb = rb;
+    g.box = g.E * rb * 2;
+    g.preg = (g.box + 1023) & ~1023;
+    g.slot = a.m * g.preg;
+    g.xbuf = NSRC * rb * (a.m + 1) * 4;
+    const size_t fixed = (size_t)a.m * g.ws + (size_t)NXCH * g.xbuf + 1024;  // + alignment slack of the ring
+    if (fixed >= budget) continue;
+    g.ring = (int)std::min<long long>(16, (long long)((budget - fixed) / g.slot));
+    const long long in_flight = (long long)(g.ring - 1) * g.slot;
+    if (g.ring >= 3 && in_flight > best) {
+      best = in_flight;
+      *geo = g;
+      *smem = fixed + (size_t)g.ring * g.slot;
+    }
+  }
+  if (best < 0) return false;
+  geo->nbatch = (a.n_tokens + geo->rb - 1) / geo->rb;
+  return true;
+}
+
+template <int M, int RB>
+cudaError_t launch_cluster_mr(const ReduceArgs& a, const RedGeo& geo, size_t smem, const CUtensorMap* hmap,
+                              cudaStream_t s) {
+  auto k = gated_reduce_cluster_kernel<M, RB>;
+  cudaError_t e;
+  // attribute and cluster occupancy depend only on the shared-memory size
+  static size_t cached_smem = 0;
+  static int cached_clusters = 0;
+  cudaLaunchConfig_t cfg = {};
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = RC;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.blockDim = dim3(NTHR);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  cfg.gridDim = dim3(RC);
+  int max_clusters = cached_smem == smem ? cached_clusters : 0;
+  if (!max_clusters) {
+    if ((e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem)) != cudaSuccess)
+      return e;
+    if ((e = cudaOccupancyMaxActiveClusters(&max_clusters, k, &cfg)) != cudaSuccess) return e;
+    if (max_clusters < 1) return cudaErrorInvalidConfiguration;
+    cached_smem = smem;
+    cached_clusters = max_clusters;
+  }
+  const long long ncl = std::min<long long>(max_clusters, geo.nbatch);
+  cfg.gridDim = dim3((unsigned)(ncl * RC));
+  return cudaLaunchKernelEx(&cfg, k, a, geo, *hmap);
+}
+
+template <int M>
+cudaError_t launch_cluster_m(const ReduceArgs& a, const RedGeo& geo, size_t smem, const CUtensorMap* hmap,
+                             cudaStream_t s) {
+  return geo.rb == 8 ? launch_cluster_mr<M, 8>(a, geo, smem, hmap, s) : launch_cluster_mr<M, 4>(a, geo, smem, hmap, s);
+}
+
+}  // namespace
+
+bool reduce_cluster_box(const ReduceArgs& a, int dtype, unsigned box[3]) {
+  RedGeo geo;
+  size_t smem;
+  if (!cluster_geometry(a, dtype, &geo, &smem)) return false;
+  box[0] = 64;
+  box[1] = (unsigned)geo.rb;
+  box[2] = (unsigned)(geo.E / 64);
+  return true;
+}
+
+cudaError_t launch_gated_reduce_cluster(const ReduceArgs& a, const CUtensorMap* hmap, cudaStream_t s) {
+  RedGeo geo;
+  size_t smem;
+  if (!cluster_geometry(a, HDF_BF16, &geo, &smem)) return cudaErrorInvalidValue;
+  switch (a.m) {
+    case 1: return launch_cluster_m<1>(a, geo, smem, hmap, s);
+    case 2: return launch_cluster_m<2>(a, geo, smem, hmap, s);
+    case 4: return launch_cluster_m<4>(a, geo, smem, hmap, s);
+    default: return cudaErrorInvalidValue;
+  }
+}
+
 }  // namespace hdf

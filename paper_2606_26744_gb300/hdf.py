@@ -74,6 +74,7 @@ _SIGS = {
     "hdf_accept_len": (c_int, [c_vp, c_i64, c_vp, c_i64, c_int, c_int, c_vp, c_vp]),
     "hdf_lm_head_argmax_static": (c_int, [c_vp, c_int, c_i64, c_int, c_vp, c_i64, c_float, c_vp, c_vp, c_vp,
                                           c_vp]),
+    "hdf_set_reduce_path": (c_int, [c_int]),
 }
 
 _lib = None
@@ -127,6 +128,14 @@ def device_status(reset: bool = True) -> int:
 
 
 # ----------------------------------------------------------------- reducer
+REDUCE_PATHS = {"auto": 0, "general": 1, "cluster": 2}
+
+
+def hdf_set_reduce_path(path: str) -> None:
+    """Kernel choice of hdf_gated_reduce: "auto", "general" or "cluster"."""
+    _check(load().hdf_set_reduce_path(REDUCE_PATHS[path]))
+
+
 def hdf_gated_reduce(H: torch.Tensor, Wf: Optional[torch.Tensor], b: Optional[torch.Tensor], *,
                      rms_eps: float = 1e-6, gate_scale: float = 1.0, gate_offset: float = 0.0,
                      path_norm_w: Optional[torch.Tensor] = None, path_norm_eps: float = 1e-6,

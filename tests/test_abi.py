@@ -51,6 +51,12 @@ def test_reduce_host_validation(lib):
     assert b"aligned" in lib.hdf_last_error()
 
 
+def test_reduce_path_switch(lib):
+    assert lib.hdf_set_reduce_path(3) == 1            # HDF_ERR_INVALID_ARG
+    for path in (1, 2, 0):                            # general, cluster, auto (left at the default)
+        assert lib.hdf_set_reduce_path(path) == 0
+
+
 def test_lm_head_and_accept_host_validation(lib):
     v = ctypes.c_void_p
     assert lib.hdf_lm_head_argmax(v(16), 9, 4, 64, v(16), 100, 1.0, v(16), None, None, v(256), 1 << 20, None) == 3

@@ -11,6 +11,15 @@ from _util import TOL_BF16, TOL_F32_REDUCE, exact_fraction, rowwise_rel, to64
 pytestmark = pytest.mark.gpu
 
 
+@pytest.fixture(params=["general", "cluster"])
+def reduce_path(request):
+    """Runs a test on each kernel of the reducer (the cluster kernel takes the
+    bf16 shapes it supports; the others fall back to the general kernel)."""
+    hdf.hdf_set_reduce_path(request.param)
+    yield request.param
+    hdf.hdf_set_reduce_path("auto")
+
+
 def _run(inp, **kw):
     H = inp["H"].cuda()
     N, m, d = H.shape
@@ -30,8 +39,11 @@ def _run(inp, **kw):
     (7, 3, 128, "f32", 0.1),
     (1, 4, 4096, "bf16", 0.1),
     (3, 1, 64, "bf16", 0.1),
+    (4099, 4, 2048, "bf16", 0.1),   # many batches per cluster: ring and exchange buffers wrap
+    (50, 1, 1024, "bf16", 0.1),
+    (777, 2, 7168, "bf16", 0.1),
 ])
-def test_reduce_parity(N, m, d, dtype, std):
+def test_reduce_parity(N, m, d, dtype, std, reduce_path):
     inp = W.make_reduce_inputs(N, m, d, dtype, std, seed=N * 131 + d)
     y, a = _run(inp)
     y_ref, a_ref = O.gated_reduce(to64(inp["H"]), to64(inp["Wf"]), to64(inp["b"]), out_dtype=dtype)
@@ -63,7 +75,7 @@ def test_reduce_m1_identity_bit_exact():
     assert torch.equal(y, H[:, 0, :])
 
 
-def test_reduce_one_hot_selects_path_bit_exact():
+def test_reduce_one_hot_selects_path_bit_exact(reduce_path):
     inp = W.make_reduce_inputs(21, 4, 2048, "bf16", 0.1, seed=4)
     H = inp["H"].cuda()
     for j in range(4):
@@ -86,7 +98,7 @@ def test_reduce_empty_is_noop():
     assert y.shape == (0, 256)
 
 
-def test_reduce_sweep_width_sampled_rows():
+def test_reduce_sweep_width_sampled_rows(reduce_path):
     # reducer-only workload width (m=4, d=7168) at 65536 tokens, checked on sampled tokens
     N, m, d = 65536, 4, 7168
     inp = W.make_reduce_inputs(N, m, d, "bf16", 0.1, seed=11, device="cuda")
