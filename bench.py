@@ -205,15 +205,23 @@ def run_ours(args, rank, world, local_rank):
     for e in [x for row in evs + outer for x in row]:
         e.record(stream)
     stream.synchronize()
-    graph = None
+    graph = staged = None
     if not args.eager:
         # the K timed steps are captured once and replayed as one graph, so the
-        # host's launch rate does not gate the GPU
+        # host's launch rate does not gate the GPU; a second graph of the same
+        # steps with an event record between stages gives the breakdown (the
+        # records cost time themselves, so the step time comes from the first)
         graph = torch.cuda.CUDAGraph()
         with torch.cuda.graph(graph, stream=stream):
             for k in range(K):
+                step(tgt)
+        staged = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(staged, stream=stream):
+            for k in range(K):
                 step(tgt, events=evs[k], outer=outer[k])
-        graph.replay()  # warm replay (untimed)
+        with torch.cuda.stream(stream):  # replay() launches on the current stream
+            graph.replay()  # warm replays (untimed)
+            staged.replay()
         stream.synchronize()
     t0 = torch.cuda.Event(enable_timing=True)
     t1 = torch.cuda.Event(enable_timing=True)
@@ -225,7 +233,8 @@ def run_ours(args, rank, world, local_rank):
     torch.cuda.synchronize()
     t0.record(stream)
     if graph is not None:
-        graph.replay()
+        with torch.cuda.stream(stream):  # replay() launches on the current stream
+            graph.replay()
     else:
         for k in range(K):
             step(tgt, events=evs[k], outer=outer[k])
@@ -236,6 +245,18 @@ def run_ours(args, rank, world, local_rank):
     clk = clocks.stop()
     ms = t0.elapsed_time(t1) / K
     acc_mean = float(acc.float().mean())
+    if staged is not None:
+        with torch.cuda.stream(stream):
+            staged.replay()
+        stream.synchronize()
+        t0.record(stream)
+        with torch.cuda.stream(stream):
+            staged.replay()
+        t1.record(stream)
+        stream.synchronize()
+        ms_staged = t0.elapsed_time(t1) / K
+    else:
+        ms_staged = ms
 
     # per-stage durations over the timed region
     names = ["gated_reduce", "ctx_norm"]
@@ -251,6 +272,10 @@ def run_ours(args, rank, world, local_rank):
         dur["lm_head"] += outer[k][1].elapsed_time(outer[k][2])
         dur["accept"] += outer[k][2].elapsed_time(outer[k][3])
     dur = {n: v / K for n, v in dur.items()}
+    # the stages tile the instrumented step: their sum can only fall short of its time
+    if sum(dur.values()) > 1.02 * ms_staged:
+        raise RuntimeError(f"stage times ({sum(dur.values()):.4f} ms) exceed the step time ({ms_staged:.4f} ms): "
+                           "the step timer does not bracket the work")
 
     # ------------------------------------------------------------ e2e
     # host buffers: the residual of every context token and the targets in,
@@ -288,7 +313,7 @@ def run_ours(args, rank, world, local_rank):
         t = torch.tensor([ms, e2e_ms], device=dev)
         torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
         ms, e2e_ms = float(t[0]), float(t[1])
-    return dict(cfg=cfg, ms=ms, e2e_ms=e2e_ms, dur=dur, clk=clk, batch=batch, n_ctx=n_ctx, lens=lens,
+    return dict(cfg=cfg, ms=ms, ms_staged=ms_staged, e2e_ms=e2e_ms, dur=dur, clk=clk, batch=batch, n_ctx=n_ctx, lens=lens,
                 h2d=h2d, d2h=d2h, acc_mean=acc_mean, tok=tok, y=y, inputs=inp, tgt=tgt)
 
 
@@ -525,7 +550,9 @@ def main():
                        "l2": "no flush: one step streams > 300 MB of weights and activations, above the 126 MB L2",
                        "timing": ("CUDA events on the launch stream around the K steps, " +
                                   ("eager launches" if args.eager else "captured once as one CUDA graph and replayed") +
-                                  "; per-stage events are recorded inside the timed steps")},
+                                  "; stage times from a second replay of the same steps with an event record "
+                                  "between stages (ms_per_step_instrumented)")},
+            "ms_per_step_instrumented": round(res["ms_staged"], 5),
             "roofline": rf,
             "reducer": {"gbs": red.get("gbs"), "frac_hbm": red.get("frac"), "us": red["us"]},
             "stages": stages,
