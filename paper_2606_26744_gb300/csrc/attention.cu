@@ -69,6 +69,7 @@ __global__ void __launch_bounds__(160, 1)
 
   const int chunk_id = blockIdx.x, h = blockIdx.y, b = blockIdx.z;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  pdl_launch_dependents();
   const int B = a.block;
   const int c0 = __ldg(a.cu_ctx + b), T = __ldg(a.cu_ctx + b + 1) - c0;
   const int nc_b = min(a.n_chunks, T > 0 ? (T + a.chunk - 1) / a.chunk : 1);
@@ -87,6 +88,7 @@ __global__ void __launch_bounds__(160, 1)
     fence_mbar_init();
   }
   __syncthreads();
+  pdl_wait();  // Q and the block / context K, V come from the kernels before
 
   if (warp == NCW) {
     if (lane == 0) {  // ------------------------------------------ producer
@@ -319,6 +321,8 @@ __global__ void __launch_bounds__(160, 1)
 // fp32 path (tiny correctness workloads): one warp per (sequence, head, query),
 // exact online softmax over the keys, lane-parallel along head_dim.
 __global__ void attn_f32_kernel(const AttnArgs a) {
+  pdl_launch_dependents();
+  pdl_wait();
   const int h = blockIdx.x, b = blockIdx.y;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int HD = a.head_dim;
@@ -377,8 +381,7 @@ cudaError_t launch_hd(const AttnArgs& a, const AttnTmaps* tm, cudaStream_t s) {
       return e;
     attr_set = true;
   }
-  k<<<dim3(a.n_chunks, a.n_heads, a.batch), 160, attn_smem<HD>(), s>>>(a, *tm);
-  return cudaGetLastError();
+  return launch_kernel(k, dim3(a.n_chunks, a.n_heads, a.batch), dim3(160), attn_smem<HD>(), s, 1u, a, *tm);
 }
 
 }  // namespace
@@ -388,8 +391,7 @@ size_t attention_smem_bytes(int head_dim) { return head_dim == 64 ? attn_smem<64
 cudaError_t launch_attention(const AttnArgs& a, const AttnTmaps* tm, int dtype, cudaStream_t s) {
   if (a.batch == 0) return cudaSuccess;
   if (dtype == HDF_F32) {
-    attn_f32_kernel<<<dim3(a.n_heads, a.batch), 128, 0, s>>>(a);
-    return cudaGetLastError();
+    return launch_kernel(attn_f32_kernel, dim3(a.n_heads, a.batch), dim3(128), 0, s, 1u, a);
   }
   if (a.head_dim == 64) return launch_hd<64>(a, tm, s);
   if (a.head_dim == 128) return launch_hd<128>(a, tm, s);

@@ -15,8 +15,10 @@
 //   all 4 warps      epilogue: tcgen05.ld 32x32b (thread i <-> TMEM lane i =
 //                    tile row i), fused RoPE / residual add / SwiGLU / LM-head
 //                    argmax + sum-exp partials, direct global stores.
-// Split-K writes fp32 partial tiles; the last CTA of a tile to arrive (atomic
-// ticket, no waiting) sums them in a fixed order and runs the epilogue.
+// Split-K: the k_splits CTAs of a tile form one thread-block cluster.  Each
+// leaves its fp32 partial tile in its own shared memory; after a cluster
+// barrier rank 0 sums the ranks' tiles in rank order over distributed shared
+// memory (no global round trip, no atomics) and runs the epilogue.
 #include <algorithm>
 #include <climits>
 
@@ -40,6 +42,8 @@ template <> struct GT<float> {
 };
 
 constexpr int stages_for(int bn) { return bn >= 256 ? 4 : (bn >= 128 ? 3 : (bn >= 64 ? 4 : 5)); }
+constexpr int kPartialOffset = 8192;  // split-K partial tile in the drained stage memory, above the
+                                      // epilogue's scratch (at most 64 x 17 floats)
 constexpr int smem_for(int bn) { return stages_for(bn) * (BM + bn) * ROW_BYTES + 1024; }
 
 __device__ __forceinline__ void operand_rows(const Operand& op, int tile_row0, int half, int tile_idx,
@@ -124,16 +128,21 @@ __device__ __forceinline__ void epilogue_chunk(const GemmArgs& g, int tile_m, in
         const bool even = (fl & 1) == 0;
         const int hh = E.head_dim >> 1;
         const int pi = (fl % E.head_dim) >> 1;
+        // all 16 positions and table entries first: independent loads in flight together
+        int pos[16];
+#pragma unroll
+        for (int k = 0; k < 16; ++k)
+          pos[k] = jb + k < g.N ? (int)min((long long)block_position(E.cu_ctx, E.block, jb + k), E.rope_rows - 1) : 0;
+        float cs[16], sn[16];
+#pragma unroll
+        for (int k = 0; k < 16; ++k) {
+          cs[k] = __ldg(E.rope_cos + (size_t)pos[k] * hh + pi);
+          sn[k] = __ldg(E.rope_sin + (size_t)pos[k] * hh + pi);
+        }
 #pragma unroll
         for (int k = 0; k < 16; ++k) {
           const float pv = __shfl_xor_sync(0xffffffffu, v[k], 1);
-          const int j = jb + k;
-          if (j < g.N) {
-            const int pos = (int)min((long long)block_position(E.cu_ctx, E.block, j), E.rope_rows - 1);
-            const float c = __ldg(E.rope_cos + (size_t)pos * hh + pi);
-            const float s = __ldg(E.rope_sin + (size_t)pos * hh + pi);
-            v[k] = even ? (v[k] * c - pv * s) : (pv * s + v[k] * c);
-          }
+          if (jb + k < g.N) v[k] = even ? (v[k] * cs[k] - pv * sn[k]) : (pv * sn[k] + v[k] * cs[k]);
         }
       }
       if (f >= g.M) return;
@@ -149,14 +158,14 @@ __device__ __forceinline__ void epilogue_chunk(const GemmArgs& g, int tile_m, in
       const int f = tile_m * BM + row;
       if (f >= g.M) return;
       const int jb = tile_n * BN + c0;
+      float* base = E.resid + (long long)jb * E.ld + f;
+      // every load before any store, so the 16 reads are in flight together
+      float r[16];
 #pragma unroll
-      for (int k = 0; k < 16; ++k) {
-        const int j = jb + k;
-        if (j < g.N) {
-          float* p = E.resid + (long long)j * E.ld + f;
-          *p = *p + v[k];
-        }
-      }
+      for (int k = 0; k < 16; ++k) r[k] = jb + k < g.N ? __ldcg(base + (long long)k * E.ld) : 0.f;
+#pragma unroll
+      for (int k = 0; k < 16; ++k)
+        if (jb + k < g.N) base[(long long)k * E.ld] = r[k] + v[k];
       return;
     }
     case kEpiSwigluT: {  // rows 0..63: gate g_f, rows 64..127: up u_f (same f)
@@ -270,9 +279,9 @@ __global__ void __launch_bounds__(128, 1) gemm_kernel(const __grid_constant__ Ge
   __shared__ __align__(8) uint64_t acc_bar;
   __shared__ uint32_t tmem_slot;
   __shared__ volatile int abort_flag;
-  __shared__ int last_flag;
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  pdl_launch_dependents();
   const int tiles_m = (g.M + BM - 1) / BM;
   const int tiles_n = (g.N + BN - 1) / BN;
   int bid = blockIdx.x;
@@ -311,27 +320,45 @@ __global__ void __launch_bounds__(128, 1) gemm_kernel(const __grid_constant__ Ge
   tc_fence_after();
   const uint32_t tmem = tmem_slot;
 
+  if (!(warp == 0 && lane == 0)) pdl_wait();  // the producer waits after its weight prefetch
   if (warp == 0 && lane == 0) {
     // ------------------------------------------------ TMA producer
-    int s = 0;
-    uint32_t ph = 0;
-    int issued = 0;
-    for (int kb = kb0; kb < kb1; ++kb) {
-      if (!mbar_wait(smem_u32(&empty_bar[s]), ph ^ 1, g.status)) { abort_flag = 1; break; }
-      if (abort_flag) break;
-      const uint32_t fb = smem_u32(&full_bar[s]);
-      mbar_arrive_expect_tx(fb, STAGE_BYTES);
-      const uint32_t sa = smem_u32(smem + s * STAGE_BYTES);
-      const uint32_t sb = sa + A_BYTES;
+    auto load_a = [&](int st, int kb) {
+      const uint32_t sa = smem_u32(smem + st * STAGE_BYTES);
       const CUtensorMap* map;
       int row;
 #pragma unroll
       for (int h = 0; h < 2; ++h) {
         operand_rows(g.A, tile_m * BM, h, tile_m, &map, &row);
-        tma_load_2d(sa + h * (64 * ROW_BYTES), map, kb * BK, row, fb);
+        tma_load_2d(sa + h * (64 * ROW_BYTES), map, kb * BK, row, smem_u32(&full_bar[st]));
       }
+    };
+    auto load_b = [&](int st, int kb) {
+      const CUtensorMap* map;
+      int row;
       operand_rows(g.B, tile_n * BN, 0, tile_n, &map, &row);
-      tma_load_2d(sb, map, kb * BK, row, fb);
+      tma_load_2d(smem_u32(smem + st * STAGE_BYTES) + A_BYTES, map, kb * BK, row, smem_u32(&full_bar[st]));
+    };
+    // the first stages' weight operand is loaded while the previous kernel
+    // may still run; the other operand only after pdl_wait()
+    const int npre = g.pre_operand ? min(STAGES, kb1 - kb0) : 0;
+    for (int i = 0; i < npre; ++i) {
+      mbar_arrive_expect_tx(smem_u32(&full_bar[i]), STAGE_BYTES);
+      if (g.pre_operand == 1) load_a(i, kb0 + i); else load_b(i, kb0 + i);
+    }
+    pdl_wait();
+    for (int i = 0; i < npre; ++i) {
+      if (g.pre_operand == 1) load_b(i, kb0 + i); else load_a(i, kb0 + i);
+    }
+    int s = npre % STAGES;
+    uint32_t ph = npre == STAGES ? 1u : 0u;
+    int issued = npre;
+    for (int kb = kb0 + npre; kb < kb1; ++kb) {
+      if (!mbar_wait(smem_u32(&empty_bar[s]), ph ^ 1, g.status)) { abort_flag = 1; break; }
+      if (abort_flag) break;
+      mbar_arrive_expect_tx(smem_u32(&full_bar[s]), STAGE_BYTES);
+      load_a(s, kb);
+      load_b(s, kb);
       ++issued;
       if (++s == STAGES) { s = 0; ph ^= 1; }
     }
@@ -374,50 +401,64 @@ __global__ void __launch_bounds__(128, 1) gemm_kernel(const __grid_constant__ Ge
   __syncthreads();
   const bool aborted = abort_flag != 0;
   const uint32_t taddr = tmem + ((uint32_t)(warp * 32) << 16);
-  if (!aborted && kb1 > kb0) {
-    if (g.k_splits == 1) {
+  if (!aborted && kb1 > kb0 && g.k_splits == 1) {
+#pragma unroll 1
+    for (int c0 = 0; c0 < BN; c0 += 16) {
+      float v[16];
+      tmem_ld16(taddr + c0, v);
+      epilogue_chunk<T, BN>(g, tile_m, tile_n, c0, v, smem);
+    }
+  }
+  if (g.k_splits > 1) {
+    // every rank: accumulator -> own shared memory [128 rows][BN] (all MMAs
+    // and copies have completed, so the stage memory is free)
+    float* part = reinterpret_cast<float*>(smem + kPartialOffset);
+    if (!aborted && kb1 > kb0) {
 #pragma unroll 1
       for (int c0 = 0; c0 < BN; c0 += 16) {
         float v[16];
         tmem_ld16(taddr + c0, v);
-        epilogue_chunk<T, BN>(g, tile_m, tile_n, c0, v, smem);
+        float4* p = reinterpret_cast<float4*>(part + tid * BN + c0);
+#pragma unroll
+        for (int i = 0; i < 4; ++i) p[i] = make_float4(v[4 * i], v[4 * i + 1], v[4 * i + 2], v[4 * i + 3]);
       }
     } else {
-      const int tile = tile_m * tiles_n + tile_n;
-      float* mine = g.ws_partial + ((size_t)(tile * g.k_splits + split) * BM + tid) * BN;
+      for (int c = 0; c < BN; ++c) part[tid * BN + c] = 0.f;
+    }
+    cluster_sync_all();  // every rank's partial tile is visible to the cluster
+    if (cluster_rank() == 0) {
+      const uint32_t mine = smem_u32(part + tid * BN);
 #pragma unroll 1
       for (int c0 = 0; c0 < BN; c0 += 16) {
         float v[16];
-        tmem_ld16(taddr + c0, v);
-        float4* p = reinterpret_cast<float4*>(mine + c0);
 #pragma unroll
-        for (int i = 0; i < 4; ++i) __stcg(p + i, make_float4(v[4 * i], v[4 * i + 1], v[4 * i + 2], v[4 * i + 3]));
-      }
-      __threadfence();
-      __syncthreads();
-      if (tid == 0) last_flag = (atomicAdd(g.counters + tile, 1) == g.k_splits - 1);
-      __syncthreads();
-      if (last_flag) {
-        __threadfence();
-        const float* base = g.ws_partial + ((size_t)tile * g.k_splits * BM + tid) * BN;
-#pragma unroll 1
-        for (int c0 = 0; c0 < BN; c0 += 16) {
-          float v[16];
+        for (int i = 0; i < 16; ++i) v[i] = 0.f;
+        // four ranks' rows in flight at a time, summed in rank order
+        for (int r0 = 0; r0 < g.k_splits; r0 += 4) {
+          float4 q[4][4];
 #pragma unroll
-          for (int i = 0; i < 16; ++i) v[i] = 0.f;
-          for (int sp = 0; sp < g.k_splits; ++sp) {
-            const float4* p = reinterpret_cast<const float4*>(base + (size_t)sp * BM * BN + c0);
+          for (int u = 0; u < 4; ++u)
+            if (r0 + u < g.k_splits) {
+              const uint32_t src = map_rank(mine + c0 * 4, (uint32_t)(r0 + u));
 #pragma unroll
-            for (int i = 0; i < 4; ++i) {
-              const float4 q = __ldcg(p + i);
-              v[4 * i] += q.x; v[4 * i + 1] += q.y; v[4 * i + 2] += q.z; v[4 * i + 3] += q.w;
+              for (int i = 0; i < 4; ++i) q[u][i] = ld_dsmem_v4(src + 16 * i);
             }
-          }
-          epilogue_chunk<T, BN>(g, tile_m, tile_n, c0, v, smem);
+#pragma unroll
+          for (int u = 0; u < 4; ++u)
+            if (r0 + u < g.k_splits) {
+#pragma unroll
+              for (int i = 0; i < 4; ++i) {
+                v[4 * i] += q[u][i].x;
+                v[4 * i + 1] += q[u][i].y;
+                v[4 * i + 2] += q[u][i].z;
+                v[4 * i + 3] += q[u][i].w;
+              }
+            }
         }
-        if (tid == 0) g.counters[tile] = 0;
+        if (!aborted) epilogue_chunk<T, BN>(g, tile_m, tile_n, c0, v, smem);
       }
     }
+    cluster_sync_all();  // rank 0 has read every rank's shared memory
   }
   tc_fence_before();
   __syncthreads();
@@ -438,9 +479,15 @@ cudaError_t launch_bn(const GemmArgs& g, cudaStream_t s) {
       return e;
     attr_set = true;
   }
+  if (g.k_splits < 1 || g.k_splits > 16) return cudaErrorInvalidValue;
   const long long tiles = (long long)((g.M + BM - 1) / BM) * ((g.N + BN - 1) / BN) * g.k_splits;
-  k<<<(unsigned)tiles, 128, smem, s>>>(g);
-  return cudaGetLastError();
+  static bool cluster_attr_set = false;
+  if (g.k_splits > 8 && !cluster_attr_set) {
+    if ((e = cudaFuncSetAttribute(k, cudaFuncAttributeNonPortableClusterSizeAllowed, 1)) != cudaSuccess) return e;
+    cluster_attr_set = true;
+  }
+  // the splits of one tile are consecutive blocks: one cluster
+  return launch_kernel(k, dim3((unsigned)tiles), dim3(128), (size_t)smem, s, (unsigned)g.k_splits, g);
 }
 
 template <typename T>

@@ -118,7 +118,9 @@ struct SplitPlan {
 };
 
 // Weights-as-A GEMM (rows = output features, columns = tokens): K-split so
-// that about two CTAs per SM stream weights, each over >= 4 k-blocks.
+// that the grid fills about one wave of two CTAs per SM (a second wave would
+// only start when the first ends), each split over >= 4 k-blocks; the splits
+// of a tile run as one cluster of at most 16 CTAs.
 SplitPlan plan_swap(int dtype, long long M, long long N, long long K) {
   SplitPlan p;
   p.bn = pick_bn(N);
@@ -126,14 +128,11 @@ SplitPlan plan_swap(int dtype, long long M, long long N, long long K) {
   p.tiles = (int)(((M + 127) / 128) * ((N + p.bn - 1) / p.bn));
   const int num_kb = (int)((K + bk - 1) / bk);
   const int target = 2 * num_sms();
-  int splits = std::max(1, (target + p.tiles - 1) / p.tiles);
-  splits = std::min(splits, std::max(1, num_kb / 4));
+  int splits = std::max(1, target / p.tiles);
+  splits = std::min(std::min(splits, 16), std::max(1, num_kb / 4));
   const int kb_per = (num_kb + splits - 1) / splits;
   p.k_splits = (num_kb + kb_per - 1) / kb_per;
   return p;
-}
-size_t split_ws_bytes(const SplitPlan& p) {
-  return p.k_splits > 1 ? (size_t)p.tiles * p.k_splits * 128 * p.bn * 4 : 0;
 }
 
 void init_gemm(GemmArgs& g, int dtype, long long M, long long N, long long K, const SplitPlan& p) {
@@ -152,8 +151,7 @@ void init_gemm(GemmArgs& g, int dtype, long long M, long long N, long long K, co
 
 // ---------------------------------------------------- draft-block layout
 struct DraftLayout {
-  size_t c, kc, vc, h, x, q, kb, vb, o, act, part_o, part_ml, split, counters, counters_bytes, total;
-  int gemm_tiles;
+  size_t c, kc, vc, h, x, q, kb, vb, o, act, part_o, part_ml, counters, counters_bytes, total;
   int chunk, n_chunks;
   SplitPlan qkv, oproj, gu, down;
 };
@@ -195,13 +193,8 @@ DraftLayout draft_layout(const hdf_draft_shape* sh) {
   L.oproj = plan_swap(sh->dtype, d, M, d);
   L.gu = plan_swap(sh->dtype, 2 * F, M, d);
   L.down = plan_swap(sh->dtype, d, M, F);
-  size_t split = std::max(std::max(split_ws_bytes(L.qkv), split_ws_bytes(L.oproj)),
-                          std::max(split_ws_bytes(L.gu), split_ws_bytes(L.down)));
-  L.split = take(split);
-  const int tiles = std::max(std::max(L.qkv.tiles, L.oproj.tiles), std::max(L.gu.tiles, L.down.tiles));
-  // GEMM split-K tickets, then attention merge tickets [batch * heads]
-  L.gemm_tiles = tiles;
-  L.counters_bytes = up256(((size_t)tiles + (size_t)sh->batch * sh->n_heads) * 4);
+  // attention merge tickets [batch * heads]
+  L.counters_bytes = up256((size_t)sh->batch * sh->n_heads * 4);
   L.counters = take(L.counters_bytes);
   L.total = off;
   return L;
@@ -349,6 +342,7 @@ int hdf_fc_reduce(const void* H, int dtype, int64_t n_tokens, int m, int d, cons
   int rc;
   if ((rc = make_map(&g.A.map[0], H, dtype, n_tokens, K, K, 64))) return rc;
   if ((rc = make_map(&g.B.map[0], W_fc, dtype, d, K, K, p.bn))) return rc;
+  g.pre_operand = 2;  // the weight
   g.epi.kind = kEpiStore;
   g.epi.out[0] = y;
   g.epi.seg_width = d;
@@ -417,7 +411,6 @@ int hdf_draft_block(const hdf_drafter_weights* w, const hdf_draft_shape* sh, con
   void* vbk = W + Lo.vb;
   void* o = W + Lo.o;
   void* act = W + Lo.act;
-  float* split = reinterpret_cast<float*>(W + Lo.split);
   int* counters = reinterpret_cast<int*>(W + Lo.counters);
 
   const int n_ev = trace ? trace->n_events : 0;
@@ -439,7 +432,7 @@ int hdf_draft_block(const hdf_drafter_weights* w, const hdf_draft_shape* sh, con
   };
 
   CK(cudaMemsetAsync(counters, 0, Lo.counters_bytes, s), "memset counters");
-  int* attn_counters = counters + Lo.gemm_tiles;
+  int* attn_counters = counters;
   // ---- context RMSNorm
   if ((rc = mark())) return rc;
   CK(launch_rmsnorm(ctx, 0, w->ctx_norm, c, dt, sh->n_ctx, (int)d, sh->norm_eps, s), "ctx norm");
@@ -456,6 +449,7 @@ int hdf_draft_block(const hdf_drafter_weights* w, const hdf_draft_shape* sh, con
       if ((rc = make_map(&g.A.map[0], c, dt, sh->n_ctx, d, d, 64))) return rc;
       if ((rc = make_map(&g.B.map[0], Lw.wk, dt, d, d, d, p.bn))) return rc;
       if ((rc = make_map(&g.B.map[1], Lw.wv, dt, d, d, d, p.bn))) return rc;
+      g.pre_operand = 2;  // weights: loaded before the context norm has finished
       g.B.rows_per_map = (int)d;
       g.epi.kind = kEpiStore;
       g.epi.out[0] = kc;
@@ -491,8 +485,7 @@ int hdf_draft_block(const hdf_drafter_weights* w, const hdf_draft_shape* sh, con
       if ((rc = make_map(&g.A.map[2], Lw.wv, dt, d, d, d, 64))) return rc;
       g.A.rows_per_map = (int)d;
       if ((rc = make_map(&g.B.map[0], x, dt, M, d, d, Lo.qkv.bn))) return rc;
-      g.ws_partial = split;
-      g.counters = counters;
+      g.pre_operand = 1;
       g.epi.kind = kEpiStoreT;
       g.epi.out[0] = q;
       g.epi.out[1] = kbk;
@@ -553,8 +546,7 @@ int hdf_draft_block(const hdf_drafter_weights* w, const hdf_draft_shape* sh, con
       init_gemm(g, dt, d, M, d, Lo.oproj);
       if ((rc = make_map(&g.A.map[0], Lw.wo, dt, d, d, d, 64))) return rc;
       if ((rc = make_map(&g.B.map[0], o, dt, M, d, d, Lo.oproj.bn))) return rc;
-      g.ws_partial = split;
-      g.counters = counters;
+      g.pre_operand = 1;
       g.epi.kind = kEpiResidT;
       g.epi.resid = h;
       g.epi.ld = d;
@@ -572,8 +564,7 @@ int hdf_draft_block(const hdf_drafter_weights* w, const hdf_draft_shape* sh, con
       if ((rc = make_map(&g.A.map[1], Lw.wu, dt, F, d, d, 64))) return rc;
       g.A.mode = kPair64;
       if ((rc = make_map(&g.B.map[0], x, dt, M, d, d, Lo.gu.bn))) return rc;
-      g.ws_partial = split;
-      g.counters = counters;
+      g.pre_operand = 1;
       g.epi.kind = kEpiSwigluT;
       g.epi.out[0] = act;
       g.epi.seg_width = (int)F;
@@ -587,8 +578,7 @@ int hdf_draft_block(const hdf_drafter_weights* w, const hdf_draft_shape* sh, con
       init_gemm(g, dt, d, M, F, Lo.down);
       if ((rc = make_map(&g.A.map[0], Lw.wd, dt, d, F, F, 64))) return rc;
       if ((rc = make_map(&g.B.map[0], act, dt, M, F, F, Lo.down.bn))) return rc;
-      g.ws_partial = split;
-      g.counters = counters;
+      g.pre_operand = 1;
       g.epi.kind = kEpiResidT;
       g.epi.resid = h;
       g.epi.ld = d;
@@ -607,7 +597,7 @@ namespace {
 struct LmLayout {
   SplitPlan p;
   int tiles_m;
-  size_t pmax, parg, psum, split, counters, total;
+  size_t pmax, parg, psum, total;
 };
 LmLayout lm_layout(int64_t M, int64_t V, int dtype, int d) {
   LmLayout L;
@@ -622,8 +612,6 @@ LmLayout lm_layout(int64_t M, int64_t V, int dtype, int d) {
   L.pmax = take((size_t)L.tiles_m * M * 4);
   L.parg = take((size_t)L.tiles_m * M * 4);
   L.psum = take((size_t)L.tiles_m * M * 4);
-  L.split = take(split_ws_bytes(L.p));
-  L.counters = take((size_t)L.p.tiles * 4);
   L.total = off;
   return L;
 }
@@ -656,15 +644,13 @@ int hdf_lm_head_argmax(const void* h, int dtype, int64_t M, int d, const void* W
   int rc;
   if ((rc = make_map(&g.A.map[0], W_lm, dtype, V, d, d, 64))) return rc;
   if ((rc = make_map(&g.B.map[0], h, dtype, M, d, d, L.p.bn))) return rc;
-  g.ws_partial = reinterpret_cast<float*>(W + L.split);
-  g.counters = reinterpret_cast<int*>(W + L.counters);
+  g.pre_operand = 1;  // the LM head weight
   g.epi.kind = kEpiLmHeadT;
   g.epi.inv_temp = inv_temp;
   g.epi.logsoftmax = logsoftmax;
   g.epi.part_max = reinterpret_cast<float*>(W + L.pmax);
   g.epi.part_arg = reinterpret_cast<int*>(W + L.parg);
   g.epi.part_sum = reinterpret_cast<float*>(W + L.psum);
-  CK(cudaMemsetAsync(g.counters, 0, (size_t)L.p.tiles * 4, s), "memset counters");
   CK(launch_gemm(g, s), "lm head gemm");
   CK(launch_lm_reduce(g.epi.part_max, g.epi.part_arg, g.epi.part_sum, L.tiles_m, M, V, inv_temp, tok, zmax,
                       logsoftmax, s),
@@ -674,8 +660,7 @@ int hdf_lm_head_argmax(const void* h, int dtype, int64_t M, int d, const void* W
 
 // ------------------------------------------ LM head on library-owned scratch
 // For callers that cannot allocate device memory themselves: the LM head's
-// scratch (split-K partial tiles, per-tile argmax / sum-exp partials and the
-// tile tickets) lives in this file-scope device array instead of a caller
+// scratch (per-tile argmax / sum-exp partials) lives in this file-scope device array instead of a caller
 // workspace.  Every GPU that loads the library holds the array until the
 // process exits; all calls share it.
 }  // extern "C"

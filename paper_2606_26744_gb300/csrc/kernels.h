@@ -7,6 +7,35 @@
 
 namespace hdf {
 
+// Launches a kernel of the draft path with programmatic dependent launch
+// (its prologue may overlap the previous kernel in the stream; the kernel
+// calls pdl_wait() before touching that kernel's results) and, when
+// cluster_x > 1, as clusters of cluster_x consecutive blocks.
+template <typename... KArgs, typename... Args>
+cudaError_t launch_kernel(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t s,
+                          unsigned cluster_x, Args&&... args) {
+  cudaLaunchConfig_t cfg = {};
+  cudaLaunchAttribute attr[2];
+  unsigned n = 0;
+  attr[n].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[n].val.programmaticStreamSerializationAllowed = 1;
+  ++n;
+  if (cluster_x > 1) {
+    attr[n].id = cudaLaunchAttributeClusterDimension;
+    attr[n].val.clusterDim.x = cluster_x;
+    attr[n].val.clusterDim.y = 1;
+    attr[n].val.clusterDim.z = 1;
+    ++n;
+  }
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cfg.attrs = attr;
+  cfg.numAttrs = n;
+  return cudaLaunchKernelEx(&cfg, kernel, static_cast<KArgs>(args)...);
+}
+
 // ------------------------------------------------------------ reducer ----
 struct ReduceArgs {
   const void* H;
@@ -77,9 +106,9 @@ struct GemmArgs {
   int M, N, K;
   int dtype;            // HDF_BF16 or HDF_F32 (tf32)
   int bn;               // tile width along N: 16, 32, 64, 128 or 256
-  int k_splits;         // >= 1; >1 needs ws_partial / counters
-  float* ws_partial;    // [tiles, k_splits, 128, bn] fp32
-  int* counters;        // [tiles], zero on entry, left zero on exit
+  int k_splits;         // 1..16; > 1 launches the splits of each tile as one thread-block cluster
+  int pre_operand;      // 1: A, 2: B does not depend on earlier kernels (weights) and is loaded
+                        // before pdl_wait(); 0: neither
   int group_n;          // raster: n-tiles swept together
   Epilogue epi;
   int* status;

@@ -33,6 +33,7 @@ __global__ void __launch_bounds__(512) gated_reduce_kernel(const ReduceArgs a, i
   __shared__ float fin[NV];
 
   const int tid = threadIdx.x, nt = blockDim.x, lane = tid & 31, warp = tid >> 5;
+  pdl_launch_dependents();
   const int nwarps = nt >> 5;
   const int d = a.d, md = M * d, nvec = d / VEC;
   const long long n = a.n_tokens;
@@ -48,6 +49,7 @@ __global__ void __launch_bounds__(512) gated_reduce_kernel(const ReduceArgs a, i
     __syncthreads();
     Wf = reinterpret_cast<const T*>(dyn_smem);
   }
+  pdl_wait();  // H, y and alpha_override may belong to the kernels before
 
   const long long ngroups = (n + G - 1) / G;
   for (long long grp = blockIdx.x; grp < ngroups; grp += gridDim.x) {
@@ -195,15 +197,14 @@ cudaError_t launch_m(const ReduceArgs& a, cudaStream_t s) {
     if ((e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, k, nt, wf_bytes)) != cudaSuccess) return e;
     if (per_sm < 1) per_sm = 1;
     const long long grid = std::min<long long>(ngroups, (long long)per_sm * sms);
-    k<<<(unsigned)grid, nt, wf_bytes, s>>>(a, vpt);
+    return launch_kernel(k, dim3((unsigned)grid), dim3(nt), wf_bytes, s, 1u, a, vpt);
   } else {
     auto k = gated_reduce_kernel<T, M, G, false>;
     if ((e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, k, nt, 0)) != cudaSuccess) return e;
     if (per_sm < 1) per_sm = 1;
     const long long grid = std::min<long long>(ngroups, (long long)per_sm * sms);
-    k<<<(unsigned)grid, nt, 0, s>>>(a, vpt);
+    return launch_kernel(k, dim3((unsigned)grid), dim3(nt), 0, s, 1u, a, vpt);
   }
-  return cudaGetLastError();
 }
 
 template <typename T>
@@ -285,29 +286,6 @@ struct RedGeo {
   long long nbatch;
 };
 
-__device__ __forceinline__ uint32_t cluster_rank() {
-  uint32_t r;
-  asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
-  return r;
-}
-__device__ __forceinline__ uint32_t cluster_id_x() {
-  uint32_t r;
-  asm volatile("mov.u32 %0, %%clusterid.x;" : "=r"(r));
-  return r;
-}
-__device__ __forceinline__ uint32_t n_clusters_x() {
-  uint32_t r;
-  asm volatile("mov.u32 %0, %%nclusterid.x;" : "=r"(r));
-  return r;
-}
-__device__ __forceinline__ uint32_t map_rank(uint32_t local, uint32_t rank) {
-  uint32_t r;
-  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(local), "r"(rank));
-  return r;
-}
-__device__ __forceinline__ void cluster_sync_all() {
-  asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::: "memory");
-}
 __device__ __forceinline__ bool mbar_try_wait_cluster(uint32_t bar, uint32_t parity) {
   uint32_t ok;
   asm volatile(
@@ -400,6 +378,7 @@ __global__ void __launch_bounds__(NTHR, 1)
   __shared__ volatile int group_abort[NGW / GGRP];  // written and read by one gate warp group only
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  pdl_launch_dependents();
   const uint32_t rank = cluster_rank(), cid = cluster_id_x(), ncl = n_clusters_x();
   const int d = a.d, E = geo.E, e0 = (int)rank * E;
   const long long n = a.n_tokens;
@@ -444,6 +423,7 @@ __global__ void __launch_bounds__(NTHR, 1)
   }
   __syncthreads();
   cluster_sync_all();  // every rank's barriers exist (and are armed) before anyone signals them remotely
+  pdl_wait();          // H and y may belong to the kernels before
 
   // a wait that every lane of the warp takes; false (for the whole warp) on
   // time-out or when another warp has given up
@@ -806,8 +786,7 @@ cudaError_t launch_cluster_mr(const ReduceArgs& a, const RedGeo& geo, size_t sme
     cached_clusters = max_clusters;
   }
   const long long ncl = std::min<long long>(max_clusters, geo.nbatch);
-  cfg.gridDim = dim3((unsigned)(ncl * RC));
-  return cudaLaunchKernelEx(&cfg, k, a, geo, *hmap);
+  return launch_kernel(k, dim3((unsigned)(ncl * RC)), dim3(NTHR), smem, s, (unsigned)RC, a, geo, *hmap);
 }
 
 template <int M>

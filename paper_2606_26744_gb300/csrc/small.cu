@@ -53,6 +53,8 @@ __global__ void __launch_bounds__(256) rmsnorm_vec_kernel(const XT* __restrict__
                                                           int block, int vocab) {
   constexpr int XV = 16 / sizeof(XT);  // input elements per 16-byte vector
   __shared__ float sh[32];
+  pdl_launch_dependents();
+  pdl_wait();
   const long long r = blockIdx.x;
   const XT* xr = x + r * d;
   if (EMBED) {  // x is the embedding table here
@@ -113,21 +115,22 @@ cudaError_t launch_norm_t(const void* x, const void* w, void* y, long long rows,
   constexpr int XV = 16 / sizeof(XT);
   const int vpt = (d / XV + 255) / 256;
   const dim3 grid((unsigned)rows);
-#define HDF_NORM_LAUNCH(N)                                                                                  \
-  rmsnorm_vec_kernel<XT, T, N, EMBED><<<grid, 256, 0, s>>>((const XT*)x, (const T*)w, (T*)y, d, eps, anchor, \
-                                                           (const T*)mask_vec, h, block, vocab)
-  if (vpt <= 1) HDF_NORM_LAUNCH(1);
-  else if (vpt <= 2) HDF_NORM_LAUNCH(2);
-  else if (vpt <= 4) HDF_NORM_LAUNCH(4);
-  else if (vpt <= 8) HDF_NORM_LAUNCH(8);
-  else if (vpt <= 16) HDF_NORM_LAUNCH(16);
-  else return cudaErrorInvalidValue;
+#define HDF_NORM_LAUNCH(N)                                                                              \
+  launch_kernel(rmsnorm_vec_kernel<XT, T, N, EMBED>, grid, dim3(256), 0, s, 1u, (const XT*)x, (const T*)w, \
+                (T*)y, d, eps, anchor, (const T*)mask_vec, h, block, vocab)
+  if (vpt <= 1) return HDF_NORM_LAUNCH(1);
+  if (vpt <= 2) return HDF_NORM_LAUNCH(2);
+  if (vpt <= 4) return HDF_NORM_LAUNCH(4);
+  if (vpt <= 8) return HDF_NORM_LAUNCH(8);
+  if (vpt <= 16) return HDF_NORM_LAUNCH(16);
 #undef HDF_NORM_LAUNCH
-  return cudaGetLastError();
+  return cudaErrorInvalidValue;
 }
 
 __global__ void accept_kernel(const int* __restrict__ draft, long long ds, const int* __restrict__ target,
                               long long ts, int batch, int nd, int* __restrict__ accept) {
+  pdl_launch_dependents();
+  pdl_wait();
   const int i = blockIdx.x * blockDim.x + threadIdx.x;
   if (i >= batch) return;
   int n = 0;
@@ -156,6 +159,8 @@ __global__ void lm_reduce_kernel(const float* __restrict__ pmax, const int* __re
                                  float it, int* tok, float* zmax, float* ls) {
   __shared__ MaxArgSum sh[32];
   __shared__ float lse_sh;
+  pdl_launch_dependents();
+  pdl_wait();
   const long long j = blockIdx.x;
   MaxArgSum acc{-INFINITY, INT_MAX, 0.f};
   for (int t = threadIdx.x; t < tiles; t += blockDim.x) {
@@ -222,15 +227,15 @@ cudaError_t launch_embed_norm(const void* embed, const void* mask_vec, const int
 cudaError_t launch_accept(const int* draft, long long ds, const int* target, long long ts, int batch, int nd,
                           int* accept, cudaStream_t s) {
   if (batch == 0) return cudaSuccess;
-  accept_kernel<<<(batch + 127) / 128, 128, 0, s>>>(draft, ds, target, ts, batch, nd, accept);
-  return cudaGetLastError();
+  return launch_kernel(accept_kernel, dim3((batch + 127) / 128), dim3(128), 0, s, 1u, draft, ds, target, ts, batch,
+                       nd, accept);
 }
 
 cudaError_t launch_lm_reduce(const float* pmax, const int* parg, const float* psum, int tiles, long long M,
                              long long V, float it, int* tok, float* zmax, float* ls, cudaStream_t s) {
   if (M == 0) return cudaSuccess;
-  lm_reduce_kernel<<<(unsigned)M, 256, 0, s>>>(pmax, parg, psum, tiles, M, V, it, tok, zmax, ls);
-  return cudaGetLastError();
+  return launch_kernel(lm_reduce_kernel, dim3((unsigned)M), dim3(256), 0, s, 1u, pmax, parg, psum, tiles, M, V, it,
+                       tok, zmax, ls);
 }
 
 }  // namespace hdf
