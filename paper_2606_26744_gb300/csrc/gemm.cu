@@ -42,8 +42,9 @@ template <> struct GT<float> {
 };
 
 constexpr int stages_for(int bn) { return bn >= 256 ? 4 : (bn >= 128 ? 3 : (bn >= 64 ? 4 : 5)); }
-constexpr int kPartialOffset = 8192;  // split-K partial tile in the drained stage memory, above the
-                                      // epilogue's scratch (at most 64 x 17 floats)
+constexpr int kPartialOffset = 8192;  // split-K partial tile, then rank 0's reduced tile, in the drained
+                                      // stage memory above the epilogue's scratch (at most 64 x 17 floats)
+static_assert(kPartialOffset + 2 * 128 * 64 * 4 <= 4 * (128 + 64) * 128, "split-K tiles fit the stages (BN <= 64)");
 constexpr int smem_for(int bn) { return stages_for(bn) * (BM + bn) * ROW_BYTES + 1024; }
 
 __device__ __forceinline__ void operand_rows(const Operand& op, int tile_row0, int half, int tile_idx,
@@ -426,39 +427,55 @@ __global__ void __launch_bounds__(128, 1) gemm_kernel(const __grid_constant__ Ge
       for (int c = 0; c < BN; ++c) part[tid * BN + c] = 0.f;
     }
     cluster_sync_all();  // every rank's partial tile is visible to the cluster
-    if (cluster_rank() == 0) {
-      const uint32_t mine = smem_u32(part + tid * BN);
+    // Every rank sums a slice of the tile's rows over all ranks (one float4
+    // column per thread and round, every source in flight at once, summed in
+    // rank order) and writes the result into rank 0's reduced tile.
+    if (BN <= 64) {
+      const int k = g.k_splits;
+      const uint32_t rank = cluster_rank();
+      const int rpr = (BM + k - 1) / k;  // rows per rank
+      const int row0 = (int)rank * rpr, nrow = max(0, min(BM, row0 + rpr) - row0);
+      constexpr int C4 = BN / 4;
+      const uint32_t part_base = smem_u32(part);
+      const uint32_t red_base = map_rank(smem_u32(smem + kPartialOffset + BM * BN * 4), 0u);
+      for (int it = tid; it < nrow * C4; it += 128) {
+        const int r = row0 + it / C4, c4 = it - (it / C4) * C4;
+        const uint32_t off = (uint32_t)((r * BN + c4 * 4) * 4);
+        float4 q[16];
+#pragma unroll
+        for (int u = 0; u < 16; ++u)
+          if (u < k) q[u] = ld_dsmem_v4(map_rank(part_base + off, (uint32_t)u));
+        float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+        for (int u = 0; u < 16; ++u)
+          if (u < k) {
+            acc.x += q[u].x;
+            acc.y += q[u].y;
+            acc.z += q[u].z;
+            acc.w += q[u].w;
+          }
+        asm volatile("st.shared::cluster.v4.f32 [%0], {%1,%2,%3,%4};" ::"r"(red_base + off), "f"(acc.x),
+                     "f"(acc.y), "f"(acc.z), "f"(acc.w)
+                     : "memory");
+      }
+    }
+    cluster_sync_all();  // rank 0's reduced tile is complete; no rank reads another's memory any more
+    if (cluster_rank() == 0 && !aborted) {
+      const float* red = reinterpret_cast<const float*>(smem + kPartialOffset + BM * BN * 4);
 #pragma unroll 1
       for (int c0 = 0; c0 < BN; c0 += 16) {
         float v[16];
 #pragma unroll
-        for (int i = 0; i < 16; ++i) v[i] = 0.f;
-        // four ranks' rows in flight at a time, summed in rank order
-        for (int r0 = 0; r0 < g.k_splits; r0 += 4) {
-          float4 q[4][4];
-#pragma unroll
-          for (int u = 0; u < 4; ++u)
-            if (r0 + u < g.k_splits) {
-              const uint32_t src = map_rank(mine + c0 * 4, (uint32_t)(r0 + u));
-#pragma unroll
-              for (int i = 0; i < 4; ++i) q[u][i] = ld_dsmem_v4(src + 16 * i);
-            }
-#pragma unroll
-          for (int u = 0; u < 4; ++u)
-            if (r0 + u < g.k_splits) {
-#pragma unroll
-              for (int i = 0; i < 4; ++i) {
-                v[4 * i] += q[u][i].x;
-                v[4 * i + 1] += q[u][i].y;
-                v[4 * i + 2] += q[u][i].z;
-                v[4 * i + 3] += q[u][i].w;
-              }
-            }
+        for (int i = 0; i < 4; ++i) {
+          const float4 q = *reinterpret_cast<const float4*>(red + tid * BN + c0 + 4 * i);
+          v[4 * i] = q.x;
+          v[4 * i + 1] = q.y;
+          v[4 * i + 2] = q.z;
+          v[4 * i + 3] = q.w;
         }
-        if (!aborted) epilogue_chunk<T, BN>(g, tile_m, tile_n, c0, v, smem);
+        epilogue_chunk<T, BN>(g, tile_m, tile_n, c0, v, smem);
       }
     }
-    cluster_sync_all();  // rank 0 has read every rank's shared memory
   }
   tc_fence_before();
   __syncthreads();
@@ -479,7 +496,7 @@ cudaError_t launch_bn(const GemmArgs& g, cudaStream_t s) {
       return e;
     attr_set = true;
   }
-  if (g.k_splits < 1 || g.k_splits > 16) return cudaErrorInvalidValue;
+  if (g.k_splits < 1 || g.k_splits > 16 || (g.k_splits > 1 && BN > 64)) return cudaErrorInvalidValue;
   const long long tiles = (long long)((g.M + BM - 1) / BM) * ((g.N + BN - 1) / BN) * g.k_splits;
   static bool cluster_attr_set = false;
   if (g.k_splits > 8 && !cluster_attr_set) {

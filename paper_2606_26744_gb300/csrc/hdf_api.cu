@@ -128,7 +128,7 @@ SplitPlan plan_swap(int dtype, long long M, long long N, long long K) {
   p.tiles = (int)(((M + 127) / 128) * ((N + p.bn - 1) / p.bn));
   const int num_kb = (int)((K + bk - 1) / bk);
   const int target = 2 * num_sms();
-  int splits = std::max(1, target / p.tiles);
+  int splits = p.bn <= 64 ? std::max(1, target / p.tiles) : 1;  // split tiles are at most 64 wide
   splits = std::min(std::min(splits, 16), std::max(1, num_kb / 4));
   const int kb_per = (num_kb + splits - 1) / splits;
   p.k_splits = (num_kb + kb_per - 1) / kb_per;
