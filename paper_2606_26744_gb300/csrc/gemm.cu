@@ -41,7 +41,7 @@ template <> struct GT<float> {
   static constexpr uint32_t FMT = 2;  // tf32
 };
 
-constexpr int stages_for(int bn) { return bn >= 256 ? 4 : (bn >= 128 ? 3 : (bn >= 64 ? 4 : 5)); }
+constexpr int stages_for(int bn) { return bn >= 256 ? 2 : (bn >= 128 ? 3 : (bn >= 64 ? 4 : 5)); }
 constexpr int kPartialOffset = 8192;  // split-K partial tile, then rank 0's reduced tile, in the drained
                                       // stage memory above the epilogue's scratch (at most 64 x 17 floats)
 static_assert(kPartialOffset + 2 * 128 * 64 * 4 <= 4 * (128 + 64) * 128, "split-K tiles fit the stages (BN <= 64)");
@@ -90,9 +90,11 @@ __device__ __forceinline__ void store16<float>(float* dst, const float* v) {
 
 // Epilogue for one 16-column chunk of the tile.  Called by all 128 threads
 // with identical (tile, c0) so that shuffles and barriers are uniform.
+// rope_row: this thread's row of the RoPE table staged in shared memory
+// (cos of the hd/2 pairs, then sin, see stage_rope_row), or nullptr.
 template <typename T, int BN>
 __device__ __forceinline__ void epilogue_chunk(const GemmArgs& g, int tile_m, int tile_n, int c0,
-                                               float* v, uint8_t* smem) {
+                                               float* v, uint8_t* smem, const float* rope_row = nullptr) {
   const Epilogue& E = g.epi;
   const int row = threadIdx.x;
   const int lane = row & 31, warp = row >> 5;
@@ -104,17 +106,28 @@ __device__ __forceinline__ void epilogue_chunk(const GemmArgs& g, int tile_m, in
       const int seg = col0 / E.seg_width;
       const int fl = col0 - seg * E.seg_width;
       if ((E.rope_mask >> seg) & 1) {
-        const int pos = (int)min((long long)ctx_position(E.cu_ctx, E.batch, t), E.rope_rows - 1);
         const int hh = E.head_dim >> 1;
-        const float* cs = E.rope_cos + (size_t)pos * hh;
-        const float* sn = E.rope_sin + (size_t)pos * hh;
+        const int pi0 = (fl % E.head_dim) >> 1;  // 8 consecutive pairs (16 | head_dim)
+        float c[8], sn[8];
+        if (rope_row) {
+          const float4* cp = reinterpret_cast<const float4*>(rope_row + pi0);
+          const float4* sp = reinterpret_cast<const float4*>(rope_row + hh + pi0);
+          const float4 c0v = cp[0], c1v = cp[1], s0v = sp[0], s1v = sp[1];
+          c[0] = c0v.x; c[1] = c0v.y; c[2] = c0v.z; c[3] = c0v.w; c[4] = c1v.x; c[5] = c1v.y; c[6] = c1v.z; c[7] = c1v.w;
+          sn[0] = s0v.x; sn[1] = s0v.y; sn[2] = s0v.z; sn[3] = s0v.w; sn[4] = s1v.x; sn[5] = s1v.y; sn[6] = s1v.z; sn[7] = s1v.w;
+        } else {
+          const int pos = (int)min((long long)ctx_position(E.cu_ctx, E.batch, t), E.rope_rows - 1);
+#pragma unroll
+          for (int i = 0; i < 8; ++i) {
+            c[i] = __ldg(E.rope_cos + (size_t)pos * hh + pi0 + i);
+            sn[i] = __ldg(E.rope_sin + (size_t)pos * hh + pi0 + i);
+          }
+        }
 #pragma unroll
         for (int i = 0; i < 8; ++i) {
-          const int pi = ((fl + 2 * i) % E.head_dim) >> 1;
-          const float c = __ldg(cs + pi), s = __ldg(sn + pi);
           const float x0 = v[2 * i], x1 = v[2 * i + 1];
-          v[2 * i] = x0 * c - x1 * s;
-          v[2 * i + 1] = x0 * s + x1 * c;
+          v[2 * i] = x0 * c[i] - x1 * sn[i];
+          v[2 * i + 1] = x0 * sn[i] + x1 * c[i];
         }
       }
       store16<T>(reinterpret_cast<T*>(E.out[seg]) + t * E.ld + fl, v);
@@ -262,6 +275,33 @@ __device__ __forceinline__ void epilogue_chunk(const GemmArgs& g, int tile_m, in
   }
 }
 
+// Row-major epilogue with RoPE on the tile's segment: the RoPE table row of
+// this thread's token (cos of the hd/2 pairs, then sin) goes into the
+// drained stage memory with every copy in flight at once.  Rows are
+// 2*(hd/2) + 4 floats apart, so eight threads reading 16 bytes each hit
+// distinct bank groups.  Returns the row, or nullptr when nothing is staged.
+template <int BN>
+__device__ __forceinline__ const float* stage_rope_row(const GemmArgs& g, int tile_m, int tile_n, uint8_t* smem) {
+  const Epilogue& E = g.epi;
+  if (E.kind != kEpiStore || E.head_dim > 128 || E.head_dim % 16) return nullptr;
+  const int seg = (tile_n * BN) / E.seg_width;
+  if (!((E.rope_mask >> seg) & 1)) return nullptr;
+  const int hh = E.head_dim >> 1, stride = 2 * hh + 4;
+  float* row = reinterpret_cast<float*>(smem) + threadIdx.x * stride;
+  const long long t = (long long)tile_m * BM + threadIdx.x;
+  if (t < g.M) {
+    const int pos = (int)min((long long)ctx_position(E.cu_ctx, E.batch, t), E.rope_rows - 1);
+    const float* cs = E.rope_cos + (size_t)pos * hh;
+    const float* sn = E.rope_sin + (size_t)pos * hh;
+    for (int i = 0; i < hh; i += 4) {
+      asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(smem_u32(row + i)), "l"(cs + i) : "memory");
+      asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(smem_u32(row + hh + i)), "l"(sn + i) : "memory");
+    }
+  }
+  asm volatile("cp.async.wait_all;" ::: "memory");
+  return row;  // read back only by this thread
+}
+
 template <typename T, int BN>
 __global__ void __launch_bounds__(128, 1) gemm_kernel(const __grid_constant__ GemmArgs g) {
   constexpr int STAGES = stages_for(BN);
@@ -403,11 +443,13 @@ __global__ void __launch_bounds__(128, 1) gemm_kernel(const __grid_constant__ Ge
   const bool aborted = abort_flag != 0;
   const uint32_t taddr = tmem + ((uint32_t)(warp * 32) << 16);
   if (!aborted && kb1 > kb0 && g.k_splits == 1) {
+    const float* rope_row = BM * (2 * 64 + 4) * 4 <= STAGES * STAGE_BYTES ? stage_rope_row<BN>(g, tile_m, tile_n, smem)
+                                                                           : nullptr;
 #pragma unroll 1
     for (int c0 = 0; c0 < BN; c0 += 16) {
       float v[16];
       tmem_ld16(taddr + c0, v);
-      epilogue_chunk<T, BN>(g, tile_m, tile_n, c0, v, smem);
+      epilogue_chunk<T, BN>(g, tile_m, tile_n, c0, v, smem, rope_row);
     }
   }
   if (g.k_splits > 1) {
