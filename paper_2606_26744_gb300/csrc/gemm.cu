@@ -42,8 +42,8 @@ template <> struct GT<float> {
 };
 
 constexpr int stages_for(int bn) { return bn >= 256 ? 2 : (bn >= 128 ? 3 : (bn >= 64 ? 4 : 5)); }
-constexpr int kPartialOffset = 8192;  // split-K partial tile, then rank 0's reduced tile, in the drained
-                                      // stage memory above the epilogue's scratch (at most 64 x 17 floats)
+constexpr int kPartialOffset = 12288;  // split-K partial tile, then rank 0's reduced tile, in the drained
+                                       // stage memory above the epilogue's scratch (at most 16 x 136 floats)
 static_assert(kPartialOffset + 2 * 128 * 64 * 4 <= 4 * (128 + 64) * 128, "split-K tiles fit the stages (BN <= 64)");
 constexpr int smem_for(int bn) { return stages_for(bn) * (BM + bn) * ROW_BYTES + 1024; }
 
@@ -209,9 +209,12 @@ __device__ __forceinline__ void epilogue_chunk(const GemmArgs& g, int tile_m, in
       return;
     }
     case kEpiLmHeadT: {  // rows = vocabulary entries, columns = tokens
-      float* rmax = reinterpret_cast<float*>(smem);  // [4][16]
-      int* rarg = reinterpret_cast<int*>(smem + 256);
-      float* rsum = reinterpret_cast<float*>(smem + 512);
+      // Per (tile, token): max, first argmax and sum of exp((z - max) * inv_temp)
+      // over the tile's 128 rows.  The chunk goes through shared memory token-
+      // major (row stride 136 floats: the 32 lanes of a read hit 32 banks);
+      // eight threads per token scan 16 rows each in increasing order, then
+      // merge (smaller index on ties).
+      float* tv = reinterpret_cast<float*>(smem);  // [16 tokens][136]
       const long long V = g.M;
       const long long vr = (long long)tile_m * BM + row;
       const bool valid = vr < V;
@@ -221,53 +224,42 @@ __device__ __forceinline__ void epilogue_chunk(const GemmArgs& g, int tile_m, in
         for (int k = 0; k < 16; ++k)
           if (jb + k < g.N) E.logsoftmax[(long long)(jb + k) * V + vr] = v[k] * E.inv_temp;
       }
-      float bv[16];
-      int bi[16];
 #pragma unroll
-      for (int k = 0; k < 16; ++k) {
-        bv[k] = valid ? v[k] : -INFINITY;
-        bi[k] = valid ? (int)vr : INT_MAX;
-      }
-#pragma unroll
-      for (int o = 16; o >= 1; o >>= 1) {
-#pragma unroll
-        for (int k = 0; k < 16; ++k) {
-          const float ov = __shfl_xor_sync(0xffffffffu, bv[k], o);
-          const int oi = __shfl_xor_sync(0xffffffffu, bi[k], o);
-          if (ov > bv[k] || (ov == bv[k] && oi < bi[k])) { bv[k] = ov; bi[k] = oi; }
-        }
-      }
-#pragma unroll
-      for (int k = 0; k < 16; ++k) {
-        float e = valid ? expf((v[k] - bv[k]) * E.inv_temp) : 0.f;
-        e = warp_sum(e);
-        if (lane == k) {
-          rmax[warp * 16 + k] = bv[k];
-          rarg[warp * 16 + k] = bi[k];
-          rsum[warp * 16 + k] = e;
-        }
-      }
+      for (int k = 0; k < 16; ++k) tv[k * 136 + row] = valid ? v[k] : -INFINITY;
       __syncthreads();
-      if (row < 16) {
-        const int k = row, j = jb + k;
-        float m = rmax[k];
-        int a = rarg[k];
-        for (int w = 1; w < 4; ++w) {
-          const float mw = rmax[w * 16 + k];
-          const int aw = rarg[w * 16 + k];
-          if (mw > m || (mw == m && aw < a)) { m = mw; a = aw; }
+      const int k = row >> 3, part = row & 7;
+      const float it = E.inv_temp;
+      float m = -INFINITY, sum = 0.f;
+      int a = INT_MAX;
+#pragma unroll 4
+      for (int i = 0; i < 16; ++i) {
+        const int r = i * 8 + part;  // this thread's rows, increasing
+        const float x = tv[k * 136 + r];
+        if (x > m) {
+          sum = (m == -INFINITY ? 0.f : sum * expf((m - x) * it)) + 1.f;
+          m = x;
+          a = tile_m * BM + r;
+        } else if (x != -INFINITY) {
+          sum += expf((x - m) * it);
         }
-        float s = 0.f;
-        for (int w = 0; w < 4; ++w) {
-          const float mw = rmax[w * 16 + k];
-          if (mw != -INFINITY) s += rsum[w * 16 + k] * expf((mw - m) * E.inv_temp);
-        }
-        if (j < g.N) {
-          const size_t o = (size_t)tile_m * g.N + j;
-          E.part_max[o] = m;
-          E.part_arg[o] = a;
-          E.part_sum[o] = s;
-        }
+      }
+#pragma unroll
+      for (int o = 1; o < 8; o <<= 1) {
+        const float om = __shfl_xor_sync(0xffffffffu, m, o);
+        const int oa = __shfl_xor_sync(0xffffffffu, a, o);
+        const float os = __shfl_xor_sync(0xffffffffu, sum, o);
+        const float nm = fmaxf(m, om);
+        const float fs = m == -INFINITY ? 0.f : sum * expf((m - nm) * it);
+        const float fo = om == -INFINITY ? 0.f : os * expf((om - nm) * it);
+        if (om > m || (om == m && oa < a)) a = oa;
+        m = nm;
+        sum = fs + fo;
+      }
+      if (part == 0 && jb + k < g.N) {
+        const size_t o = (size_t)tile_m * g.N + jb + k;
+        E.part_max[o] = m;
+        E.part_arg[o] = a;
+        E.part_sum[o] = sum;
       }
       __syncthreads();
       return;
