@@ -107,7 +107,7 @@ HDF_API int hdf_gated_reduce(const void* H, int dtype, int64_t n_tokens, int m, 
  * memory and exchange the gate partials over distributed shared memory
  * (bf16, m in {1,2,4}, d % 512 == 0, no alpha_override or path_norm_w; the
  * general kernel runs otherwise).  HDF_REDUCE_AUTO (the default) takes the
- * cluster kernel for m >= 2 and n_tokens >= 8192, where it is faster.
+ * general kernel, the faster of the two on every shape measured.
  * Process-wide; returns HDF_ERR_INVALID_ARG for another value.  The paper
  * has no counterpart: it is a tuning and test hook. */
 enum { HDF_REDUCE_AUTO = 0, HDF_REDUCE_GENERAL = 1, HDF_REDUCE_CLUSTER = 2 };

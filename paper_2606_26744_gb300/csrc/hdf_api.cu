@@ -299,8 +299,7 @@ int hdf_gated_reduce(const void* H, int dtype, int64_t n_tokens, int m, int d, c
   a.status = device_status_ptr();
   unsigned box[3];
   const int path = g_reduce_path.load();
-  const bool cluster_wanted =
-      path == HDF_REDUCE_CLUSTER || (path == HDF_REDUCE_AUTO && m >= 2 && n_tokens >= 8192);
+  const bool cluster_wanted = path == HDF_REDUCE_CLUSTER;  // auto: the general kernel, faster on every shape measured
   if (cluster_wanted && reduce_cluster_box(a, dtype, box)) {
     // 3-D view of H: {64 elements, tokens, 128-byte chunks of a token row}
     auto fn = encode_fn();

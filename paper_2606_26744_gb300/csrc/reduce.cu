@@ -31,6 +31,8 @@ __global__ void __launch_bounds__(512) gated_reduce_kernel(const ReduceArgs a, i
   extern __shared__ __align__(16) uint8_t dyn_smem[];
   __shared__ float red[32][NV];
   __shared__ float fin[NV];
+  __shared__ float bias_s[M];
+  __shared__ float gate_s[G][M][2];  // alpha and the path-norm factor of each (token, path)
 
   const int tid = threadIdx.x, nt = blockDim.x, lane = tid & 31, warp = tid >> 5;
   pdl_launch_dependents();
@@ -49,6 +51,8 @@ __global__ void __launch_bounds__(512) gated_reduce_kernel(const ReduceArgs a, i
     __syncthreads();
     Wf = reinterpret_cast<const T*>(dyn_smem);
   }
+  if (tid < M && use_gate) bias_s[tid] = a.b[tid];
+  __syncthreads();
   pdl_wait();  // H, y and alpha_override may belong to the kernels before
 
   const long long ngroups = (n + G - 1) / G;
@@ -114,39 +118,49 @@ __global__ void __launch_bounds__(512) gated_reduce_kernel(const ReduceArgs a, i
     }
     __syncthreads();
 
-    // ---- gates
-    float alpha[G][M], rp[G][M];
-#pragma unroll
-    for (int g = 0; g < G; ++g) {
+    // ---- gates: one thread per (token, path), shared through shared memory
+    if (tid < G * M) {
+      const int g = tid / M, j = tid - g * M;
       const float* f = fin + g * 2 * M;
       float ss = 0.f;
 #pragma unroll
       for (int p = 0; p < M; ++p) ss += f[M + p];
       const float r = rsqrtf(ss / (float)md + a.rms_eps);
       const long long t = t0 + g;
+      float al;
+      if (a.alpha_override) {
+        al = (t < n) ? a.alpha_override[t * M + j] : 0.f;
+      } else {
+        const float logit = a.gate_scale * r * f[j] + bias_s[j];
+        al = 1.0f / (1.0f + expf(-logit)) + a.gate_offset;
+      }
+      gate_s[g][j][0] = al;
+      gate_s[g][j][1] = a.path_norm_w ? rsqrtf(f[M + j] / (float)d + a.path_norm_eps) : 1.f;
+      if (a.alpha_out && t < n) a.alpha_out[t * M + j] = al;
+    }
+    __syncthreads();
+    float alpha[G][M], rp[G][M];
+#pragma unroll
+    for (int g = 0; g < G; ++g)
 #pragma unroll
       for (int j = 0; j < M; ++j) {
-        if (a.alpha_override) {
-          alpha[g][j] = (t < n) ? a.alpha_override[t * M + j] : 0.f;
-        } else {
-          const float logit = a.gate_scale * r * f[j] + a.b[j];
-          alpha[g][j] = 1.0f / (1.0f + expf(-logit)) + a.gate_offset;
-        }
-        rp[g][j] = a.path_norm_w ? rsqrtf(f[M + j] / (float)d + a.path_norm_eps) : 1.f;
+        alpha[g][j] = gate_s[g][j][0];
+        rp[g][j] = gate_s[g][j][1];
       }
-      if (a.alpha_out && tid < M && t < n) {
-#pragma unroll
-        for (int j = 0; j < M; ++j)
-          if (j == tid) a.alpha_out[t * M + j] = alpha[g][j];
-      }
-    }
 
-    // ---- phase 2: weighted sum over paths (H re-read from L2), one store
+    // ---- phase 2: weighted sum over paths (H re-read from L2), one store;
+    // every load of a vector's G x M values is issued before its stores
     const T* pnw = reinterpret_cast<const T*>(a.path_norm_w);
-    T* y = reinterpret_cast<T*>(a.y);
+    T* __restrict__ y = reinterpret_cast<T*>(a.y);
     for (int k = 0; k < vpt; ++k) {
       const int v = tid + k * nt;
       if (v >= nvec) continue;
+      uint4 raw[G][M];
+#pragma unroll
+      for (int g = 0; g < G; ++g)
+#pragma unroll
+        for (int p = 0; p < M; ++p)
+          raw[g][p] = t0 + g < n ? ld_nc16(H + (t0 + g) * md + p * d + v * VEC) : make_uint4(0, 0, 0, 0);
 #pragma unroll
       for (int g = 0; g < G; ++g) {
         const long long t = t0 + g;
@@ -157,7 +171,7 @@ __global__ void __launch_bounds__(512) gated_reduce_kernel(const ReduceArgs a, i
 #pragma unroll
         for (int p = 0; p < M; ++p) {
           float h[VEC];
-          V16<T>::unpack(ld_nc16(H + t * md + p * d + v * VEC), h);
+          V16<T>::unpack(raw[g][p], h);
           if (pnw) {
             float gm[VEC];
             V16<T>::unpack(ld_nc16(pnw + p * d + v * VEC), gm);
@@ -190,21 +204,18 @@ cudaError_t launch_m(const ReduceArgs& a, cudaStream_t s) {
   if ((e = cudaGetDevice(&dev)) != cudaSuccess) return e;
   if ((e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev)) != cudaSuccess) return e;
   const long long ngroups = (a.n_tokens + G - 1) / G;
-  if (wf_smem) {
-    auto k = gated_reduce_kernel<T, M, G, true>;
-    if ((e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)wf_bytes)) != cudaSuccess)
-      return e;
-    if ((e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, k, nt, wf_bytes)) != cudaSuccess) return e;
+  auto go = [&](auto k, size_t smem) -> cudaError_t {
+    cudaError_t e2;
+    if (smem > 48 * 1024 &&
+        (e2 = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem)) != cudaSuccess)
+      return e2;
+    if ((e2 = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, k, nt, smem)) != cudaSuccess) return e2;
     if (per_sm < 1) per_sm = 1;
     const long long grid = std::min<long long>(ngroups, (long long)per_sm * sms);
-    return launch_kernel(k, dim3((unsigned)grid), dim3(nt), wf_bytes, s, 1u, a, vpt);
-  } else {
-    auto k = gated_reduce_kernel<T, M, G, false>;
-    if ((e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, k, nt, 0)) != cudaSuccess) return e;
-    if (per_sm < 1) per_sm = 1;
-    const long long grid = std::min<long long>(ngroups, (long long)per_sm * sms);
-    return launch_kernel(k, dim3((unsigned)grid), dim3(nt), 0, s, 1u, a, vpt);
-  }
+    return launch_kernel(k, dim3((unsigned)grid), dim3(nt), smem, s, 1u, a, vpt);
+  };
+  if (wf_smem) return go(gated_reduce_kernel<T, M, G, true>, wf_bytes);
+  return go(gated_reduce_kernel<T, M, G, false>, 0);
 }
 
 template <typename T>
