@@ -277,6 +277,32 @@ def run_ours(args, rank, world, local_rank):
         raise RuntimeError(f"stage times ({sum(dur.values()):.4f} ms) exceed the step time ({ms_staged:.4f} ms): "
                            "the step timer does not bracket the work")
 
+    # ------------------------------------------------ KL target (Eq. 2)
+    # teacher / student log-softmax rows of the first P = 2 block positions
+    # of every sequence, as the LM head writes them; timed alone (it is a
+    # training-time quantity, not part of the draft step)
+    kl_rows_n, V = batch * 2, cfg.vocab
+    gk = torch.Generator(device=dev).manual_seed(seed + 7)
+    ls_t = torch.log_softmax(torch.randn(kl_rows_n, V, device=dev, generator=gk) * 3, dim=1)
+    ls_s = torch.log_softmax(torch.randn(kl_rows_n, V, device=dev, generator=gk) * 3, dim=1)
+    klr = torch.empty(kl_rows_n, device=dev)
+    klm = torch.empty(1, device=dev)
+    klws = torch.empty(max(1, hdf.load().hdf_kl_distill_workspace_size(kl_rows_n, V)), dtype=torch.uint8, device=dev)
+    for _ in range(3):
+        hdf.hdf_kl_distill(ls_t, ls_s, t_kd=1.0, kl_rows=klr, kl_mean=klm, ws=klws, stream=stream)
+    stream.synchronize()
+    k0 = torch.cuda.Event(enable_timing=True)
+    k1 = torch.cuda.Event(enable_timing=True)
+    k0.record(stream)
+    for _ in range(20):
+        hdf.hdf_kl_distill(ls_t, ls_s, t_kd=1.0, kl_rows=klr, kl_mean=klm, ws=klws, stream=stream)
+    k1.record(stream)
+    stream.synchronize()
+    kl_us = k0.elapsed_time(k1) / 20 * 1000
+    kl = {"rows": kl_rows_n, "vocab": V, "us": round(kl_us, 2),
+          "gbs": round(2 * kl_rows_n * V * 4 / kl_us / 1e3, 1), "launches": 2}
+    del ls_t, ls_s
+
     # ------------------------------------------------------------ e2e
     # host buffers: the residual of every context token and the targets in,
     # drafts and accepted lengths out, through the same C-ABI calls.
@@ -313,7 +339,7 @@ def run_ours(args, rank, world, local_rank):
         t = torch.tensor([ms, e2e_ms], device=dev)
         torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
         ms, e2e_ms = float(t[0]), float(t[1])
-    return dict(cfg=cfg, ms=ms, ms_staged=ms_staged, e2e_ms=e2e_ms, dur=dur, clk=clk, batch=batch, n_ctx=n_ctx, lens=lens,
+    return dict(cfg=cfg, ms=ms, ms_staged=ms_staged, e2e_ms=e2e_ms, dur=dur, clk=clk, kl=kl, batch=batch, n_ctx=n_ctx, lens=lens,
                 h2d=h2d, d2h=d2h, acc_mean=acc_mean, tok=tok, y=y, inputs=inp, tgt=tgt)
 
 
@@ -555,6 +581,7 @@ def main():
             "ms_per_step_instrumented": round(res["ms_staged"], 5),
             "roofline": rf,
             "reducer": {"gbs": red.get("gbs"), "frac_hbm": red.get("frac"), "us": red["us"]},
+            "kl_target": dict(res["kl"], frac_hbm=round(res["kl"]["gbs"] / pk["hbm_gbs"], 3)),
             "stages": stages,
             "e2e": {"value": round(e2e_val, 2), "unit": "blocks/s", "h2d_bytes_per_step": res["h2d"],
                     "d2h_bytes_per_step": res["d2h"]},

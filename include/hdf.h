@@ -8,6 +8,7 @@
  *   hdf_lm_head_argmax  Sec. 2.3: logits, argmax drafts, optional log-softmax
  *                       at temperature T_KD (the q^{T_KD} of Eq. 2)
  *   hdf_accept_len      Sec. 3.4: accepted-prefix length of each block
+ * and, for training-time distillation, hdf_kl_distill (Eq. 2, Sec. 2.3).
  *
  * Conventions shared by every call
  *   - All tensor arguments are DEVICE pointers owned by the caller, row-major,
@@ -261,6 +262,31 @@ HDF_API int hdf_lm_head_argmax_static(const void* h, int dtype, int64_t M, int d
 HDF_API int hdf_accept_len(const int32_t* draft, int64_t draft_stride,
                    const int32_t* target, int64_t target_stride,
                    int batch, int n_draft, int32_t* accept, hdf_stream_t stream);
+
+/* ------------------------------------------------------------------------
+ * (5) KL distillation target — Eq. 2 (Sec. 2.3):
+ *   kl_rows[r] = KL(p_r || q_r) = sum_v p_r(v) * (ls_teacher[r][v] - ls_student[r][v])
+ *   kl_mean    = t_kd^2 / rows * sum_r kl_rows[r]
+ * where p_r = exp(ls_teacher[r]) and both inputs are log-softmax rows at
+ * temperature t_kd, as hdf_lm_head_argmax writes them with inv_temp =
+ * 1 / t_kd (teacher: the target LM head on the path-mean residual, which
+ * hdf_gated_reduce gives with alpha_override = 1/m; student: the draft
+ * logits of the first P block positions).  For a batch of blocks with P rows
+ * each, kl_mean is the batch mean of L_KL.  L = L_CE + alpha * L_KL (Eq. 3)
+ * is left to the caller.
+ *   ls_teacher, ls_student  [rows, V] fp32 (device), rows >= 0, V >= 1
+ *   kl_rows                 [rows] fp32 or NULL
+ *   kl_mean                 [1] fp32 or NULL
+ *   ws / ws_bytes           scratch of hdf_kl_distill_workspace_size(rows, V)
+ *                           bytes, 256-byte aligned
+ * Teacher entries of -inf contribute 0; a student -inf where the teacher
+ * is finite gives +inf.  The sums run in a fixed order (bitwise
+ * reproducible).  rows == 0 launches nothing.
+ * ---------------------------------------------------------------------- */
+HDF_API size_t hdf_kl_distill_workspace_size(int64_t rows, int64_t V);
+HDF_API int hdf_kl_distill(const float* ls_teacher, const float* ls_student, int64_t rows, int64_t V,
+                           float t_kd, float* kl_rows, float* kl_mean, void* ws, size_t ws_bytes,
+                           hdf_stream_t stream);
 
 #ifdef __cplusplus
 }

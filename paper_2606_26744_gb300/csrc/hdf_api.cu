@@ -657,6 +657,30 @@ int hdf_lm_head_argmax(const void* h, int dtype, int64_t M, int d, const void* W
   return HDF_OK;
 }
 
+// ----------------------------------------------------- KL distillation
+size_t hdf_kl_distill_workspace_size(int64_t rows, int64_t V) {
+  if (rows <= 0 || V <= 0) return 0;
+  return up256((size_t)rows * kl_chunks(V) * 4);
+}
+
+int hdf_kl_distill(const float* ls_teacher, const float* ls_student, int64_t rows, int64_t V, float t_kd,
+                   float* kl_rows, float* kl_mean, void* ws, size_t ws_bytes, hdf_stream_t stream) {
+  g_err.clear();
+  if (rows < 0 || V <= 0 || rows > 65535 || V > ((int64_t)1 << 40)) return fail(HDF_ERR_SHAPE, "rows / V");
+  if (!(t_kd > 0) || !std::isfinite(t_kd)) return fail(HDF_ERR_INVALID_ARG, "t_kd must be > 0");
+  if (rows == 0) return HDF_OK;
+  if (!ls_teacher || !ls_student) return fail(HDF_ERR_INVALID_ARG, "ls_teacher and ls_student are required");
+  if (!aligned16(ls_teacher) || !aligned16(ls_student))
+    return fail(HDF_ERR_ALIGNMENT, "ls_teacher and ls_student must be 16-byte aligned");
+  const size_t need = hdf_kl_distill_workspace_size(rows, V);
+  if (!ws || ws_bytes < need || (reinterpret_cast<uintptr_t>(ws) & 255))
+    return fail(HDF_ERR_WORKSPACE, "workspace %zu bytes (need %zu, 256-byte aligned)", ws_bytes, need);
+  CK(launch_kl_distill(ls_teacher, ls_student, rows, V, t_kd, kl_rows, kl_mean, static_cast<float*>(ws),
+                       (cudaStream_t)stream),
+     "kl distill");
+  return HDF_OK;
+}
+
 // ------------------------------------------ LM head on library-owned scratch
 // For callers that cannot allocate device memory themselves: the LM head's
 // scratch (per-tile argmax / sum-exp partials) lives in this file-scope device array instead of a caller

@@ -133,6 +133,13 @@ cudaError_t launch_lm_reduce(const float* part_max, const int* part_arg, const f
                              int tiles, long long M, long long V, float inv_temp, int* tok,
                              float* zmax, float* logsoftmax, cudaStream_t s);
 
+// --------------------------------------------------------------- KL ----
+constexpr int KL_CHUNK = 8192;  // vocabulary entries per CTA of the partial-sum stage
+int kl_chunks(long long V);
+// partial: [rows, kl_chunks(V)] fp32 scratch
+cudaError_t launch_kl_distill(const float* lt, const float* ls, long long rows, long long V, float t_kd,
+                              float* kl_rows, float* kl_mean, float* partial, cudaStream_t s);
+
 // -------------------------------------------------------- attention ----
 struct AttnArgs {
   const void* q;       // [M, d]  block queries (M = batch * block)

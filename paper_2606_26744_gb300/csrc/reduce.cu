@@ -29,7 +29,7 @@ __global__ void __launch_bounds__(512) gated_reduce_kernel(const ReduceArgs a, i
   constexpr int NV = next_pow2(G * 2 * M);  // reduced values per token group (padded)
   static_assert(NV <= 32, "reduction values must fit one warp");
   extern __shared__ __align__(16) uint8_t dyn_smem[];
-  __shared__ float red[32][NV];
+  __shared__ float red[16][NV];  // one row per warp (at most 512 threads)
   __shared__ float fin[NV];
   __shared__ float bias_s[M];
   __shared__ float gate_s[G][M][2];  // alpha and the path-norm factor of each (token, path)
@@ -198,6 +198,8 @@ cudaError_t launch_m(const ReduceArgs& a, cudaStream_t s) {
   int nt = (nvec + vpt - 1) / vpt;
   nt = ((nt + 31) / 32) * 32;
   const size_t wf_bytes = (size_t)M * M * a.d * sizeof(T);
+  // W_f in shared memory up to 160 KB: larger (m = 4, d = 7168) would leave
+  // one CTA per SM, which costs more than reading W_f through L1 / L2
   const bool wf_smem = wf_bytes <= 160 * 1024 && a.alpha_override == nullptr;
   int dev = 0, sms = 0, per_sm = 0;
   cudaError_t e;

@@ -75,6 +75,8 @@ _SIGS = {
     "hdf_lm_head_argmax_static": (c_int, [c_vp, c_int, c_i64, c_int, c_vp, c_i64, c_float, c_vp, c_vp, c_vp,
                                           c_vp]),
     "hdf_set_reduce_path": (c_int, [c_int]),
+    "hdf_kl_distill_workspace_size": (c_size, [c_i64, c_i64]),
+    "hdf_kl_distill": (c_int, [c_vp, c_vp, c_i64, c_i64, c_float, c_vp, c_vp, c_vp, c_size, c_vp]),
 }
 
 _lib = None
@@ -294,3 +296,24 @@ def hdf_accept_len(draft: torch.Tensor, target: torch.Tensor, *, n_draft: Option
     _check(load().hdf_accept_len(_p(draft), draft_stride, _p(target), target.stride(0), batch, n_draft,
                                  _p(accept), _stream(stream)))
     return accept
+
+
+# ---------------------------------------------------------- KL distillation
+def hdf_kl_distill(ls_teacher: torch.Tensor, ls_student: torch.Tensor, *, t_kd: float = 1.0,
+                   kl_rows: Optional[torch.Tensor] = None, kl_mean: Optional[torch.Tensor] = None,
+                   ws: Optional[torch.Tensor] = None, stream=None):
+    """Eq. 2: per-row KL(p || q) of two [rows, V] fp32 log-softmax arrays at
+    temperature t_kd, and t_kd^2 / rows * their sum."""
+    rows, V = ls_teacher.shape
+    dev = ls_teacher.device
+    if kl_rows is None:
+        kl_rows = torch.empty((rows,), dtype=torch.float32, device=dev)
+    if kl_mean is None:
+        kl_mean = torch.empty((1,), dtype=torch.float32, device=dev)
+    lib = load()
+    need = lib.hdf_kl_distill_workspace_size(rows, V)
+    if ws is None:
+        ws = torch.empty(max(need, 1), dtype=torch.uint8, device=dev)
+    _check(lib.hdf_kl_distill(_p(ls_teacher), _p(ls_student), rows, V, t_kd, _p(kl_rows), _p(kl_mean), _p(ws),
+                              ws.numel(), _stream(stream)))
+    return kl_rows, kl_mean

@@ -57,6 +57,16 @@ def test_reduce_path_switch(lib):
         assert lib.hdf_set_reduce_path(path) == 0
 
 
+def test_kl_host_validation(lib):
+    v = ctypes.c_void_p
+    assert lib.hdf_kl_distill(v(16), v(16), 2, 100, 0.0, None, None, v(256), 4096, None) == 1   # t_kd <= 0
+    assert lib.hdf_kl_distill(v(16), v(16), -1, 100, 1.0, None, None, v(256), 4096, None) == 2  # rows < 0
+    assert lib.hdf_kl_distill(None, None, 0, 100, 1.0, None, None, None, 0, None) == 0         # empty
+    assert lib.hdf_kl_distill(v(16), v(24), 2, 100, 1.0, None, None, v(256), 4096, None) == 4  # alignment
+    assert lib.hdf_kl_distill(v(16), v(16), 2, 100, 1.0, None, None, None, 0, None) == 5       # workspace
+    assert lib.hdf_kl_distill_workspace_size(2, 8193) == 256                                   # 2 x 2 partials
+
+
 def test_lm_head_and_accept_host_validation(lib):
     v = ctypes.c_void_p
     assert lib.hdf_lm_head_argmax(v(16), 9, 4, 64, v(16), 100, 1.0, v(16), None, None, v(256), 1 << 20, None) == 3
