@@ -20,6 +20,8 @@ Passages followed (HyperDFlash paper):
   * Sec. 2.1 / 2.3: anchor-plus-mask block, draft slot k predicts a+k.
   * Sec. 2.3, Eq. 2: log-softmax at temperature T_KD for the KL target.
   * Sec. 3.4: accepted length; tau counts the bonus token.
+  * Sec. 1 / Tables 2-3 (T = 1 rows): speculative-sampling verification,
+    accept with probability min(1, p/q) and resample from max(0, p - q).
 
 Readings of passages the paper leaves open are listed in the design notes;
 the ones used here are: RMSNorm over all m*d entries with eps and no weight
@@ -299,6 +301,68 @@ def accept_len(draft, target) -> np.ndarray:
             n += 1
         out[i] = n
     return out
+
+
+def accept_sample(p_target, q_draft, draft, u, r):
+    """Temperature-1 verification of one drafted block per sequence by
+    speculative sampling (the T = 1 rows of Tables 2 and 3; the rule is the
+    standard one the paper relies on without restating it):
+      * draft slot k is accepted when u[i,k] / 2^32 < p(x) / q(x), x = draft[i,k],
+        with the ratio one IEEE fp32 division; the first rejection ends the block;
+      * the next token is drawn from norm(max(0, p - q)) at the rejected slot
+        (from p there if that residual is empty), or from p at the bonus slot
+        n_draft when every draft is accepted;
+      * the draw is an inverse-CDF lookup with the 32-bit uniform r[i] over
+        integer weights floor(w * 2^40): the first v whose prefix sum exceeds
+        floor(r * R / 2^32), R = total weight (exact integer arithmetic).
+    p_target [batch, n_draft + 1, V], q_draft [batch, n_draft, V] float32
+    probabilities; draft [batch, n_draft] ids; u [batch, n_draft], r [batch]
+    uint32.  Returns (accept [batch], next [batch]); next = -1 when the chosen
+    distribution has no weight at all (invalid input)."""
+    p_target = np.asarray(p_target, dtype=np.float32)
+    q_draft = np.asarray(q_draft, dtype=np.float32)
+    draft = np.asarray(draft)
+    u = np.asarray(u, dtype=np.uint64)
+    r = np.asarray(r, dtype=np.uint64)
+    batch, nd = draft.shape
+    acc = np.zeros(batch, dtype=np.int64)
+    nxt = np.zeros(batch, dtype=np.int64)
+
+    def draw(w32, ri):
+        wi = [int(np.floor(float(x) * 2.0 ** 40)) for x in w32]   # exact: w <= 1, float64 product exact
+        total = sum(wi)
+        if total == 0:
+            return None
+        thr = (int(ri) * total) >> 32
+        run = 0
+        for v, x in enumerate(wi):
+            run += x
+            if run > thr:
+                return v
+        return len(wi) - 1
+
+    for i in range(batch):
+        n = 0
+        while n < nd:
+            x = int(draft[i, n])
+            if x < 0 or x >= p_target.shape[2]:   # an id outside the vocabulary is rejected
+                break
+            with np.errstate(divide="ignore", invalid="ignore"):   # p/0 = inf (accept), 0/0 = nan (reject)
+                ratio = np.float32(p_target[i, n, x]) / np.float32(q_draft[i, n, x])   # IEEE fp32 division
+            if float(u[i, n]) / 2.0 ** 32 < float(ratio):
+                n += 1
+            else:
+                break
+        acc[i] = n
+        if n < nd:
+            res = np.maximum(p_target[i, n] - q_draft[i, n], np.float32(0))      # fp32 subtraction
+            v = draw(res, r[i])
+            if v is None:
+                v = draw(p_target[i, n], r[i])
+        else:
+            v = draw(p_target[i, nd], r[i])
+        nxt[i] = -1 if v is None else v
+    return acc, nxt
 
 
 def mean_accepted_length(accept) -> float:

@@ -384,3 +384,58 @@ def test_kl_pins():
     # T^2 factor: logits scaled with T keep p, q fixed, loss scales by T^2
     np.testing.assert_allclose(O.kl_distill(2 * t, 2 * s, 2.0),
                                4 * O.kl_distill(t, s, 1.0), rtol=1e-13)
+
+
+# ---------------------------------------------- speculative-sampling verification
+def _dist(rng, V):
+    w = rng.random(V).astype(np.float64) + 0.05
+    return (w / w.sum()).astype(np.float32)
+
+
+def test_accept_sample_output_is_distributed_as_p():
+    """The defining property of speculative sampling: with x ~ q, accept with
+    probability min(1, p(x)/q(x)), else draw from norm(max(0, p - q)), the
+    emitted token is distributed exactly as p.  Integrated over dense grids of
+    the two uniforms (u, r) and exactly over x."""
+    rng = np.random.default_rng(5)
+    V, G = 5, 96
+    p0, q0 = _dist(rng, V), _dist(rng, V)
+    grid = ((np.arange(G) + 0.5) * 2.0 ** 32 / G).astype(np.uint64)
+    freq = np.zeros(V)
+    for x in range(V):
+        # batch over (u, r) pairs for this drafted x
+        uu, rr = np.meshgrid(grid, grid, indexing="ij")
+        n = uu.size
+        p = np.broadcast_to(np.stack([p0, p0])[None], (n, 2, V))
+        q = np.broadcast_to(q0[None, None], (n, 1, V))
+        acc, nxt = O.accept_sample(p, q, np.full((n, 1), x), uu.reshape(n, 1), rr.reshape(n))
+        first = np.where(acc == 1, x, nxt)
+        freq += q0[x] * np.bincount(first, minlength=V) / n
+    np.testing.assert_allclose(freq, p0, atol=2.5 / G)
+
+
+def test_accept_sample_special_cases():
+    rng = np.random.default_rng(6)
+    V, nd = 7, 4
+    p = np.stack([_dist(rng, V) for _ in range(nd + 1)])[None]
+    u = np.full((1, nd), 2 ** 32 - 1, dtype=np.uint64)          # the largest uniform
+    acc, nxt = O.accept_sample(p, p[:, :nd], np.zeros((1, nd), int), u, np.array([0]))
+    assert acc[0] == nd and nxt[0] == 0                          # q == p: ratio 1 > u, bonus from p[nd]
+    q1 = np.zeros((1, nd, V), np.float32); q1[:, :, 2] = 1       # draft certain of token 2
+    p1 = np.zeros((1, nd + 1, V), np.float32); p1[:, :, 5] = 1   # target certain of token 5
+    acc, nxt = O.accept_sample(p1, q1, np.full((1, nd), 2), np.zeros((1, nd), np.uint64), np.array([123]))
+    assert acc[0] == 0 and nxt[0] == 5                           # p/q = 0: rejected, residual = p
+    acc, _ = O.accept_sample(p, p[:, :nd], np.array([[0, 1, V, 2]]), u, np.array([0]))
+    assert acc[0] == 2                                           # an id outside the vocabulary is rejected
+
+
+def test_accept_sample_inverse_cdf_boundaries():
+    # uniform residual over 4 tokens: weights 2^38 each, R = 2^40, threshold = r * 2^8
+    p = np.zeros((1, 2, 4), np.float32); p[0, 0] = 0.25
+    q = np.zeros((1, 1, 4), np.float32)
+    draft = np.array([[0]])
+    u = np.array([[2 ** 32 - 1]], dtype=np.uint64)                # p/q = inf: accepted ... so use p at slot 1
+    p[0, 1] = 0.25
+    for r, want in [(0, 0), (2 ** 30 - 1, 0), (2 ** 30, 1), (2 ** 31, 2), (2 ** 32 - 1, 3)]:
+        _, nxt = O.accept_sample(p, q, draft, u, np.array([r], dtype=np.uint64))
+        assert nxt[0] == want, (r, nxt[0])
