@@ -303,6 +303,30 @@ def run_ours(args, rank, world, local_rank):
           "gbs": round(2 * kl_rows_n * V * 4 / kl_us / 1e3, 1), "launches": 2}
     del ls_t, ls_s
 
+    # ------------------------------------ T = 1 verification (speculative sampling)
+    # target / draft probabilities of every block slot, drafts sampled from q,
+    # uniforms as 32-bit integers; timed alone like the KL target
+    nd = B - 1
+    pv = torch.softmax(torch.randn(batch, B, V, device=dev, generator=gk) * 2, dim=-1)
+    qv = torch.softmax(0.7 * torch.log(pv[:, :nd]) + 0.3 * torch.randn(batch, nd, V, device=dev, generator=gk), -1)
+    dr = torch.multinomial(qv.reshape(-1, V), 1, generator=gk).view(batch, nd).to(torch.int32)
+    uv = torch.randint(-2 ** 31, 2 ** 31 - 1, (batch, nd), device=dev, dtype=torch.int32, generator=gk)
+    rv = torch.randint(-2 ** 31, 2 ** 31 - 1, (batch,), device=dev, dtype=torch.int32, generator=gk)
+    va = torch.empty(batch, dtype=torch.int32, device=dev)
+    vn = torch.empty(batch, dtype=torch.int32, device=dev)
+    for _ in range(3):
+        hdf.hdf_accept_sample(pv, qv, dr, uv, rv, accept=va, next_tok=vn, stream=stream)
+    stream.synchronize()
+    k0.record(stream)
+    for _ in range(20):
+        hdf.hdf_accept_sample(pv, qv, dr, uv, rv, accept=va, next_tok=vn, stream=stream)
+    k1.record(stream)
+    stream.synchronize()
+    v_us = k0.elapsed_time(k1) / 20 * 1000
+    verify_t1 = {"batch": batch, "n_draft": nd, "vocab": V, "us": round(v_us, 2),
+                 "mean_accept": round(float(va.float().mean()), 3), "launches": 1}
+    del pv, qv
+
     # ------------------------------------------------------------ e2e
     # host buffers: the residual of every context token and the targets in,
     # drafts and accepted lengths out, through the same C-ABI calls.
@@ -339,7 +363,7 @@ def run_ours(args, rank, world, local_rank):
         t = torch.tensor([ms, e2e_ms], device=dev)
         torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
         ms, e2e_ms = float(t[0]), float(t[1])
-    return dict(cfg=cfg, ms=ms, ms_staged=ms_staged, e2e_ms=e2e_ms, dur=dur, clk=clk, kl=kl, batch=batch, n_ctx=n_ctx, lens=lens,
+    return dict(cfg=cfg, ms=ms, ms_staged=ms_staged, e2e_ms=e2e_ms, dur=dur, clk=clk, kl=kl, verify_t1=verify_t1, batch=batch, n_ctx=n_ctx, lens=lens,
                 h2d=h2d, d2h=d2h, acc_mean=acc_mean, tok=tok, y=y, inputs=inp, tgt=tgt)
 
 
@@ -582,6 +606,7 @@ def main():
             "roofline": rf,
             "reducer": {"gbs": red.get("gbs"), "frac_hbm": red.get("frac"), "us": red["us"]},
             "kl_target": dict(res["kl"], frac_hbm=round(res["kl"]["gbs"] / pk["hbm_gbs"], 3)),
+            "verify_t1": res["verify_t1"],
             "stages": stages,
             "e2e": {"value": round(e2e_val, 2), "unit": "blocks/s", "h2d_bytes_per_step": res["h2d"],
                     "d2h_bytes_per_step": res["d2h"]},

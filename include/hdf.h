@@ -8,7 +8,8 @@
  *   hdf_lm_head_argmax  Sec. 2.3: logits, argmax drafts, optional log-softmax
  *                       at temperature T_KD (the q^{T_KD} of Eq. 2)
  *   hdf_accept_len      Sec. 3.4: accepted-prefix length of each block
- * and, for training-time distillation, hdf_kl_distill (Eq. 2, Sec. 2.3).
+ * hdf_accept_sample is the temperature-1 (sampling) form of step 4, and
+ * hdf_kl_distill the training-time distillation target (Eq. 2, Sec. 2.3).
  *
  * Conventions shared by every call
  *   - All tensor arguments are DEVICE pointers owned by the caller, row-major,
@@ -262,6 +263,32 @@ HDF_API int hdf_lm_head_argmax_static(const void* h, int dtype, int64_t M, int d
 HDF_API int hdf_accept_len(const int32_t* draft, int64_t draft_stride,
                    const int32_t* target, int64_t target_stride,
                    int batch, int n_draft, int32_t* accept, hdf_stream_t stream);
+
+/* ------------------------------------------------------------------------
+ * (4') Temperature-1 block verification by speculative sampling (the T = 1
+ * rows of Tables 2 and 3; the paper uses the standard rule without
+ * restating it).  For sequence i:
+ *   draft slot k (k = 0, 1, ...) is accepted when u[i][k] / 2^32 < p / q with
+ *   p = p_target[i][k][x], q = q_draft[i][k][x], x = draft[i][k], the ratio
+ *   one IEEE fp32 division (q = 0 accepts, 0/0 rejects, x outside [0, V)
+ *   rejects); the first rejection ends the block:  accept[i] = slots accepted.
+ *   next_tok[i] is drawn from norm(max(0, p - q)) at the rejected slot (from p
+ *   there if that residual is empty), or from p_target[i][n_draft] (the bonus
+ *   slot) when every draft is accepted: the first v whose prefix sum of
+ *   floor(w * 2^40) exceeds floor(r[i] * R / 2^32), R the total (exact
+ *   integer arithmetic); -1 when the distribution has no weight.
+ *   p_target [batch, n_draft + 1, V]  fp32 probabilities (target model, T = 1)
+ *   q_draft  [batch, n_draft, V]      fp32 probabilities (drafter)
+ *   draft    row i at draft + i*draft_stride (e.g. hdf_lm_head_argmax's tok
+ *            + 1 with stride B, or sampled drafts)
+ *   u [batch, n_draft], r [batch]     uint32 uniforms, drawn by the caller
+ *   1 <= V <= 2^22, n_draft >= 0; batch == 0 launches nothing.
+ * Every decision is exact: the same inputs give the same accept / next_tok.
+ * ---------------------------------------------------------------------- */
+HDF_API int hdf_accept_sample(const float* p_target, const float* q_draft, const int32_t* draft,
+                              int64_t draft_stride, const uint32_t* u, const uint32_t* r, int batch,
+                              int n_draft, int64_t V, int32_t* accept, int32_t* next_tok,
+                              hdf_stream_t stream);
 
 /* ------------------------------------------------------------------------
  * (5) KL distillation target — Eq. 2 (Sec. 2.3):

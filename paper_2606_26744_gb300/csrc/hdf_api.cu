@@ -657,6 +657,23 @@ int hdf_lm_head_argmax(const void* h, int dtype, int64_t M, int d, const void* W
   return HDF_OK;
 }
 
+// ------------------------------------------------ T = 1 verification
+int hdf_accept_sample(const float* p_target, const float* q_draft, const int32_t* draft, int64_t draft_stride,
+                      const uint32_t* u, const uint32_t* r, int batch, int n_draft, int64_t V, int32_t* accept,
+                      int32_t* next_tok, hdf_stream_t stream) {
+  g_err.clear();
+  if (batch < 0 || n_draft < 0 || V < 1 || V > ((int64_t)1 << 22))
+    return fail(HDF_ERR_SHAPE, "batch / n_draft / V (1..2^22)");
+  if (batch == 0) return HDF_OK;
+  if (n_draft > 0 && draft_stride < n_draft) return fail(HDF_ERR_SHAPE, "draft_stride < n_draft");
+  if (!p_target || !r || !accept || !next_tok || (n_draft > 0 && (!q_draft || !draft || !u)))
+    return fail(HDF_ERR_INVALID_ARG, "null pointer");
+  CK(launch_accept_sample(p_target, q_draft, draft, draft_stride, u, r, batch, n_draft, V, accept, next_tok,
+                          (cudaStream_t)stream),
+     "accept sample");
+  return HDF_OK;
+}
+
 // ----------------------------------------------------- KL distillation
 size_t hdf_kl_distill_workspace_size(int64_t rows, int64_t V) {
   if (rows <= 0 || V <= 0) return 0;

@@ -133,6 +133,11 @@ cudaError_t launch_lm_reduce(const float* part_max, const int* part_arg, const f
                              int tiles, long long M, long long V, float inv_temp, int* tok,
                              float* zmax, float* logsoftmax, cudaStream_t s);
 
+// ------------------------------------------------ T = 1 verification ----
+cudaError_t launch_accept_sample(const float* p, const float* q, const int* draft, long long dstride,
+                                 const unsigned* u, const unsigned* r, int batch, int nd, long long V, int* accept,
+                                 int* next_tok, cudaStream_t s);
+
 // --------------------------------------------------------------- KL ----
 constexpr int KL_CHUNK = 8192;  // vocabulary entries per CTA of the partial-sum stage
 int kl_chunks(long long V);

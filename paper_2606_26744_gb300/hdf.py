@@ -75,6 +75,7 @@ _SIGS = {
     "hdf_lm_head_argmax_static": (c_int, [c_vp, c_int, c_i64, c_int, c_vp, c_i64, c_float, c_vp, c_vp, c_vp,
                                           c_vp]),
     "hdf_set_reduce_path": (c_int, [c_int]),
+    "hdf_accept_sample": (c_int, [c_vp, c_vp, c_vp, c_i64, c_vp, c_vp, c_int, c_int, c_i64, c_vp, c_vp, c_vp]),
     "hdf_kl_distill_workspace_size": (c_size, [c_i64, c_i64]),
     "hdf_kl_distill": (c_int, [c_vp, c_vp, c_i64, c_i64, c_float, c_vp, c_vp, c_vp, c_size, c_vp]),
 }
@@ -317,3 +318,24 @@ def hdf_kl_distill(ls_teacher: torch.Tensor, ls_student: torch.Tensor, *, t_kd: 
     _check(lib.hdf_kl_distill(_p(ls_teacher), _p(ls_student), rows, V, t_kd, _p(kl_rows), _p(kl_mean), _p(ws),
                               ws.numel(), _stream(stream)))
     return kl_rows, kl_mean
+
+
+# ------------------------------------------------------ T = 1 verification
+def hdf_accept_sample(p_target: torch.Tensor, q_draft: torch.Tensor, draft: torch.Tensor, u: torch.Tensor,
+                      r: torch.Tensor, *, accept: Optional[torch.Tensor] = None,
+                      next_tok: Optional[torch.Tensor] = None, stream=None):
+    """Speculative-sampling verification: p_target [batch, n+1, V], q_draft
+    [batch, n, V] fp32 probabilities, draft [batch, n] int32 (row stride
+    draft.stride(0)), u [batch, n] and r [batch] uint32 uniforms (int32
+    tensors holding the same bits).  Returns (accept, next_tok) int32."""
+    batch, n1, V = p_target.shape
+    nd = n1 - 1
+    dev = p_target.device
+    if accept is None:
+        accept = torch.empty((batch,), dtype=torch.int32, device=dev)
+    if next_tok is None:
+        next_tok = torch.empty((batch,), dtype=torch.int32, device=dev)
+    _check(load().hdf_accept_sample(_p(p_target), _p(q_draft) if nd > 0 else None, _p(draft) if nd > 0 else None,
+                                    draft.stride(0) if nd > 0 else 0, _p(u) if nd > 0 else None, _p(r), batch, nd,
+                                    V, _p(accept), _p(next_tok), _stream(stream)))
+    return accept, next_tok

@@ -57,6 +57,14 @@ def test_reduce_path_switch(lib):
         assert lib.hdf_set_reduce_path(path) == 0
 
 
+def test_accept_sample_host_validation(lib):
+    v = ctypes.c_void_p
+    assert lib.hdf_accept_sample(v(16), v(16), v(16), 3, v(16), v(16), 2, 7, 100, v(16), v(16), None) == 2  # stride
+    assert lib.hdf_accept_sample(v(16), v(16), v(16), 7, v(16), v(16), 2, 7, 1 << 23, v(16), v(16), None) == 2
+    assert lib.hdf_accept_sample(v(16), None, v(16), 7, v(16), v(16), 2, 7, 100, v(16), v(16), None) == 1
+    assert lib.hdf_accept_sample(None, None, None, 0, None, None, 0, 7, 100, None, None, None) == 0  # empty
+
+
 def test_kl_host_validation(lib):
     v = ctypes.c_void_p
     assert lib.hdf_kl_distill(v(16), v(16), 2, 100, 0.0, None, None, v(256), 4096, None) == 1   # t_kd <= 0
