@@ -10,6 +10,8 @@
  *   hdf_accept_len      Sec. 3.4: accepted-prefix length of each block
  * hdf_accept_sample is the temperature-1 (sampling) form of step 4, and
  * hdf_kl_distill the training-time distillation target (Eq. 2, Sec. 2.3).
+ * hdf_ctx_append + hdf_draft_block_cached split step 2 for serving: the
+ * context projection of each accepted token runs once, into a K/V cache.
  *
  * Conventions shared by every call
  *   - All tensor arguments are DEVICE pointers owned by the caller, row-major,
@@ -28,7 +30,9 @@
  *     storage; GEMMs then run on the tensor cores' tf32 mode).
  *   - Kernels that wait on hardware barriers give up after a bounded time and
  *     record HDF_ERR_DEVICE_CHECK in a device status word that
- *     hdf_device_status() reads; they never trap.
+ *     hdf_device_status() reads; they never trap.  Bounds that depend on
+ *     device data (cache lengths) are checked the same way: the access is
+ *     skipped and the status word records it.
  */
 #ifndef HDF_H
 #define HDF_H
@@ -57,7 +61,8 @@ enum hdf_status {
   HDF_ERR_WORKSPACE = 5,    /* workspace missing, misaligned or too small */
   HDF_ERR_CUDA = 6,         /* a CUDA runtime/driver call or launch failed */
   HDF_ERR_UNSUPPORTED = 7,  /* valid request this build does not implement */
-  HDF_ERR_DEVICE_CHECK = 8  /* a kernel's bounded wait gave up (device word) */
+  HDF_ERR_DEVICE_CHECK = 8  /* a kernel's bounded wait gave up, or a device-side
+                               bound check failed (device word) */
 };
 
 enum hdf_dtype { HDF_F32 = 0, HDF_BF16 = 1 };
@@ -204,6 +209,66 @@ HDF_API int hdf_draft_block(const hdf_drafter_weights* w, const hdf_draft_shape*
                     void* ws, size_t ws_bytes,
                     const hdf_trace* trace, /* NULL: no timing events */
                     hdf_stream_t stream);
+
+/* ------------------------------------------------------------------------
+ * (2') Incremental form of step 2 for serving.  In the formula above, the
+ *     context keys and values of row t of sequence i depend only on that
+ *     row's reduced state and on t:  K_c[t] = RoPE(c_t W_k^T, t),
+ *     V_c[t] = c_t W_v^T.  The pre-collapse residual of an accepted token
+ *     never changes (Sec. 1: it is stored once, for MTP).  So a serving loop
+ *     keeps K_c and V_c of every layer in a cache and, each round, projects
+ *     only the tokens accepted since the last round.
+ *
+ *   hdf_ctx_append          c = RMSNorm_{ctx_norm}(ctx_new), then per layer
+ *                           writes K_c, V_c of the new rows at positions
+ *                           len[i] .. len[i] + n_i - 1 of sequence i, then
+ *                           len[i] += n_i
+ *   hdf_draft_block_cached  the block forward of step 2 (same formula, same
+ *                           h_out), with T_i = len[i] and K_c, V_c read from
+ *                           the cache instead of projected from ctx
+ *
+ * Appending the rows of a context in any number of rounds and then calling
+ * hdf_draft_block_cached gives exactly (bit for bit) the hdf_draft_block
+ * output for the whole context, when both use the same shape.max_ctx: every
+ * row is projected by the same kernel with the same reduction order, and
+ * the attention splits the keys the same way.
+ * ---------------------------------------------------------------------- */
+typedef struct {
+  void* k;       /* [n_layers, batch, capacity, d] dtype: K_c of each layer (RoPE applied) */
+  void* v;       /* [n_layers, batch, capacity, d] dtype: V_c of each layer */
+  int32_t* len;  /* [batch] DEVICE: rows held per sequence (T_i); the caller
+                    zeroes it for a new sequence, hdf_ctx_append advances it */
+  int capacity;  /* rows reserved per sequence, >= 1 */
+} hdf_ctx_cache;
+
+/* ctx_new [n_ctx, d] dtype: reduced states (y of Eq. 1) of the new rows,
+ *         grouped by sequence: rows cu_new[i] .. cu_new[i+1] of sequence i.
+ * cu_new  [batch + 1] DEVICE int32, non-decreasing, cu_new[0] = 0.
+ * shape.n_ctx is the host's row count of ctx_new; rows at or past
+ * cu_new[batch] (<= n_ctx) are skipped, so one captured CUDA graph serves
+ * rounds with any number of accepted tokens.  shape.max_ctx is unused.
+ * A row whose position would reach cache->capacity is not written: len[i]
+ * stops at capacity and HDF_ERR_DEVICE_CHECK is recorded in the device
+ * status word (hdf_device_status).  Requires rope_max_pos >= capacity.
+ * Workspace: hdf_ctx_append_workspace_size(shape). */
+HDF_API size_t hdf_ctx_append_workspace_size(const hdf_draft_shape* shape);
+HDF_API int hdf_ctx_append(const hdf_drafter_weights* w, const hdf_draft_shape* shape,
+                           const void* ctx_new, const int32_t* cu_new, const hdf_ctx_cache* cache,
+                           void* ws, size_t ws_bytes, hdf_stream_t stream);
+
+/* Block forward over the cached context.  shape.max_ctx bounds every len[i]
+ * (it sizes the attention split; <= cache->capacity); shape.n_ctx is unused.
+ * A len[i] above max_ctx is a contract violation: the keys past max_ctx are
+ * not attended and HDF_ERR_DEVICE_CHECK is recorded.  Rows of the cache at
+ * or past len[i] may hold anything (they are never read into a result).
+ * Requires rope_max_pos >= max_ctx + block.  trace: as for
+ * hdf_draft_block (the context-norm and context-K/V stages are empty).
+ * Workspace: hdf_draft_block_cached_workspace_size(shape). */
+HDF_API size_t hdf_draft_block_cached_workspace_size(const hdf_draft_shape* shape);
+HDF_API int hdf_draft_block_cached(const hdf_drafter_weights* w, const hdf_draft_shape* shape,
+                                   const hdf_ctx_cache* cache, const int32_t* anchor, void* h_out,
+                                   void* ws, size_t ws_bytes, const hdf_trace* trace,
+                                   hdf_stream_t stream);
 
 /* cos/sin tables for the drafter's RoPE: entry [p][i] = cos/sin of
  * p * theta^(-2i/head_dim), computed in fp64 on the device and stored fp32.

@@ -47,6 +47,24 @@ __device__ __forceinline__ void mma16816(float* d, const uint32_t* a, uint32_t b
       : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
 }
 
+// First row and key count of sequence b's context: packed rows from cu_ctx,
+// or the cached rows b * ctx_stride + [0, ctx_len[b]).  A cached length
+// outside [0, max_len] is limited to it and recorded (by one thread).
+__device__ __forceinline__ void context_span(const AttnArgs& a, int b, bool report, int* c0, int* T) {
+  if (a.ctx_len) {
+    int t = a.ctx_len[b];
+    if (t < 0 || t > a.max_len) {
+      if (report) record_device_error(a.status);
+      t = t < 0 ? 0 : a.max_len;
+    }
+    *c0 = (int)(b * a.ctx_stride);
+    *T = t;
+  } else {
+    *c0 = a.cu_ctx[b];
+    *T = a.cu_ctx[b + 1] - *c0;
+  }
+}
+
 // byte offset of the 16-byte chunk c (0..7) of row r in a 128-byte-swizzled box
 __device__ __forceinline__ uint32_t sw128(int r, int c) {
   return (uint32_t)(r * 128 + ((c ^ (r & 7)) << 4));
@@ -71,15 +89,6 @@ __global__ void __launch_bounds__(160, 1)
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   pdl_launch_dependents();
   const int B = a.block;
-  const int c0 = __ldg(a.cu_ctx + b), T = __ldg(a.cu_ctx + b + 1) - c0;
-  const int nc_b = min(a.n_chunks, T > 0 ? (T + a.chunk - 1) / a.chunk : 1);
-  if (chunk_id >= nc_b) return;
-  const int kbeg = chunk_id * a.chunk;
-  const int kend = min(T, kbeg + a.chunk);
-  const int n_ctx_tiles = kend > kbeg ? (kend - kbeg + KT - 1) / KT : 0;
-  const bool has_block = chunk_id == nc_b - 1;
-  const int ntiles = n_ctx_tiles + (has_block ? 1 : 0);
-
   if (tid == 0) {
     for (int s = 0; s < NSTAGE; ++s) {
       mbar_init(smem_u32(&full_bar[s]), 1);
@@ -88,7 +97,16 @@ __global__ void __launch_bounds__(160, 1)
     fence_mbar_init();
   }
   __syncthreads();
-  pdl_wait();  // Q and the block / context K, V come from the kernels before
+  pdl_wait();  // Q, the block / context K, V and the cache lengths come from the kernels before
+  int c0, T;
+  context_span(a, b, chunk_id == 0 && h == 0 && tid == 0, &c0, &T);
+  const int nc_b = min(a.n_chunks, T > 0 ? (T + a.chunk - 1) / a.chunk : 1);
+  if (chunk_id >= nc_b) return;
+  const int kbeg = chunk_id * a.chunk;
+  const int kend = min(T, kbeg + a.chunk);
+  const int n_ctx_tiles = kend > kbeg ? (kend - kbeg + KT - 1) / KT : 0;
+  const bool has_block = chunk_id == nc_b - 1;
+  const int ntiles = n_ctx_tiles + (has_block ? 1 : 0);
 
   if (warp == NCW) {
     if (lane == 0) {  // ------------------------------------------ producer
@@ -143,6 +161,18 @@ __global__ void __launch_bounds__(160, 1)
       const int valid = blk ? B : min(KT, kend - kbeg - t * KT);
       const uint32_t kbase = smem_u32(smem + s * STAGE_BYTES);
       const uint32_t vbase = kbase + TILE_BYTES;
+      if (a.ctx_len && !blk && valid < KT) {
+        // cache rows past the sequence's length may hold anything; their
+        // softmax weight is 0, so zero their V for an exact 0 contribution
+        uint8_t* vt = smem + s * STAGE_BYTES + TILE_BYTES;
+        for (int i = lane; i < (KT - valid) * HALVES * 8; i += 32) {
+          const int r = valid + i / (HALVES * 8), rem = i % (HALVES * 8);
+          *reinterpret_cast<uint4*>(vt + (rem >> 3) * (KT * 128) + r * 128 + (rem & 7) * 16) = make_uint4(0, 0, 0, 0);
+        }
+        // the stage is refilled by TMA (async proxy) after these generic stores
+        asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+        __syncwarp();
+      }
 
       // S = Q K^T for 64 keys: 8 n-blocks of 8 keys
       float sc[8][4];
@@ -332,7 +362,8 @@ __global__ void attn_f32_kernel(const AttnArgs a) {
   const float* Kb = reinterpret_cast<const float*>(a.kb);
   const float* Vb = reinterpret_cast<const float*>(a.vb);
   float* out = reinterpret_cast<float*>(a.out);
-  const int c0 = a.cu_ctx[b], T = a.cu_ctx[b + 1] - c0;
+  int c0, T;
+  context_span(a, b, h == 0 && threadIdx.x == 0, &c0, &T);
   const float scale = rsqrtf((float)HD);
   for (int r = warp; r < a.block; r += blockDim.x >> 5) {
     const size_t qrow = (size_t)b * a.block + r;

@@ -68,9 +68,39 @@ __device__ __forceinline__ int ctx_position(const int* cu, int batch, long long 
   }
   return (int)(t - __ldg(cu + lo));
 }
-__device__ __forceinline__ int block_position(const int* cu, int block, int j) {
-  const int b = j / block;
-  return (__ldg(cu + b + 1) - __ldg(cu + b)) + (j - b * block);
+__device__ __forceinline__ int block_position(const Epilogue& E, int j) {
+  const int b = j / E.block;
+  const int T = E.pos_mode == 4 ? __ldg(E.ctx_len + b) : __ldg(E.cu_ctx + b + 1) - __ldg(E.cu_ctx + b);
+  return T + (j - b * E.block);
+}
+
+// Context row t of a kEpiStore GEMM: its output row (or -1: not stored) and
+// its RoPE position.  Mode 3 appends to a cache: sequence b's rows go after
+// the ctx_len[b] rows it already holds, rows past cu[batch] are skipped, and
+// a row that would pass the cache capacity is skipped and recorded.
+__device__ __forceinline__ long long ctx_store_row(const Epilogue& E, long long t, int* pos, int* status) {
+  if (E.pos_mode == 1) {
+    *pos = ctx_position(E.cu_ctx, E.batch, t);
+    return t;
+  }
+  if (E.pos_mode != 3) {
+    *pos = 0;
+    return t;
+  }
+  *pos = 0;
+  if (t >= __ldg(E.cu_ctx + E.batch)) return -1;
+  int lo = 0, hi = E.batch;
+  while (hi - lo > 1) {
+    const int mid = (lo + hi) >> 1;
+    if (__ldg(E.cu_ctx + mid) <= t) lo = mid; else hi = mid;
+  }
+  const long long p = (long long)__ldg(E.ctx_len + lo) + (t - __ldg(E.cu_ctx + lo));
+  if (p < 0 || p >= E.cache_cap) {
+    record_device_error(status);
+    return -1;
+  }
+  *pos = (int)p;
+  return (long long)lo * E.cache_cap + p;
 }
 
 template <typename T>
@@ -92,9 +122,12 @@ __device__ __forceinline__ void store16<float>(float* dst, const float* v) {
 // with identical (tile, c0) so that shuffles and barriers are uniform.
 // rope_row: this thread's row of the RoPE table staged in shared memory
 // (cos of the hd/2 pairs, then sin, see stage_rope_row), or nullptr.
+// srow: kEpiStore output row of this thread's token from ctx_store_row (-1:
+// not stored).
 template <typename T, int BN>
 __device__ __forceinline__ void epilogue_chunk(const GemmArgs& g, int tile_m, int tile_n, int c0,
-                                               float* v, uint8_t* smem, const float* rope_row = nullptr) {
+                                               float* v, uint8_t* smem, const float* rope_row, long long srow,
+                                               int spos) {
   const Epilogue& E = g.epi;
   const int row = threadIdx.x;
   const int lane = row & 31, warp = row >> 5;
@@ -102,7 +135,7 @@ __device__ __forceinline__ void epilogue_chunk(const GemmArgs& g, int tile_m, in
     case kEpiStore: {  // rows = tokens, columns = output features
       const long long t = (long long)tile_m * BM + row;
       const int col0 = tile_n * BN + c0;
-      if (t >= g.M || col0 >= g.N) return;
+      if (t >= g.M || col0 >= g.N || srow < 0) return;
       const int seg = col0 / E.seg_width;
       const int fl = col0 - seg * E.seg_width;
       if ((E.rope_mask >> seg) & 1) {
@@ -116,7 +149,7 @@ __device__ __forceinline__ void epilogue_chunk(const GemmArgs& g, int tile_m, in
           c[0] = c0v.x; c[1] = c0v.y; c[2] = c0v.z; c[3] = c0v.w; c[4] = c1v.x; c[5] = c1v.y; c[6] = c1v.z; c[7] = c1v.w;
           sn[0] = s0v.x; sn[1] = s0v.y; sn[2] = s0v.z; sn[3] = s0v.w; sn[4] = s1v.x; sn[5] = s1v.y; sn[6] = s1v.z; sn[7] = s1v.w;
         } else {
-          const int pos = (int)min((long long)ctx_position(E.cu_ctx, E.batch, t), E.rope_rows - 1);
+          const int pos = (int)min((long long)spos, E.rope_rows - 1);
 #pragma unroll
           for (int i = 0; i < 8; ++i) {
             c[i] = __ldg(E.rope_cos + (size_t)pos * hh + pi0 + i);
@@ -130,7 +163,7 @@ __device__ __forceinline__ void epilogue_chunk(const GemmArgs& g, int tile_m, in
           v[2 * i + 1] = x0 * sn[i] + x1 * c[i];
         }
       }
-      store16<T>(reinterpret_cast<T*>(E.out[seg]) + t * E.ld + fl, v);
+      store16<T>(reinterpret_cast<T*>(E.out[seg]) + srow * E.ld + fl, v);
       return;
     }
     case kEpiStoreT: {  // rows = output features, columns = tokens
@@ -146,7 +179,7 @@ __device__ __forceinline__ void epilogue_chunk(const GemmArgs& g, int tile_m, in
         int pos[16];
 #pragma unroll
         for (int k = 0; k < 16; ++k)
-          pos[k] = jb + k < g.N ? (int)min((long long)block_position(E.cu_ctx, E.block, jb + k), E.rope_rows - 1) : 0;
+          pos[k] = jb + k < g.N ? (int)min((long long)block_position(E, jb + k), E.rope_rows - 1) : 0;
         float cs[16], sn[16];
 #pragma unroll
         for (int k = 0; k < 16; ++k) {
@@ -273,7 +306,8 @@ __device__ __forceinline__ void epilogue_chunk(const GemmArgs& g, int tile_m, in
 // 2*(hd/2) + 4 floats apart, so eight threads reading 16 bytes each hit
 // distinct bank groups.  Returns the row, or nullptr when nothing is staged.
 template <int BN>
-__device__ __forceinline__ const float* stage_rope_row(const GemmArgs& g, int tile_m, int tile_n, uint8_t* smem) {
+__device__ __forceinline__ const float* stage_rope_row(const GemmArgs& g, int tile_m, int tile_n, uint8_t* smem,
+                                                       int spos) {
   const Epilogue& E = g.epi;
   if (E.kind != kEpiStore || E.head_dim > 128 || E.head_dim % 16) return nullptr;
   const int seg = (tile_n * BN) / E.seg_width;
@@ -282,7 +316,7 @@ __device__ __forceinline__ const float* stage_rope_row(const GemmArgs& g, int ti
   float* row = reinterpret_cast<float*>(smem) + threadIdx.x * stride;
   const long long t = (long long)tile_m * BM + threadIdx.x;
   if (t < g.M) {
-    const int pos = (int)min((long long)ctx_position(E.cu_ctx, E.batch, t), E.rope_rows - 1);
+    const int pos = (int)min((long long)spos, E.rope_rows - 1);
     const float* cs = E.rope_cos + (size_t)pos * hh;
     const float* sn = E.rope_sin + (size_t)pos * hh;
     for (int i = 0; i < hh; i += 4) {
@@ -434,14 +468,19 @@ __global__ void __launch_bounds__(128, 1) gemm_kernel(const __grid_constant__ Ge
   __syncthreads();
   const bool aborted = abort_flag != 0;
   const uint32_t taddr = tmem + ((uint32_t)(warp * 32) << 16);
+  int spos = 0;
+  const long long srow = g.epi.kind == kEpiStore && (long long)tile_m * BM + tid < g.M
+                             ? ctx_store_row(g.epi, (long long)tile_m * BM + tid, &spos, g.status)
+                             : -1;
   if (!aborted && kb1 > kb0 && g.k_splits == 1) {
-    const float* rope_row = BM * (2 * 64 + 4) * 4 <= STAGES * STAGE_BYTES ? stage_rope_row<BN>(g, tile_m, tile_n, smem)
-                                                                           : nullptr;
+    const float* rope_row = BM * (2 * 64 + 4) * 4 <= STAGES * STAGE_BYTES
+                                ? stage_rope_row<BN>(g, tile_m, tile_n, smem, spos)
+                                : nullptr;
 #pragma unroll 1
     for (int c0 = 0; c0 < BN; c0 += 16) {
       float v[16];
       tmem_ld16(taddr + c0, v);
-      epilogue_chunk<T, BN>(g, tile_m, tile_n, c0, v, smem, rope_row);
+      epilogue_chunk<T, BN>(g, tile_m, tile_n, c0, v, smem, rope_row, srow, spos);
     }
   }
   if (g.k_splits > 1) {
@@ -507,7 +546,7 @@ __global__ void __launch_bounds__(128, 1) gemm_kernel(const __grid_constant__ Ge
           v[4 * i + 2] = q.z;
           v[4 * i + 3] = q.w;
         }
-        epilogue_chunk<T, BN>(g, tile_m, tile_n, c0, v, smem);
+        epilogue_chunk<T, BN>(g, tile_m, tile_n, c0, v, smem, nullptr, srow, spos);
       }
     }
   }

@@ -363,30 +363,18 @@ int hdf_rope_table(double theta, int head_dim, int64_t max_pos, float* cos_out, 
 }
 
 // --------------------------------------------------------- draft block
-size_t hdf_draft_block_workspace_size(const hdf_draft_shape* shape) {
-  if (check_draft_shape(shape) != HDF_OK) return 0;
-  return draft_layout(shape).total;
-}
+}  // extern "C"
 
-int hdf_draft_block(const hdf_drafter_weights* w, const hdf_draft_shape* sh, const void* ctx,
-                    const int32_t* cu_ctx, const int32_t* anchor, void* h_out, void* ws, size_t ws_bytes,
-                    const hdf_trace* trace, hdf_stream_t stream) {
-  g_err.clear();
-  int rc = check_draft_shape(sh);
-  if (rc) return rc;
+namespace {
+
+// Weight pointers and RoPE table of a draft call: non-null and 16-byte aligned.
+int check_drafter_weights(const hdf_drafter_weights* w, const hdf_draft_shape* sh) {
   if (!w || !w->layers) return fail(HDF_ERR_INVALID_ARG, "weights / layers NULL");
-  const int dt = sh->dtype;
-  const long long M = (long long)sh->batch * sh->block;
-  const long long d = sh->d, F = sh->ffn;
-  if (M == 0) return HDF_OK;
-  if (!cu_ctx || !anchor || !h_out || (sh->n_ctx > 0 && !ctx)) return fail(HDF_ERR_INVALID_ARG, "null input");
   if (!w->embed || !w->mask_vec || !w->ctx_norm || !w->final_norm || !w->rope_cos || !w->rope_sin)
     return fail(HDF_ERR_INVALID_ARG, "null weight");
-  if (w->rope_max_pos < (long long)sh->max_ctx + sh->block)
-    return fail(HDF_ERR_SHAPE, "rope_max_pos %lld < max_ctx + block", (long long)w->rope_max_pos);
-  const void* ptrs[] = {ctx, h_out, w->embed, w->mask_vec, w->ctx_norm, w->final_norm};
+  const void* ptrs[] = {w->embed, w->mask_vec, w->ctx_norm, w->final_norm};
   for (const void* p : ptrs)
-    if (p && !aligned16(p)) return fail(HDF_ERR_ALIGNMENT, "tensor not 16-byte aligned");
+    if (!aligned16(p)) return fail(HDF_ERR_ALIGNMENT, "weight not 16-byte aligned");
   for (int l = 0; l < sh->n_layers; ++l) {
     const hdf_layer_weights& L = w->layers[l];
     const void* lp[] = {L.attn_norm, L.wq, L.wk, L.wv, L.wo, L.mlp_norm, L.wg, L.wu, L.wd};
@@ -395,10 +383,86 @@ int hdf_draft_block(const hdf_drafter_weights* w, const hdf_draft_shape* sh, con
       if (!aligned16(p)) return fail(HDF_ERR_ALIGNMENT, "layer %d weight misaligned", l);
     }
   }
-  const DraftLayout Lo = draft_layout(sh);
+  return HDF_OK;
+}
+
+int check_cache(const hdf_ctx_cache* cache, const hdf_draft_shape* sh) {
+  if (!cache || !cache->k || !cache->v || !cache->len) return fail(HDF_ERR_INVALID_ARG, "cache / k / v / len NULL");
+  if (!aligned16(cache->k) || !aligned16(cache->v) || (reinterpret_cast<uintptr_t>(cache->len) & 3))
+    return fail(HDF_ERR_ALIGNMENT, "cache k / v must be 16-byte aligned, len 4-byte aligned");
+  if (cache->capacity < 1) return fail(HDF_ERR_SHAPE, "cache capacity %d", cache->capacity);
+  if ((long long)sh->batch * cache->capacity > 0x7fffffffLL)
+    return fail(HDF_ERR_SHAPE, "batch * capacity must stay below 2^31 rows");
+  return HDF_OK;
+}
+
+// Byte offset of layer l in a cache tensor [n_layers, batch, capacity, d].
+size_t cache_layer_offset(const hdf_draft_shape* sh, const hdf_ctx_cache* cache, int l) {
+  return (size_t)l * sh->batch * (size_t)cache->capacity * sh->d * esize(sh->dtype);
+}
+
+// [K_c | V_c] = c [W_k; W_v]^T with RoPE on K_c (context rows as GEMM rows,
+// no K split, so every row's sums run in the same order whatever the launch).
+// pos_mode 1: rows land packed in kout / vout; pos_mode 3: rows are appended
+// to a cache (cu = cu_new, len, cap).
+int launch_ctx_kv(const hdf_drafter_weights* w, const hdf_layer_weights& Lw, const hdf_draft_shape* sh,
+                  const void* c, long long rows, int bn, void* kout, void* vout, const int32_t* cu, int pos_mode,
+                  const int32_t* len, long long cap, cudaStream_t s) {
+  const int dt = sh->dtype;
+  const long long d = sh->d;
+  SplitPlan p{bn, 1, 0};
+  GemmArgs g;
+  init_gemm(g, dt, rows, 2 * d, d, p);
+  g.group_n = 8;
+  int rc;
+  if ((rc = make_map(&g.A.map[0], c, dt, rows, d, d, 64))) return rc;
+  if ((rc = make_map(&g.B.map[0], Lw.wk, dt, d, d, d, p.bn))) return rc;
+  if ((rc = make_map(&g.B.map[1], Lw.wv, dt, d, d, d, p.bn))) return rc;
+  g.pre_operand = 2;  // weights: loaded before the context norm has finished
+  g.B.rows_per_map = (int)d;
+  g.epi.kind = kEpiStore;
+  g.epi.out[0] = kout;
+  g.epi.out[1] = vout;
+  g.epi.seg_width = (int)d;
+  g.epi.ld = d;
+  g.epi.rope_mask = 1;
+  g.epi.rope_cos = w->rope_cos;
+  g.epi.rope_sin = w->rope_sin;
+  g.epi.rope_rows = w->rope_max_pos;
+  g.epi.head_dim = sh->head_dim;
+  g.epi.cu_ctx = cu;
+  g.epi.batch = sh->batch;
+  g.epi.block = sh->block;
+  g.epi.pos_mode = pos_mode;
+  g.epi.ctx_len = len;
+  g.epi.cache_cap = cap;
+  CK(launch_gemm(g, s), "ctx kv gemm");
+  return HDF_OK;
+}
+
+// Tile width of the context K/V GEMM: 256 columns, or 128 when a 256-wide
+// grid would leave most SMs idle (few new rows in an append).
+int ctx_kv_bn(const hdf_draft_shape* sh, long long rows) {
+  if (sh->d % 256) return 128;
+  const long long tiles = ((rows + 127) / 128) * (2LL * sh->d / 256);
+  return tiles >= num_sms() ? 256 : 128;
+}
+
+// The block forward of hdf_draft_block.  Context from packed rows (ctx,
+// cu_ctx: normed and projected here) or from a K/V cache (cache != null).
+int draft_forward(const hdf_drafter_weights* w, const hdf_draft_shape* sh, const void* ctx, const int32_t* cu_ctx,
+                  const hdf_ctx_cache* cache, const int32_t* anchor, void* h_out, void* ws, size_t ws_bytes,
+                  const hdf_trace* trace, cudaStream_t s) {
+  int rc;
+  const int dt = sh->dtype;
+  const long long M = (long long)sh->batch * sh->block;
+  const long long d = sh->d, F = sh->ffn;
+  const bool cached = cache != nullptr;
+  hdf_draft_shape lsh = *sh;
+  if (cached) lsh.n_ctx = 0;  // no context rows to project: the layout holds the block only
+  const DraftLayout Lo = draft_layout(&lsh);
   if (!ws || ws_bytes < Lo.total || (reinterpret_cast<uintptr_t>(ws) & 255))
     return fail(HDF_ERR_WORKSPACE, "workspace %zu bytes (need %zu, 256-byte aligned)", ws_bytes, Lo.total);
-  cudaStream_t s = (cudaStream_t)stream;
   char* W = static_cast<char*>(ws);
   void* c = W + Lo.c;
   void* kc = W + Lo.kc;
@@ -411,6 +475,7 @@ int hdf_draft_block(const hdf_drafter_weights* w, const hdf_draft_shape* sh, con
   void* o = W + Lo.o;
   void* act = W + Lo.act;
   int* counters = reinterpret_cast<int*>(W + Lo.counters);
+  const long long n_ctx = cached ? 0 : sh->n_ctx;
 
   const int n_ev = trace ? trace->n_events : 0;
   const int want_ev = 3 + HDF_DRAFT_STAGES_PER_LAYER * sh->n_layers;
@@ -434,37 +499,23 @@ int hdf_draft_block(const hdf_drafter_weights* w, const hdf_draft_shape* sh, con
   int* attn_counters = counters;
   // ---- context RMSNorm
   if ((rc = mark())) return rc;
-  CK(launch_rmsnorm(ctx, 0, w->ctx_norm, c, dt, sh->n_ctx, (int)d, sh->norm_eps, s), "ctx norm");
+  if (n_ctx > 0) CK(launch_rmsnorm(ctx, 0, w->ctx_norm, c, dt, n_ctx, (int)d, sh->norm_eps, s), "ctx norm");
 
   for (int l = 0; l < sh->n_layers; ++l) {
     const hdf_layer_weights& Lw = w->layers[l];
     // ---- conditioning projection: [K_c | V_c] = c [W_k; W_v]^T, RoPE on K_c
     if ((rc = mark())) return rc;
-    if (sh->n_ctx > 0) {
-      SplitPlan p{d % 256 == 0 ? 256 : 128, 1, 0};
-      GemmArgs g;
-      init_gemm(g, dt, sh->n_ctx, 2 * d, d, p);
-      g.group_n = 8;
-      if ((rc = make_map(&g.A.map[0], c, dt, sh->n_ctx, d, d, 64))) return rc;
-      if ((rc = make_map(&g.B.map[0], Lw.wk, dt, d, d, d, p.bn))) return rc;
-      if ((rc = make_map(&g.B.map[1], Lw.wv, dt, d, d, d, p.bn))) return rc;
-      g.pre_operand = 2;  // weights: loaded before the context norm has finished
-      g.B.rows_per_map = (int)d;
-      g.epi.kind = kEpiStore;
-      g.epi.out[0] = kc;
-      g.epi.out[1] = vc;
-      g.epi.seg_width = (int)d;
-      g.epi.ld = d;
-      g.epi.rope_mask = 1;
-      g.epi.rope_cos = w->rope_cos;
-      g.epi.rope_sin = w->rope_sin;
-      g.epi.rope_rows = w->rope_max_pos;
-      g.epi.head_dim = sh->head_dim;
-      g.epi.cu_ctx = cu_ctx;
-      g.epi.batch = sh->batch;
-      g.epi.block = sh->block;
-      g.epi.pos_mode = 1;
-      CK(launch_gemm(g, s), "ctx kv gemm");
+    if (n_ctx > 0 &&
+        (rc = launch_ctx_kv(w, Lw, sh, c, n_ctx, d % 256 == 0 ? 256 : 128, kc, vc, cu_ctx, 1, nullptr, 0, s)))
+      return rc;
+    // context K / V of this layer: the workspace, or the cache
+    const void* kctx = kc;
+    const void* vctx = vc;
+    long long ctx_rows = n_ctx;
+    if (cached) {
+      kctx = static_cast<const char*>(cache->k) + cache_layer_offset(sh, cache, l);
+      vctx = static_cast<const char*>(cache->v) + cache_layer_offset(sh, cache, l);
+      ctx_rows = (long long)sh->batch * cache->capacity;
     }
     // ---- block input / attention norm
     if ((rc = mark())) return rc;
@@ -497,9 +548,10 @@ int hdf_draft_block(const hdf_drafter_weights* w, const hdf_draft_shape* sh, con
       g.epi.rope_rows = w->rope_max_pos;
       g.epi.head_dim = sh->head_dim;
       g.epi.cu_ctx = cu_ctx;
+      g.epi.ctx_len = cached ? cache->len : nullptr;
       g.epi.batch = sh->batch;
       g.epi.block = sh->block;
-      g.epi.pos_mode = 2;
+      g.epi.pos_mode = cached ? 4 : 2;
       CK(launch_gemm(g, s), "qkv gemm");
     }
     // ---- attention over [K_c; K_b]
@@ -510,9 +562,12 @@ int hdf_draft_block(const hdf_drafter_weights* w, const hdf_draft_shape* sh, con
       a.q = q;
       a.kb = kbk;
       a.vb = vbk;
-      a.kc = kc;
-      a.vc = vc;
-      a.cu_ctx = cu_ctx;
+      a.kc = kctx;
+      a.vc = vctx;
+      a.cu_ctx = cached ? nullptr : cu_ctx;
+      a.ctx_len = cached ? cache->len : nullptr;
+      a.ctx_stride = cached ? cache->capacity : 0;
+      a.max_len = sh->max_ctx;
       a.out = o;
       a.part_o = reinterpret_cast<float*>(W + Lo.part_o);
       a.part_ml = reinterpret_cast<float*>(W + Lo.part_ml);
@@ -521,16 +576,16 @@ int hdf_draft_block(const hdf_drafter_weights* w, const hdf_draft_shape* sh, con
       a.n_heads = sh->n_heads;
       a.head_dim = sh->head_dim;
       a.d = (int)d;
-      a.n_ctx = sh->n_ctx;
+      a.n_ctx = ctx_rows;
       a.chunk = Lo.chunk;
       a.n_chunks = Lo.n_chunks;
       a.counters = attn_counters;
       a.status = device_status_ptr();
       AttnTmaps tm;
       if (dt == HDF_BF16) {
-        const void* kc_src = sh->n_ctx > 0 ? kc : kbk;
-        const void* vc_src = sh->n_ctx > 0 ? vc : vbk;
-        const long long rows = sh->n_ctx > 0 ? sh->n_ctx : M;
+        const void* kc_src = ctx_rows > 0 ? kctx : kbk;
+        const void* vc_src = ctx_rows > 0 ? vctx : vbk;
+        const long long rows = ctx_rows > 0 ? ctx_rows : M;
         if ((rc = make_map(&tm.k, kc_src, dt, rows, d, d, 64))) return rc;
         if ((rc = make_map(&tm.v, vc_src, dt, rows, d, d, 64))) return rc;
         if ((rc = make_map(&tm.kb, kbk, dt, M, d, d, 64))) return rc;
@@ -588,6 +643,92 @@ int hdf_draft_block(const hdf_drafter_weights* w, const hdf_draft_shape* sh, con
   if ((rc = mark())) return rc;
   CK(launch_rmsnorm(h, 1, w->final_norm, h_out, dt, M, (int)d, sh->norm_eps, s), "final norm");
   if ((rc = mark())) return rc;
+  return HDF_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+size_t hdf_draft_block_workspace_size(const hdf_draft_shape* shape) {
+  if (check_draft_shape(shape) != HDF_OK) return 0;
+  return draft_layout(shape).total;
+}
+
+int hdf_draft_block(const hdf_drafter_weights* w, const hdf_draft_shape* sh, const void* ctx,
+                    const int32_t* cu_ctx, const int32_t* anchor, void* h_out, void* ws, size_t ws_bytes,
+                    const hdf_trace* trace, hdf_stream_t stream) {
+  g_err.clear();
+  int rc = check_draft_shape(sh);
+  if (rc) return rc;
+  if ((rc = check_drafter_weights(w, sh))) return rc;
+  if ((long long)sh->batch * sh->block == 0) return HDF_OK;
+  if (!cu_ctx || !anchor || !h_out || (sh->n_ctx > 0 && !ctx)) return fail(HDF_ERR_INVALID_ARG, "null input");
+  if (w->rope_max_pos < (long long)sh->max_ctx + sh->block)
+    return fail(HDF_ERR_SHAPE, "rope_max_pos %lld < max_ctx + block", (long long)w->rope_max_pos);
+  if ((ctx && !aligned16(ctx)) || !aligned16(h_out)) return fail(HDF_ERR_ALIGNMENT, "tensor not 16-byte aligned");
+  return draft_forward(w, sh, ctx, cu_ctx, nullptr, anchor, h_out, ws, ws_bytes, trace, (cudaStream_t)stream);
+}
+
+size_t hdf_draft_block_cached_workspace_size(const hdf_draft_shape* shape) {
+  if (check_draft_shape(shape) != HDF_OK) return 0;
+  hdf_draft_shape s = *shape;
+  s.n_ctx = 0;
+  return draft_layout(&s).total;
+}
+
+int hdf_draft_block_cached(const hdf_drafter_weights* w, const hdf_draft_shape* sh, const hdf_ctx_cache* cache,
+                           const int32_t* anchor, void* h_out, void* ws, size_t ws_bytes, const hdf_trace* trace,
+                           hdf_stream_t stream) {
+  g_err.clear();
+  int rc = check_draft_shape(sh);
+  if (rc) return rc;
+  if ((rc = check_drafter_weights(w, sh))) return rc;
+  if ((rc = check_cache(cache, sh))) return rc;
+  if (sh->max_ctx > cache->capacity)
+    return fail(HDF_ERR_SHAPE, "max_ctx %d > cache capacity %d", sh->max_ctx, cache->capacity);
+  if ((long long)sh->batch * sh->block == 0) return HDF_OK;
+  if (!anchor || !h_out) return fail(HDF_ERR_INVALID_ARG, "null input");
+  if (!aligned16(h_out)) return fail(HDF_ERR_ALIGNMENT, "h_out not 16-byte aligned");
+  if (w->rope_max_pos < (long long)sh->max_ctx + sh->block)
+    return fail(HDF_ERR_SHAPE, "rope_max_pos %lld < max_ctx + block", (long long)w->rope_max_pos);
+  return draft_forward(w, sh, nullptr, nullptr, cache, anchor, h_out, ws, ws_bytes, trace, (cudaStream_t)stream);
+}
+
+size_t hdf_ctx_append_workspace_size(const hdf_draft_shape* shape) {
+  if (check_draft_shape(shape) != HDF_OK) return 0;
+  return std::max<size_t>(256, up256((size_t)shape->n_ctx * shape->d * esize(shape->dtype)));
+}
+
+int hdf_ctx_append(const hdf_drafter_weights* w, const hdf_draft_shape* sh, const void* ctx_new,
+                   const int32_t* cu_new, const hdf_ctx_cache* cache, void* ws, size_t ws_bytes,
+                   hdf_stream_t stream) {
+  g_err.clear();
+  int rc = check_draft_shape(sh);
+  if (rc) return rc;
+  if ((rc = check_drafter_weights(w, sh))) return rc;
+  if ((rc = check_cache(cache, sh))) return rc;
+  if (sh->batch == 0 || sh->n_ctx == 0) return HDF_OK;
+  if (!ctx_new || !cu_new) return fail(HDF_ERR_INVALID_ARG, "ctx_new / cu_new NULL");
+  if (!aligned16(ctx_new)) return fail(HDF_ERR_ALIGNMENT, "ctx_new not 16-byte aligned");
+  if (w->rope_max_pos < cache->capacity)
+    return fail(HDF_ERR_SHAPE, "rope_max_pos %lld < cache capacity %d", (long long)w->rope_max_pos, cache->capacity);
+  const size_t need = hdf_ctx_append_workspace_size(sh);
+  if (!ws || ws_bytes < need || (reinterpret_cast<uintptr_t>(ws) & 255))
+    return fail(HDF_ERR_WORKSPACE, "workspace %zu bytes (need %zu, 256-byte aligned)", ws_bytes, need);
+  cudaStream_t s = (cudaStream_t)stream;
+  const long long d = sh->d;
+  void* c = ws;
+  CK(launch_rmsnorm(ctx_new, 0, w->ctx_norm, c, sh->dtype, sh->n_ctx, (int)d, sh->norm_eps, s), "ctx norm");
+  const int bn = ctx_kv_bn(sh, sh->n_ctx);
+  for (int l = 0; l < sh->n_layers; ++l) {
+    char* kl = static_cast<char*>(cache->k) + cache_layer_offset(sh, cache, l);
+    char* vl = static_cast<char*>(cache->v) + cache_layer_offset(sh, cache, l);
+    if ((rc = launch_ctx_kv(w, w->layers[l], sh, c, sh->n_ctx, bn, kl, vl, cu_new, 3, cache->len,
+                            cache->capacity, s)))
+      return rc;
+  }
+  CK(launch_cache_advance(cache->len, cu_new, sh->batch, cache->capacity, device_status_ptr(), s), "cache advance");
   return HDF_OK;
 }
 

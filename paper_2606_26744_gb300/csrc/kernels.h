@@ -91,7 +91,10 @@ struct Epilogue {
   const int* cu_ctx;    // positions: context rows -> t - cu[b]
   int batch;
   int block;            // block rows: pos = T_b + (j % block)
-  int pos_mode;         // 0 none, 1 context rows, 2 block rows
+  int pos_mode;         // 0 none, 1 context rows, 2 block rows (T_b from cu_ctx),
+                        // 3 context rows appended to a cache, 4 block rows (T_b = ctx_len[b])
+  const int* ctx_len;   // modes 3, 4: rows already in the cache per sequence
+  long long cache_cap;  // mode 3: row t of sequence b goes to row b * cache_cap + ctx_len[b] + t - cu[b]
   float* resid;         // kEpiResidT
   // kEpiLmHeadT
   float inv_temp;
@@ -133,6 +136,9 @@ cudaError_t launch_lm_reduce(const float* part_max, const int* part_arg, const f
                              int tiles, long long M, long long V, float inv_temp, int* tok,
                              float* zmax, float* logsoftmax, cudaStream_t s);
 
+// len[b] += cu[b+1] - cu[b], limited to cap (status recorded past it)
+cudaError_t launch_cache_advance(int* len, const int* cu, int batch, long long cap, int* status, cudaStream_t s);
+
 // ------------------------------------------------ T = 1 verification ----
 cudaError_t launch_accept_sample(const float* p, const float* q, const int* draft, long long dstride,
                                  const unsigned* u, const unsigned* r, int batch, int nd, long long V, int* accept,
@@ -152,7 +158,10 @@ struct AttnArgs {
   const void* vb;      // [M, d]
   const void* kc;      // [n_ctx, d] context keys
   const void* vc;      // [n_ctx, d]
-  const int* cu_ctx;   // [batch + 1]
+  const int* cu_ctx;   // [batch + 1]; or null with ctx_len set:
+  const int* ctx_len;  // [batch] cached rows: sequence b's keys are rows b * ctx_stride + [0, ctx_len[b])
+  long long ctx_stride;
+  int max_len;         // with ctx_len: keys past max_len are not attended (status recorded)
   void* out;           // [M, d]
   float* part_o;       // [batch, heads, chunks, block, hd]
   float* part_ml;      // [batch, heads, chunks, block, 2]

@@ -138,6 +138,25 @@ __global__ void accept_kernel(const int* __restrict__ draft, long long ds, const
   accept[i] = n;
 }
 
+// Cache length update after an append: len[b] += n_b (n_b = cu[b+1] - cu[b]),
+// limited to the capacity; a count that is negative or passes the capacity
+// is recorded (the append kernel skipped those rows).
+__global__ void cache_advance_kernel(int* __restrict__ len, const int* __restrict__ cu, int batch, long long cap,
+                                     int* status) {
+  pdl_launch_dependents();
+  pdl_wait();  // every layer's append has read len
+  const int b = blockIdx.x * blockDim.x + threadIdx.x;
+  if (b >= batch) return;
+  const long long n = (long long)cu[b + 1] - cu[b];
+  long long t = (long long)len[b] + n;
+  if (n < 0 || t > cap) {
+    record_device_error(status);
+    t = t < 0 ? 0 : (t > cap ? cap : t);
+    if (n < 0) t = len[b];
+  }
+  len[b] = (int)t;
+}
+
 struct MaxArgSum {
   float m;
   int a;
@@ -229,6 +248,12 @@ cudaError_t launch_accept(const int* draft, long long ds, const int* target, lon
   if (batch == 0) return cudaSuccess;
   return launch_kernel(accept_kernel, dim3((batch + 127) / 128), dim3(128), 0, s, 1u, draft, ds, target, ts, batch,
                        nd, accept);
+}
+
+cudaError_t launch_cache_advance(int* len, const int* cu, int batch, long long cap, int* status, cudaStream_t s) {
+  if (batch == 0) return cudaSuccess;
+  return launch_kernel(cache_advance_kernel, dim3((batch + 127) / 128), dim3(128), 0, s, 1u, len, cu, batch, cap,
+                       status);
 }
 
 cudaError_t launch_lm_reduce(const float* pmax, const int* parg, const float* psum, int tiles, long long M,

@@ -55,6 +55,10 @@ class Trace(ctypes.Structure):
     _fields_ = [("events", ctypes.POINTER(c_vp)), ("n_events", c_int)]
 
 
+class CtxCache(ctypes.Structure):
+    _fields_ = [("k", c_vp), ("v", c_vp), ("len", c_vp), ("capacity", c_int)]
+
+
 _SIGS = {
     "hdf_version": (c_int, []),
     "hdf_status_str": (ctypes.c_char_p, [c_int]),
@@ -67,6 +71,13 @@ _SIGS = {
     "hdf_draft_block_workspace_size": (c_size, [ctypes.POINTER(DraftShape)]),
     "hdf_draft_block": (c_int, [ctypes.POINTER(DrafterWeights), ctypes.POINTER(DraftShape), c_vp, c_vp,
                                 c_vp, c_vp, c_vp, c_size, ctypes.POINTER(Trace), c_vp]),
+    "hdf_ctx_append_workspace_size": (c_size, [ctypes.POINTER(DraftShape)]),
+    "hdf_ctx_append": (c_int, [ctypes.POINTER(DrafterWeights), ctypes.POINTER(DraftShape), c_vp, c_vp,
+                               ctypes.POINTER(CtxCache), c_vp, c_size, c_vp]),
+    "hdf_draft_block_cached_workspace_size": (c_size, [ctypes.POINTER(DraftShape)]),
+    "hdf_draft_block_cached": (c_int, [ctypes.POINTER(DrafterWeights), ctypes.POINTER(DraftShape),
+                                       ctypes.POINTER(CtxCache), c_vp, c_vp, c_vp, c_size, ctypes.POINTER(Trace),
+                                       c_vp]),
     "hdf_rope_table": (c_int, [ctypes.c_double, c_int, c_i64, c_vp, c_vp, c_vp]),
     "hdf_lm_head_workspace_size": (c_size, [c_i64, c_int, c_i64, c_int]),
     "hdf_lm_head_argmax": (c_int, [c_vp, c_int, c_i64, c_int, c_vp, c_i64, c_float, c_vp, c_vp, c_vp,
@@ -231,6 +242,67 @@ class Drafter:
                                    _p(h_out), _p(ws), ws.numel(), ctypes.byref(tr) if tr is not None else None,
                                    _stream(stream)))
         return h_out
+
+    # ------------------------------------------------ incremental (cached) form
+    def new_cache(self, batch: int, capacity: int, device, zero: bool = False) -> "ContextCache":
+        """Per-layer K_c / V_c cache [n_layers, batch, capacity, d] and the
+        device row counts (zero: an empty cache for every sequence)."""
+        return ContextCache(self.n_layers, batch, capacity, self.d, self.w["embed"].dtype, device, zero)
+
+    def append_workspace_size(self, batch: int, block: int, n_new: int) -> int:
+        sh = self.shape(batch, block, n_new, 0)
+        return load().hdf_ctx_append_workspace_size(ctypes.byref(sh))
+
+    def cached_workspace_size(self, batch: int, block: int, max_ctx: int) -> int:
+        sh = self.shape(batch, block, 0, max_ctx)
+        return load().hdf_draft_block_cached_workspace_size(ctypes.byref(sh))
+
+    def hdf_ctx_append(self, ctx_new: torch.Tensor, cu_new: torch.Tensor, cache: "ContextCache", *, block: int,
+                       ws: Optional[torch.Tensor] = None, stream=None) -> None:
+        batch = cu_new.shape[0] - 1
+        sh = self.shape(batch, block, ctx_new.shape[0], 0)
+        lib = load()
+        if ws is None:
+            ws = torch.empty(max(lib.hdf_ctx_append_workspace_size(ctypes.byref(sh)), 1), dtype=torch.uint8,
+                             device=ctx_new.device)
+        _check(lib.hdf_ctx_append(ctypes.byref(self._w), ctypes.byref(sh), _p(ctx_new), _p(cu_new),
+                                  ctypes.byref(cache.c), _p(ws), ws.numel(), _stream(stream)))
+
+    def hdf_draft_block_cached(self, cache: "ContextCache", anchor: torch.Tensor, *, block: int, max_ctx: int,
+                               h_out: Optional[torch.Tensor] = None, ws: Optional[torch.Tensor] = None,
+                               events: Optional[Sequence] = None, stream=None) -> torch.Tensor:
+        batch = anchor.shape[0]
+        sh = self.shape(batch, block, 0, max_ctx)
+        lib = load()
+        dev = anchor.device
+        if ws is None:
+            ws = torch.empty(max(lib.hdf_draft_block_cached_workspace_size(ctypes.byref(sh)), 1),
+                             dtype=torch.uint8, device=dev)
+        if h_out is None:
+            h_out = torch.empty((batch * block, self.d), dtype=self.w["embed"].dtype, device=dev)
+        tr = None
+        if events is not None:
+            arr = (c_vp * len(events))(*[e.cuda_event for e in events])
+            tr = Trace(ctypes.cast(arr, ctypes.POINTER(c_vp)), len(events))
+            self._keep = arr
+        _check(lib.hdf_draft_block_cached(ctypes.byref(self._w), ctypes.byref(sh), ctypes.byref(cache.c),
+                                          _p(anchor), _p(h_out), _p(ws), ws.numel(),
+                                          ctypes.byref(tr) if tr is not None else None, _stream(stream)))
+        return h_out
+
+
+class ContextCache:
+    """Device tensors of an hdf_ctx_cache: k, v [n_layers, batch, capacity, d]
+    and len [batch] int32 (rows held per sequence)."""
+
+    def __init__(self, n_layers: int, batch: int, capacity: int, d: int, dtype: torch.dtype, device,
+                 zero: bool = False):
+        alloc = torch.zeros if zero else torch.empty
+        self.k = alloc((n_layers, batch, capacity, d), dtype=dtype, device=device)
+        self.v = alloc((n_layers, batch, capacity, d), dtype=dtype, device=device)
+        self.len = torch.zeros((batch,), dtype=torch.int32, device=device)
+        self.capacity = capacity
+        self.c = CtxCache(self.k.data_ptr(), self.v.data_ptr(), self.len.data_ptr(), capacity)
 
 
 # ----------------------------------------------------------------- LM head

@@ -94,3 +94,62 @@ def test_draft_block_host_validation(lib):
     assert lib.hdf_draft_block(ctypes.byref(w), ctypes.byref(bad2), None, None, None, None, None, 0, None, None) == 2
     assert lib.hdf_draft_block(None, ctypes.byref(sh), None, None, None, None, None, 0, None, None) == 1
     assert lib.hdf_draft_block_workspace_size(ctypes.byref(bad)) == 0
+
+
+def _fake_weights(n_layers, rope_max_pos):
+    """Drafter weights whose pointers are aligned but never dereferenced
+    (every call below returns during host validation)."""
+    layers = (hdf.LayerWeights * n_layers)()
+    for i in range(n_layers):
+        for k in ("attn_norm", "wq", "wk", "wv", "wo", "mlp_norm", "wg", "wu", "wd"):
+            setattr(layers[i], k, 4096)
+    w = hdf.DrafterWeights(4096, 4096, 4096, 4096, 4096, 4096, rope_max_pos,
+                           ctypes.cast(layers, ctypes.POINTER(hdf.LayerWeights)))
+    return w, layers
+
+
+def test_ctx_cache_host_validation(lib):
+    v = ctypes.c_void_p
+    w, _keep = _fake_weights(2, 4096 + 16)
+    sh = hdf.DraftShape(1, 4, 16, 2048, 16, 128, 8192, 32768, 2, 4096, 20, 1e-6)   # 20 new rows
+    good = hdf.CtxCache(4096, 8192, 256, 4096)
+    ws = v(1 << 20)
+    # append: no cache, zero capacity, misaligned k, rope table too short, workspace too small
+    assert lib.hdf_ctx_append(ctypes.byref(w), ctypes.byref(sh), v(4096), v(256), None, ws, 1 << 20, None) == 1
+    bad = hdf.CtxCache(4096, 8192, 256, 0)
+    assert lib.hdf_ctx_append(ctypes.byref(w), ctypes.byref(sh), v(4096), v(256), ctypes.byref(bad), ws, 1 << 20,
+                              None) == 2
+    bad = hdf.CtxCache(4100, 8192, 256, 4096)
+    assert lib.hdf_ctx_append(ctypes.byref(w), ctypes.byref(sh), v(4096), v(256), ctypes.byref(bad), ws, 1 << 20,
+                              None) == 4
+    huge = hdf.CtxCache(4096, 8192, 256, 1 << 30)   # batch * capacity >= 2^31 rows
+    assert lib.hdf_ctx_append(ctypes.byref(w), ctypes.byref(sh), v(4096), v(256), ctypes.byref(huge), ws, 1 << 20,
+                              None) == 2
+    w_short, _k2 = _fake_weights(2, 1000)
+    assert lib.hdf_ctx_append(ctypes.byref(w_short), ctypes.byref(sh), v(4096), v(256), ctypes.byref(good), ws,
+                              1 << 20, None) == 2
+    need = lib.hdf_ctx_append_workspace_size(ctypes.byref(sh))
+    assert need == ((20 * 2048 * 2 + 255) // 256) * 256
+    assert lib.hdf_ctx_append(ctypes.byref(w), ctypes.byref(sh), v(4096), v(256), ctypes.byref(good), ws, need - 1,
+                              None) == 5
+    assert lib.hdf_ctx_append(ctypes.byref(w), ctypes.byref(sh), None, v(256), ctypes.byref(good), ws, need,
+                              None) == 1
+    # nothing to append: returns before any launch
+    empty = hdf.DraftShape(1, 4, 16, 2048, 16, 128, 8192, 32768, 2, 4096, 0, 1e-6)
+    assert lib.hdf_ctx_append(ctypes.byref(w), ctypes.byref(empty), None, None, ctypes.byref(good), None, 0,
+                              None) == 0
+    # cached block forward: max_ctx above the capacity, no workspace, empty batch
+    small = hdf.CtxCache(4096, 8192, 256, 1024)
+    assert lib.hdf_draft_block_cached(ctypes.byref(w), ctypes.byref(sh), ctypes.byref(small), v(256), v(4096), ws,
+                                      1 << 20, None, None) == 2
+    assert lib.hdf_draft_block_cached(ctypes.byref(w), ctypes.byref(sh), ctypes.byref(good), v(256), v(4096), None,
+                                      0, None, None) == 5
+    assert lib.hdf_draft_block_cached(ctypes.byref(w), ctypes.byref(sh), None, v(256), v(4096), ws, 1 << 20,
+                                      None, None) == 1
+    nob = hdf.DraftShape(1, 0, 16, 2048, 16, 128, 8192, 32768, 2, 4096, 0, 1e-6)
+    assert lib.hdf_draft_block_cached(ctypes.byref(w), ctypes.byref(nob), ctypes.byref(good), None, None, None, 0,
+                                      None, None) == 0
+    # the cached form needs no context buffers in its workspace
+    cold = hdf.DraftShape(1, 4, 16, 2048, 16, 128, 8192, 32768, 2, 4096, 4 * 4096, 1e-6)
+    assert (lib.hdf_draft_block_cached_workspace_size(ctypes.byref(cold)) + 3 * 4 * 4096 * 2048 * 2
+            <= lib.hdf_draft_block_workspace_size(ctypes.byref(cold)))
