@@ -327,6 +327,11 @@ def run_ours(args, rank, world, local_rank):
                  "mean_accept": round(float(va.float().mean()), 3), "launches": 1}
     del pv, qv
 
+    # ------------------------------------------- warm (incremental) step
+    warm = None
+    if not args.no_warm:
+        warm = measure_warm(cfg, inp, drafter, y, tok.clone(), tgt, stream, min(K, 100), dev, peaks())
+
     # ------------------------------------------------------------ e2e
     # host buffers: the residual of every context token and the targets in,
     # drafts and accepted lengths out, through the same C-ABI calls.
@@ -363,8 +368,140 @@ def run_ours(args, rank, world, local_rank):
         t = torch.tensor([ms, e2e_ms], device=dev)
         torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
         ms, e2e_ms = float(t[0]), float(t[1])
-    return dict(cfg=cfg, ms=ms, ms_staged=ms_staged, e2e_ms=e2e_ms, dur=dur, clk=clk, kl=kl, verify_t1=verify_t1, batch=batch, n_ctx=n_ctx, lens=lens,
+    return dict(cfg=cfg, ms=ms, ms_staged=ms_staged, e2e_ms=e2e_ms, dur=dur, clk=clk, kl=kl, verify_t1=verify_t1,
+                warm=warm, batch=batch, n_ctx=n_ctx, lens=lens,
                 h2d=h2d, d2h=d2h, acc_mean=acc_mean, tok=tok, y=y, inputs=inp, tgt=tgt)
+
+
+# ------------------------------------------- warm (incremental) serving step
+WARM_NEW_ROWS = 5  # new context rows per sequence per round: mean accepted length 4, plus the bonus token
+
+
+def _timing_event():
+    # external: inside graph capture the record becomes a timing node
+    try:
+        return torch.cuda.Event(enable_timing=True, external=True)
+    except TypeError:
+        return torch.cuda.Event(enable_timing=True)
+
+
+def warm_launches(cfg):
+    # reduce; append: norm, one K/V GEMM per layer, length advance; cached
+    # block: 7 kernels per layer and the final norm; LM head (2); accept
+    return 1 + (2 + cfg.n_layers) + (7 * cfg.n_layers + 1) + 2 + 1
+
+
+def measure_warm(cfg, inp, drafter, y, tok_cold, tgt, stream, steps, dev, pk):
+    """One serving round of the incremental path, as one CUDA graph: rewind
+    the cache lengths, reduce the residuals of the WARM_NEW_ROWS newest tokens
+    of every sequence, append them to the K/V cache, block forward over the
+    cache, LM head, accepted length.  The cache holds every other context row
+    (appended once, untimed), so each round drafts over the same contexts as
+    the cold step and must give its drafts exactly."""
+    from paper_2606_26744_gb300 import hdf
+    batch, B, d = cfg.batch, cfg.block, cfg.d
+    lens = inp["ctx_lens"]
+    cu = inp["cu_ctx"].tolist()
+    max_ctx = max(lens)
+    pre = [max(0, t - WARM_NEW_ROWS) for t in lens]
+    new = [t - p for t, p in zip(lens, pre)]
+    w = inp["weights"]
+    with torch.cuda.stream(stream):
+        cache = drafter.new_cache(batch, max(1, max_ctx), dev)
+        idx_pre = torch.cat([torch.arange(cu[i], cu[i] + pre[i]) for i in range(batch)]).to(dev)
+        cu_pre = torch.tensor([0] + list(np.cumsum(pre)), dtype=torch.int32, device=dev)
+        drafter.hdf_ctx_append(y[idx_pre].contiguous(), cu_pre, cache, block=B, stream=stream)
+        len0 = cache.len.clone()
+        idx_new = torch.cat([torch.arange(cu[i] + pre[i], cu[i] + lens[i]) for i in range(batch)]).to(dev)
+        H_new = inp["H"][idx_new].contiguous()
+        Wf, b = inp["Wf"], inp["b"]
+        n_new = int(sum(new))
+        cu_new = torch.tensor([0] + list(np.cumsum(new)), dtype=torch.int32, device=dev)
+        y_new = torch.empty((n_new, d), dtype=cfg.torch_dtype, device=dev)
+        ws_a = torch.empty(max(1, drafter.append_workspace_size(batch, B, n_new)), dtype=torch.uint8, device=dev)
+        ws_c = torch.empty(max(1, drafter.cached_workspace_size(batch, B, max_ctx)), dtype=torch.uint8, device=dev)
+        M = batch * B
+        h = torch.empty((M, d), dtype=cfg.torch_dtype, device=dev)
+        tok = torch.empty(M, dtype=torch.int32, device=dev)
+        zmax = torch.empty(M, dtype=torch.float32, device=dev)
+        ls = torch.empty((M, cfg.vocab), dtype=torch.float32, device=dev) if cfg.logsoftmax else None
+        lmws = torch.empty(hdf.lm_head_workspace_size(M, d, cfg.vocab, cfg.torch_dtype), dtype=torch.uint8,
+                           device=dev)
+        acc = torch.empty(batch, dtype=torch.int32, device=dev)
+        anchor = inp["anchor"].to(dev)
+    stream.synchronize()
+    names = ["reduce", "append", "draft_block_cached", "lm_head", "accept"]
+
+    def wstep(ev=None):
+        def mark(i):
+            if ev is not None:
+                ev[i].record(stream)
+        with torch.cuda.stream(stream):
+            cache.len.copy_(len0, non_blocking=True)
+        mark(0)
+        hdf.hdf_gated_reduce(H_new, Wf, b, y=y_new, stream=stream)
+        mark(1)
+        drafter.hdf_ctx_append(y_new, cu_new, cache, block=B, ws=ws_a, stream=stream)
+        mark(2)
+        drafter.hdf_draft_block_cached(cache, anchor, block=B, max_ctx=max_ctx, h_out=h, ws=ws_c, stream=stream)
+        mark(3)
+        hdf.hdf_lm_head_argmax(h, w["lm_head"], logsoftmax=cfg.logsoftmax, tok=tok, zmax=zmax, ls=ls, ws=lmws,
+                               stream=stream)
+        mark(4)
+        hdf.hdf_accept_len(tok[1:], tgt, n_draft=B - 1, draft_stride=B, batch=batch, accept=acc, stream=stream)
+        mark(5)
+
+    for _ in range(3):
+        wstep()
+    stream.synchronize()
+    if hdf.device_status() != 0:
+        raise RuntimeError("warm step: a device-side check failed")
+    same = bool(torch.equal(tok, tok_cold))
+    if not same:
+        raise RuntimeError("warm step drafts differ from the cold step's")
+    K = steps
+    evs = [[_timing_event() for _ in range(6)] for _ in range(K)]
+    for e in [x for row in evs for x in row]:
+        e.record(stream)
+    stream.synchronize()
+    graph = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(graph, stream=stream):
+        for _ in range(K):
+            wstep()
+    staged = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(staged, stream=stream):
+        for k in range(K):
+            wstep(evs[k])
+    with torch.cuda.stream(stream):
+        graph.replay()
+        staged.replay()
+    stream.synchronize()
+    t0, t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    t0.record(stream)
+    with torch.cuda.stream(stream):
+        graph.replay()
+    t1.record(stream)
+    stream.synchronize()
+    ms = t0.elapsed_time(t1) / K
+    with torch.cuda.stream(stream):
+        staged.replay()
+    stream.synchronize()
+    dur = {n: sum(evs[k][i].elapsed_time(evs[k][i + 1]) for k in range(K)) / K for i, n in enumerate(names)}
+    if not torch.equal(tok, tok_cold):
+        raise RuntimeError("warm step drafts differ from the cold step's after the graph replays")
+    work = stage_work(cfg, n_new, batch, lens)
+    byt = sum(v[0] for v in work.values())
+    gbs = byt / (ms / 1e3) / 1e9
+    out = {"workload": cfg.name, "new_rows_per_seq": WARM_NEW_ROWS, "ctx_per_seq": lens if batch <= 8 else None,
+           "ms": round(ms, 5), "blocks_per_s": round(batch / (ms / 1e3), 2),
+           "stages_us": {n: round(v * 1e3, 2) for n, v in dur.items()},
+           "algorithmic_bytes": int(byt), "gbs": round(gbs, 1), "frac_hbm": round(gbs / pk["hbm_gbs"], 3),
+           "roofline_ms": round(byt / (pk["hbm_gbs"] * 1e9) * 1e3, 4), "launches": warm_launches(cfg),
+           "drafts_equal_cold": same,
+           "timing": "K rounds captured as one CUDA graph, CUDA events around the replay; stage times from a "
+                     "second graph with event records between stages"}
+    del cache
+    return out
 
 
 # DRAM bytes (read + write) per launch from the ncu captures summarised in
@@ -554,6 +691,7 @@ def main():
     ap.add_argument("--config", default="decode", choices=sorted(W.CONFIGS) + ["sweep"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--eager", action="store_true", help="launch the timed steps one by one (no CUDA graph)")
+    ap.add_argument("--no-warm", action="store_true", help="skip the incremental (K/V cache) serving step")
     ap.add_argument("--sweep-n", type=int, nargs="*", default=None, help="token counts of the reducer sweep")
     ap.add_argument("--fc-max-n", type=int, default=262144, help="largest N for the fc comparison")
     args = ap.parse_args()
@@ -607,6 +745,7 @@ def main():
             "reducer": {"gbs": red.get("gbs"), "frac_hbm": red.get("frac"), "us": red["us"]},
             "kl_target": dict(res["kl"], frac_hbm=round(res["kl"]["gbs"] / pk["hbm_gbs"], 3)),
             "verify_t1": res["verify_t1"],
+            "warm_step": res["warm"],
             "stages": stages,
             "e2e": {"value": round(e2e_val, 2), "unit": "blocks/s", "h2d_bytes_per_step": res["h2d"],
                     "d2h_bytes_per_step": res["d2h"]},

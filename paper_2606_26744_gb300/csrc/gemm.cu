@@ -17,9 +17,12 @@
 //                    argmax + sum-exp partials, direct global stores.
 // Split-K: the k_splits CTAs of a tile form one thread-block cluster.  Each
 // leaves its fp32 partial tile in its own shared memory; after a cluster
-// barrier rank 0 sums the ranks' tiles in rank order over distributed shared
-// memory (no global round trip, no atomics) and runs the epilogue.
+// barrier every rank sums one slice of the tile's rows over all ranks, in
+// rank order, over distributed shared memory, and writes the sums into rank
+// 0's partial tile in place (no other rank reads that slice); after a second
+// barrier rank 0 runs the epilogue.  No global round trip, no atomics.
 #include <algorithm>
+#include <atomic>
 #include <climits>
 
 #include "common.cuh"
@@ -41,10 +44,15 @@ template <> struct GT<float> {
   static constexpr uint32_t FMT = 2;  // tf32
 };
 
+// Rings of ~96 KB, so that two CTAs share an SM: two independent producers
+// keep more loads in flight than one CTA with a ring twice as deep
+// (measured on the skinny weight-streaming GEMMs of the draft step).
 constexpr int stages_for(int bn) { return bn >= 256 ? 2 : (bn >= 128 ? 3 : (bn >= 64 ? 4 : 5)); }
-constexpr int kPartialOffset = 12288;  // split-K partial tile, then rank 0's reduced tile, in the drained
+constexpr int kPartialOffset = 12288;  // split-K partial tile (rank 0's is reduced in place), in the drained
                                        // stage memory above the epilogue's scratch (at most 16 x 136 floats)
-static_assert(kPartialOffset + 2 * 128 * 64 * 4 <= 4 * (128 + 64) * 128, "split-K tiles fit the stages (BN <= 64)");
+constexpr bool partial_fits(int bn) { return kPartialOffset + BM * bn * 4 <= stages_for(bn) * (BM + bn) * ROW_BYTES; }
+static_assert(partial_fits(16) && partial_fits(32) && partial_fits(64) && partial_fits(128),
+              "split-K partial tile fits the stage memory (BN <= 128)");
 constexpr int smem_for(int bn) { return stages_for(bn) * (BM + bn) * ROW_BYTES + 1024; }
 
 __device__ __forceinline__ void operand_rows(const Operand& op, int tile_row0, int half, int tile_idx,
@@ -502,15 +510,16 @@ __global__ void __launch_bounds__(128, 1) gemm_kernel(const __grid_constant__ Ge
     cluster_sync_all();  // every rank's partial tile is visible to the cluster
     // Every rank sums a slice of the tile's rows over all ranks (one float4
     // column per thread and round, every source in flight at once, summed in
-    // rank order) and writes the result into rank 0's reduced tile.
-    if (BN <= 64) {
+    // rank order) and writes the result over rank 0's partial of that slice:
+    // the slice is read and written by this rank only.
+    if (BN <= 128) {
       const int k = g.k_splits;
       const uint32_t rank = cluster_rank();
       const int rpr = (BM + k - 1) / k;  // rows per rank
       const int row0 = (int)rank * rpr, nrow = max(0, min(BM, row0 + rpr) - row0);
       constexpr int C4 = BN / 4;
       const uint32_t part_base = smem_u32(part);
-      const uint32_t red_base = map_rank(smem_u32(smem + kPartialOffset + BM * BN * 4), 0u);
+      const uint32_t red_base = map_rank(part_base, 0u);
       for (int it = tid; it < nrow * C4; it += 128) {
         const int r = row0 + it / C4, c4 = it - (it / C4) * C4;
         const uint32_t off = (uint32_t)((r * BN + c4 * 4) * 4);
@@ -532,9 +541,9 @@ __global__ void __launch_bounds__(128, 1) gemm_kernel(const __grid_constant__ Ge
                      : "memory");
       }
     }
-    cluster_sync_all();  // rank 0's reduced tile is complete; no rank reads another's memory any more
+    cluster_sync_all();  // rank 0's tile holds the sums; no rank reads another's memory any more
     if (cluster_rank() == 0 && !aborted) {
-      const float* red = reinterpret_cast<const float*>(smem + kPartialOffset + BM * BN * 4);
+      const float* red = part;
 #pragma unroll 1
       for (int c0 = 0; c0 < BN; c0 += 16) {
         float v[16];
@@ -558,26 +567,64 @@ __global__ void __launch_bounds__(128, 1) gemm_kernel(const __grid_constant__ Ge
   }
 }
 
+// Function attributes of one instantiation, set once per process: the
+// dynamic shared memory and clusters of up to 16 CTAs.
+template <typename T, int BN>
+cudaError_t prepare_bn() {
+  static cudaError_t state = [] {
+    auto k = gemm_kernel<T, BN>;
+    cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, smem_for(BN));
+    if (e == cudaSuccess) e = cudaFuncSetAttribute(k, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+    return e;
+  }();
+  return state;
+}
+
 template <typename T, int BN>
 cudaError_t launch_bn(const GemmArgs& g, cudaStream_t s) {
-  auto k = gemm_kernel<T, BN>;
-  const int smem = smem_for(BN);
-  static bool attr_set = false;  // per instantiation; set once per process
   cudaError_t e;
-  if (!attr_set) {
-    if ((e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, smem)) != cudaSuccess)
-      return e;
-    attr_set = true;
-  }
-  if (g.k_splits < 1 || g.k_splits > 16 || (g.k_splits > 1 && BN > 64)) return cudaErrorInvalidValue;
+  if ((e = prepare_bn<T, BN>()) != cudaSuccess) return e;
+  if (g.k_splits < 1 || g.k_splits > 16 || (g.k_splits > 1 && BN > 128)) return cudaErrorInvalidValue;
   const long long tiles = (long long)((g.M + BM - 1) / BM) * ((g.N + BN - 1) / BN) * g.k_splits;
-  static bool cluster_attr_set = false;
-  if (g.k_splits > 8 && !cluster_attr_set) {
-    if ((e = cudaFuncSetAttribute(k, cudaFuncAttributeNonPortableClusterSizeAllowed, 1)) != cudaSuccess) return e;
-    cluster_attr_set = true;
-  }
   // the splits of one tile are consecutive blocks: one cluster
-  return launch_kernel(k, dim3((unsigned)tiles), dim3(128), (size_t)smem, s, (unsigned)g.k_splits, g);
+  return launch_kernel(gemm_kernel<T, BN>, dim3((unsigned)tiles), dim3(128), (size_t)smem_for(BN), s,
+                       (unsigned)g.k_splits, g);
+}
+
+// CTAs resident at once when the grid is made of clusters of `cluster` CTAs
+// (the occupancy API packs clusters into GPCs); -1 if it cannot be asked.
+template <typename T, int BN>
+int resident_ctas_bn(int cluster) {
+  if (prepare_bn<T, BN>() != cudaSuccess) return -1;
+  cudaLaunchConfig_t cfg = {};
+  cudaLaunchAttribute attr;
+  attr.id = cudaLaunchAttributeClusterDimension;
+  attr.val.clusterDim.x = (unsigned)cluster;
+  attr.val.clusterDim.y = 1;
+  attr.val.clusterDim.z = 1;
+  cfg.gridDim = dim3((unsigned)cluster * 64u);
+  cfg.blockDim = dim3(128);
+  cfg.dynamicSmemBytes = (size_t)smem_for(BN);
+  cfg.attrs = &attr;
+  cfg.numAttrs = 1;
+  int n = 0;
+  if (cudaOccupancyMaxActiveClusters(&n, gemm_kernel<T, BN>, &cfg) != cudaSuccess || n <= 0) {
+    cudaGetLastError();
+    return -1;
+  }
+  return n * cluster;
+}
+
+template <typename T>
+int resident_ctas_t(int bn, int cluster) {
+  switch (bn) {
+    case 16: return resident_ctas_bn<T, 16>(cluster);
+    case 32: return resident_ctas_bn<T, 32>(cluster);
+    case 64: return resident_ctas_bn<T, 64>(cluster);
+    case 128: return resident_ctas_bn<T, 128>(cluster);
+    case 256: return resident_ctas_bn<T, 256>(cluster);
+    default: return -1;
+  }
 }
 
 template <typename T>
@@ -595,6 +642,20 @@ cudaError_t launch_t(const GemmArgs& g, cudaStream_t s) {
 }  // namespace
 
 int gemm_stages(int, int bn) { return stages_for(bn); }
+
+int gemm_resident_ctas(int dtype, int bn, int cluster) {
+  if (cluster < 1 || cluster > 16) return -1;
+  const int bi = bn == 16 ? 0 : bn == 32 ? 1 : bn == 64 ? 2 : bn == 128 ? 3 : bn == 256 ? 4 : -1;
+  if (bi < 0) return -1;
+  static std::atomic<int> cache[2][5][17];  // 0: not asked yet
+  std::atomic<int>& c = cache[dtype == HDF_BF16 ? 0 : 1][bi][cluster];
+  int v = c.load(std::memory_order_relaxed);
+  if (v == 0) {
+    v = dtype == HDF_BF16 ? resident_ctas_t<__nv_bfloat16>(bn, cluster) : resident_ctas_t<float>(bn, cluster);
+    c.store(v, std::memory_order_relaxed);
+  }
+  return v;
+}
 size_t gemm_smem_bytes(int, int bn) { return (size_t)smem_for(bn); }
 
 cudaError_t launch_gemm(const GemmArgs& g, cudaStream_t s) {

@@ -5,6 +5,7 @@
 #include <cudaTypedefs.h>
 
 #include <algorithm>
+#include <climits>
 #include <cmath>
 #include <cstdarg>
 #include <cstdio>
@@ -117,22 +118,42 @@ struct SplitPlan {
   int bn, k_splits, tiles;
 };
 
-// Weights-as-A GEMM (rows = output features, columns = tokens): K-split so
-// that the grid fills about one wave of two CTAs per SM (a second wave would
-// only start when the first ends), each split over >= 4 k-blocks; the splits
-// of a tile run as one cluster of at most 16 CTAs.
+// Weights-as-A GEMM (rows = output features, columns = tokens), bound by
+// streaming the operands through shared memory.  Two CTAs share an SM, and
+// the CTAs resident at once are twice what the occupancy API gives per
+// cluster size (it packs clusters into GPCs but counts one CTA per SM for a
+// kernel holding tensor memory; else two per SM).  A CTA's time is about the
+// bytes it loads, k-blocks x (128 + bn) rows; a split pays 2 + bn/8 k-blocks
+// for storing, exchanging and summing its partial tile and waiting for the
+// slowest rank of its cluster (fitted to measured plan sweeps).  The plan
+// (tile width: the one covering the tokens, or 128 when that is 256; K split
+// with >= 4 k-blocks per split, at most 16, one thread-block cluster per tile)
+// is the one with the least waves x cost per CTA.
 SplitPlan plan_swap(int dtype, long long M, long long N, long long K) {
-  SplitPlan p;
-  p.bn = pick_bn(N);
   const int bk = dtype == HDF_BF16 ? 64 : 32;
-  p.tiles = (int)(((M + 127) / 128) * ((N + p.bn - 1) / p.bn));
   const int num_kb = (int)((K + bk - 1) / bk);
-  const int target = 2 * num_sms();
-  int splits = p.bn <= 64 ? std::max(1, target / p.tiles) : 1;  // split tiles are at most 64 wide
-  splits = std::min(std::min(splits, 16), std::max(1, num_kb / 4));
-  const int kb_per = (num_kb + splits - 1) / splits;
-  p.k_splits = (num_kb + kb_per - 1) / kb_per;
-  return p;
+  const int bn0 = pick_bn(N);
+  const int widths[2] = {bn0, bn0 == 256 ? 128 : 0};
+  SplitPlan best{bn0, 1, (int)(((M + 127) / 128) * ((N + bn0 - 1) / bn0))};
+  long long best_cost = LLONG_MAX;
+  for (int bn : widths) {
+    if (bn == 0) continue;
+    const long long tiles = ((M + 127) / 128) * ((N + bn - 1) / bn);
+    const int max_splits = bn <= 128 ? std::min(16, std::max(1, num_kb / 4)) : 1;
+    for (int s = 1; s <= max_splits; ++s) {
+      const int kb_per = (num_kb + s - 1) / s;
+      if ((num_kb + kb_per - 1) / kb_per != s) continue;  // no empty split
+      const int api = gemm_resident_ctas(dtype, bn, s);
+      const long long slots = 2LL * (api > 0 ? api : num_sms());
+      const long long waves = (tiles * s + slots - 1) / slots;
+      const long long cost = waves * (kb_per + (s > 1 ? 2 + bn / 8 : 0)) * (128 + bn);
+      if (cost < best_cost) {
+        best_cost = cost;
+        best = SplitPlan{bn, s, (int)tiles};
+      }
+    }
+  }
+  return best;
 }
 
 void init_gemm(GemmArgs& g, int dtype, long long M, long long N, long long K, const SplitPlan& p) {

@@ -109,7 +109,7 @@ struct GemmArgs {
   int M, N, K;
   int dtype;            // HDF_BF16 or HDF_F32 (tf32)
   int bn;               // tile width along N: 16, 32, 64, 128 or 256
-  int k_splits;         // 1..16; > 1 launches the splits of each tile as one thread-block cluster
+  int k_splits;         // 1..16 (> 1 needs bn <= 128): the splits of a tile run as one thread-block cluster
   int pre_operand;      // 1: A, 2: B does not depend on earlier kernels (weights) and is loaded
                         // before pdl_wait(); 0: neither
   int group_n;          // raster: n-tiles swept together
@@ -118,6 +118,9 @@ struct GemmArgs {
 };
 cudaError_t launch_gemm(const GemmArgs& g, cudaStream_t s);
 int gemm_stages(int dtype, int bn);
+// CTAs of the GEMM resident at once in clusters of `cluster` (1..16); -1 when
+// the device cannot be asked
+int gemm_resident_ctas(int dtype, int bn, int cluster);
 size_t gemm_smem_bytes(int dtype, int bn);
 
 // ----------------------------------------------------- small kernels ----

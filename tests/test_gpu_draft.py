@@ -134,3 +134,17 @@ def test_serve_widths_short_ragged_context():
 def test_large_widths_short_context():
     cfg = W.scaled(W.CONFIGS["large"], vocab=8192, n_layers=1)
     run_step(cfg, seed=10, ctx_lens=[300, 129])
+
+
+def test_batch8_block16_128_tokens():
+    """128 block tokens (the large workload's batch x block): the block GEMMs
+    take 128- or 64-wide tiles with a K split reduced across a cluster."""
+    cfg = W.DraftConfig("b8", m=4, d=1024, block=16, n_layers=2, n_heads=8, head_dim=128, ffn=2816,
+                        vocab=8192, batch=8, ctx_len=200)
+    run_step(cfg, seed=11, ctx_lens=[200, 3, 64, 65, 130, 1, 199, 90])
+
+
+def test_batch6_block16_96_tokens_fp32():
+    cfg = W.DraftConfig("b6f32", m=4, d=256, block=16, n_layers=1, n_heads=2, head_dim=128, ffn=1024,
+                        vocab=2048, batch=6, ctx_len=70, dtype="f32")
+    run_step(cfg, seed=12, ctx_lens=[70, 1, 5, 64, 33, 17])
