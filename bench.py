@@ -508,9 +508,13 @@ def measure_warm(cfg, inp, drafter, y, tok_cold, tgt, stream, steps, dev, pk):
 # profiles/*_decode.md, decode workload only; an entry must be removed when
 # its kernel changes.
 NCU_DRAM_BYTES_DECODE = {
-    "L0.ctx_kv_gemm": 26287872 + 1280,
-    "lm_head": 134363136 + 3645184,
-    "L0.attention": 17014528,
+    "L0.ctx_kv_gemm": 26288384 + 2816,
+    "L0.qkv_gemm": 25340160,
+    "L0.o_gemm": 8668928,
+    "L0.gate_up_gemm": 67264512 + 452864,
+    "L0.down_gemm": 34031360,
+    "lm_head": 134365952 + 3178496,
+    "L0.attention": 17016576,
     "gated_reduce": 33669120,
 }
 
