@@ -107,17 +107,19 @@ HDF_API int hdf_gated_reduce(const void* H, int dtype, int64_t n_tokens, int m, 
                      const float* alpha_override,
                      void* y, float* alpha_out, hdf_stream_t stream);
 
-/* Kernel choice of hdf_gated_reduce; both compute Eq. 1 and agree within
+/* Kernel choice of hdf_gated_reduce; all compute Eq. 1 and agree within
  * fp32 summation order.  HDF_REDUCE_GENERAL: one CTA streams whole tokens and
  * re-reads them from L2 for the weighted sum (every dtype and option).
  * HDF_REDUCE_CLUSTER: 8-CTA clusters split d, keep W_f slices in shared
- * memory and exchange the gate partials over distributed shared memory
- * (bf16, m in {1,2,4}, d % 512 == 0, no alpha_override or path_norm_w; the
- * general kernel runs otherwise).  HDF_REDUCE_AUTO (the default) takes the
- * general kernel, the faster of the two on every shape measured.
- * Process-wide; returns HDF_ERR_INVALID_ARG for another value.  The paper
- * has no counterpart: it is a tuning and test hook. */
-enum { HDF_REDUCE_AUTO = 0, HDF_REDUCE_GENERAL = 1, HDF_REDUCE_CLUSTER = 2 };
+ * memory and exchange the gate partials of small token batches over
+ * distributed shared memory.  HDF_REDUCE_TILE: 8-CTA clusters split d over
+ * tiles of 32 tokens, gate dots on the tensor cores, one exchange per tile.
+ * CLUSTER and TILE need bf16, m in {1,2,4}, d % 512 == 0 and neither
+ * alpha_override nor path_norm_w; the general kernel runs otherwise.
+ * HDF_REDUCE_AUTO (the default) takes the fastest kernel measured for the
+ * shape.  Process-wide; returns HDF_ERR_INVALID_ARG for another value.  The
+ * paper has no counterpart: it is a tuning and test hook. */
+enum { HDF_REDUCE_AUTO = 0, HDF_REDUCE_GENERAL = 1, HDF_REDUCE_CLUSTER = 2, HDF_REDUCE_TILE = 3 };
 HDF_API int hdf_set_reduce_path(int path);
 
 /* Generic fc reducer of vanilla DFlash (Sec. 2.2, Table 1 "generic fc"),

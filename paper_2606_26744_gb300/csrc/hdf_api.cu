@@ -105,6 +105,22 @@ int make_map(CUtensorMap* m, const void* ptr, int dtype, long long rows, long lo
   return HDF_OK;
 }
 
+// 3-D view of a bf16 H [n_tokens, m, d]: {64 elements, tokens, 128-byte
+// chunks of a token row}, 128-byte swizzle, the given box.
+int make_chunk_map(CUtensorMap* hm, const void* H, long long n_tokens, int m, int d, const unsigned box[3]) {
+  auto fn = encode_fn();
+  if (!fn) return fail(HDF_ERR_CUDA, "cuTensorMapEncodeTiled unavailable");
+  cuuint64_t dims[3] = {64, (cuuint64_t)n_tokens, (cuuint64_t)((long long)m * d / 64)};
+  cuuint64_t strides[2] = {(cuuint64_t)((long long)m * d * 2), 128};
+  cuuint32_t bx[3] = {box[0], box[1], box[2]};
+  cuuint32_t estr[3] = {1, 1, 1};
+  CUresult r = fn(hm, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(H), dims, strides, bx, estr,
+                  CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_NONE,
+                  CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  if (r != CUDA_SUCCESS) return fail(HDF_ERR_CUDA, "cuTensorMapEncodeTiled (3-D view of H) failed (%d)", (int)r);
+  return HDF_OK;
+}
+
 // ------------------------------------------------------------ GEMM plans
 int pick_bn(long long n) {
   if (n <= 16) return 16;
@@ -278,7 +294,7 @@ static std::atomic<int> g_reduce_path{HDF_REDUCE_AUTO};
 
 int hdf_set_reduce_path(int path) {
   g_err.clear();
-  if (path != HDF_REDUCE_AUTO && path != HDF_REDUCE_GENERAL && path != HDF_REDUCE_CLUSTER)
+  if (path != HDF_REDUCE_AUTO && path != HDF_REDUCE_GENERAL && path != HDF_REDUCE_CLUSTER && path != HDF_REDUCE_TILE)
     return fail(HDF_ERR_INVALID_ARG, "reduce path %d", path);
   g_reduce_path.store(path);
   return HDF_OK;
@@ -302,6 +318,7 @@ int hdf_gated_reduce(const void* H, int dtype, int64_t n_tokens, int m, int d, c
   if (!std::isfinite(rms_eps) || !std::isfinite(gate_scale) || !std::isfinite(gate_offset) ||
       !std::isfinite(path_norm_eps) || rms_eps < 0 || path_norm_eps < 0)
     return fail(HDF_ERR_INVALID_ARG, "non-finite or negative scalar");
+  int rc;
   ReduceArgs a;
   a.H = H;
   a.Wf = Wf;
@@ -320,20 +337,18 @@ int hdf_gated_reduce(const void* H, int dtype, int64_t n_tokens, int m, int d, c
   a.status = device_status_ptr();
   unsigned box[3];
   const int path = g_reduce_path.load();
+  unsigned tail_box[3];
+  if (path == HDF_REDUCE_TILE && reduce_tile_boxes(a, dtype, box, tail_box)) {
+    CUtensorMap hm[2];
+    if ((rc = make_chunk_map(&hm[0], H, n_tokens, m, d, box))) return rc;
+    if ((rc = make_chunk_map(&hm[1], H, n_tokens, m, d, tail_box))) return rc;
+    CK(launch_gated_reduce_tile(a, hm, (cudaStream_t)stream), "gated_reduce tile launch");
+    return HDF_OK;
+  }
   const bool cluster_wanted = path == HDF_REDUCE_CLUSTER;  // auto: the general kernel, faster on every shape measured
   if (cluster_wanted && reduce_cluster_box(a, dtype, box)) {
-    // 3-D view of H: {64 elements, tokens, 128-byte chunks of a token row}
-    auto fn = encode_fn();
-    if (!fn) return fail(HDF_ERR_CUDA, "cuTensorMapEncodeTiled unavailable");
     CUtensorMap hm;
-    cuuint64_t dims[3] = {64, (cuuint64_t)n_tokens, (cuuint64_t)((long long)m * d / 64)};
-    cuuint64_t strides[2] = {(cuuint64_t)((long long)m * d * 2), 128};
-    cuuint32_t bx[3] = {box[0], box[1], box[2]};
-    cuuint32_t estr[3] = {1, 1, 1};
-    CUresult r = fn(&hm, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(H), dims, strides, bx, estr,
-                    CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_NONE,
-                    CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
-    if (r != CUDA_SUCCESS) return fail(HDF_ERR_CUDA, "cuTensorMapEncodeTiled (3-D view of H) failed (%d)", (int)r);
+    if ((rc = make_chunk_map(&hm, H, n_tokens, m, d, box))) return rc;
     CK(launch_gated_reduce_cluster(a, &hm, (cudaStream_t)stream), "gated_reduce cluster launch");
     return HDF_OK;
   }

@@ -56,6 +56,12 @@ cudaError_t launch_gated_reduce(const ReduceArgs& a, int dtype, cudaStream_t s);
 // when the shape or options need the general kernel above.
 bool reduce_cluster_box(const ReduceArgs& a, int dtype, unsigned box[3]);
 cudaError_t launch_gated_reduce_cluster(const ReduceArgs& a, const CUtensorMap* h_map, cudaStream_t s);
+// bf16 tile path: boxes {64, 32, C} and {64, 32, tail} of the 3-D view {64
+// elements, tokens, 128-byte chunks} of H (128-byte swizzle) that the caller
+// encodes as h_maps[0], h_maps[1]; false when the shape or options need the
+// general kernel.
+bool reduce_tile_boxes(const ReduceArgs& a, int dtype, unsigned box[3], unsigned tail_box[3]);
+cudaError_t launch_gated_reduce_tile(const ReduceArgs& a, const CUtensorMap* h_maps, cudaStream_t s);
 
 // --------------------------------------------------------------- GEMM ----
 // D[M, N] = A[M, K] * B[N, K]^T, both operands K-major, loaded by TMA with

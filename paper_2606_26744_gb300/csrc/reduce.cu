@@ -832,4 +832,460 @@ cudaError_t launch_gated_reduce_cluster(const ReduceArgs& a, const CUtensorMap* 
   }
 }
 
+// ===========================================================================
+// bf16 tile path (persistent, warp-specialised).
+//
+// A cluster of TP_S = 8 CTAs walks tiles of TP_T = 32 consecutive tokens; CTA
+// rank c owns elements [c*E, (c+1)*E) of each of the m paths (E = d/8), so
+// its W_f slice (m x m*E) stays in shared memory.  Roles, meeting only at
+// mbarriers:
+//   producer warp   streams pass 1 of every tile from HBM into a 128 KB ring:
+//                   one TMA box per stage from the 3-D view {64 elements,
+//                   tokens, 128-byte chunks} of H, 4 chunks (512 contiguous
+//                   bytes) of 32 tokens, landing as planes [32 tokens][64
+//                   elements] with the 128-byte swizzle; it never waits on
+//                   the gates, so HBM streaming continues across tiles
+//   2 gate warps    one per 16-token row tile: the m gate dots on mma.sync
+//                   m16n8k16 (tokens are the rows, the W_f slice is B) and
+//                   the sums of squares from the same A fragments; each sends
+//                   its [16 tokens][m + 1] partials to every rank with
+//                   st.async, which completes the receiver's exchange
+//                   mbarrier on bytes
+//   alpha warp      on every rank: waits for the 16 senders of a tile, sums
+//                   each token's partials over the 8 ranks in rank order (so
+//                   every rank gets the same alpha, Eq. 1) and publishes alpha
+//   8 weighted      y = sum_j alpha_j H_j for the CTA's slice of the tile,
+//   warps           reading H again from L2 (streamed microseconds before)
+//                   with 16 loads in flight per lane, one store per output
+// Gate warps run at most TP_LA tiles ahead of their own alpha warp, which
+// bounds how far any rank runs ahead in the exchange (TP_NX buffers).  H comes
+// from HBM once, W_f once per CTA.  Every wait is time-limited.
+namespace {
+
+constexpr int TP_S = 8;                    // CTAs per cluster
+constexpr int TP_T = 32;                   // tokens per tile
+constexpr int TP_C = 4;                    // 128-byte chunks per token in a box
+constexpr int TP_PLANE = TP_T * 128;       // one [32 tokens x 64 elements] bf16 plane
+constexpr int TP_SB = TP_C * TP_PLANE;     // bytes per ring stage
+constexpr int TP_NST = 8;                  // ring stages (128 KB)
+constexpr int TP_NGW = 4;                  // gate warps: (row tile, box parity)
+constexpr int TP_NWW = 8;                  // weighted warps
+constexpr int TP_THR = 32 * (2 + TP_NGW + TP_NWW);
+constexpr int TP_LA = 2;                   // gate warps run at most this many tiles ahead of the alpha warp
+constexpr int TP_NX = 2 * TP_LA + 2;       // exchange buffers
+constexpr int TP_NAB = 3;                  // alpha buffers
+constexpr int TP_PS = 8;                   // floats per token in an exchange row (m + 1 <= 5 used)
+constexpr int TP_XBYTES = TP_S * TP_T * TP_PS * 4;  // one tile's partials from all senders
+constexpr int TP_U = 4;                    // weighted outputs per lane and round
+
+struct TileGeo {
+  int ec;    // elements per path in a CTA slice (multiple of 64)
+  int nkb;   // 128-byte chunks per path slice
+  int ngrp;  // boxes per path slice: ngrp - 1 of TP_C chunks, then one of tail chunks
+  int tail;  // chunks in the last box of a path slice (1..TP_C)
+  int wrow;  // row stride (elements) of the W_f slice in shared memory
+  long long ntiles;
+};
+struct TileMaps {
+  CUtensorMap main;  // box {64, 32, TP_C}
+  CUtensorMap tail;  // box {64, 32, tail}
+};
+
+__device__ __forceinline__ void st_async_v4(uint32_t addr, float4 v, uint32_t bar) {
+  asm volatile("st.async.shared::cluster.mbarrier::complete_tx::bytes.v4.f32 [%0], {%1,%2,%3,%4}, [%5];" ::"r"(addr),
+               "f"(v.x), "f"(v.y), "f"(v.z), "f"(v.w), "r"(bar)
+               : "memory");
+}
+
+template <int M>
+__global__ void __launch_bounds__(TP_THR, 1) gated_reduce_tile_kernel(const ReduceArgs a,
+                                                                      const __grid_constant__ TileMaps maps,
+                                                                      const TileGeo geo) {
+  extern __shared__ uint8_t tp_smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(tp_smem_raw) + 1023) &
+                                             ~static_cast<uintptr_t>(1023));
+  uint8_t* ring = smem;                                                              // [NST][SB]
+  float* xbuf = reinterpret_cast<float*>(smem + TP_NST * TP_SB);                     // [NX][S][T][PS]
+  float* red = xbuf + TP_NX * TP_S * TP_T * TP_PS;                                  // [2 halves][32][PS]
+  float* alpha_s = red + TP_NGW * 16 * TP_PS;                                        // [NAB][T][4]
+  __nv_bfloat16* wsl = reinterpret_cast<__nv_bfloat16*>(alpha_s + TP_NAB * TP_T * 4);  // [M][wrow]
+  __shared__ __align__(8) uint64_t full_bar[TP_NST];
+  __shared__ __align__(8) uint64_t empty_bar[TP_NST];
+  __shared__ __align__(8) uint64_t xfull[TP_NX];
+  __shared__ __align__(8) uint64_t xdone[TP_NX];
+  __shared__ __align__(8) uint64_t alpha_ready[TP_NAB];
+  __shared__ __align__(8) uint64_t alpha_free[TP_NAB];
+  __shared__ float bias_s[4];
+  __shared__ volatile int abort_flag;
+
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  pdl_launch_dependents();
+  const uint32_t rank = cluster_rank(), cid = cluster_id_x(), ncl = n_clusters_x();
+  const long long N = a.n_tokens;
+  const int d = a.d, ec = geo.ec, ngrp = geo.ngrp, NB = M * ngrp;  // boxes per tile
+  const long long nl = geo.ntiles > (long long)cid ? (geo.ntiles - cid + ncl - 1) / ncl : 0;
+
+  {  // W_f slice: wsl[j][p*ec + e] = W_f[j][p*d + rank*ec + e]
+    const __nv_bfloat16* Wf = reinterpret_cast<const __nv_bfloat16*>(a.Wf);
+    const int v8 = ec / 8, per_row = M * v8;
+    for (int i = tid; i < M * per_row; i += TP_THR) {
+      const int j = i / per_row, r = i - j * per_row, pth = r / v8, e8 = r - pth * v8;
+      const uint4 v = __ldg(reinterpret_cast<const uint4*>(Wf + (size_t)j * M * d + (size_t)pth * d +
+                                                           (size_t)rank * ec + e8 * 8));
+      *reinterpret_cast<uint4*>(wsl + (size_t)j * geo.wrow + pth * ec + e8 * 8) = v;
+    }
+  }
+  if (tid < M) bias_s[tid] = a.b[tid];
+  if (tid == 0) {
+    for (int i = 0; i < TP_NST; ++i) {
+      mbar_init(smem_u32(&full_bar[i]), 1);
+      mbar_init(smem_u32(&empty_bar[i]), 2);  // the two gate warps (row tiles) of the box's parity
+    }
+    for (int i = 0; i < TP_NX; ++i) {
+      mbar_init(smem_u32(&xfull[i]), 1);  // completes on the bytes of every sender
+      mbar_init(smem_u32(&xdone[i]), 1);
+    }
+    for (int i = 0; i < TP_NAB; ++i) {
+      mbar_init(smem_u32(&alpha_ready[i]), 1);
+      mbar_init(smem_u32(&alpha_free[i]), TP_NWW);
+    }
+    abort_flag = 0;
+    fence_mbar_init();
+    for (int b = 0; b < TP_NX && b < nl; ++b) mbar_arrive_expect_tx(smem_u32(&xfull[b]), TP_XBYTES);
+  }
+  __syncthreads();
+  cluster_sync_all();  // every rank's barriers exist and are armed before anyone signals them
+  pdl_wait();          // H and y may belong to the kernels before
+
+  // a wait every lane of the warp takes; false for the whole warp on time-out
+  // or when another role has given up
+  auto warp_wait = [&](uint32_t bar, uint32_t parity, bool cluster_scope) -> bool {
+    bool got = cluster_scope ? mbar_wait_cluster(bar, parity, a.status) : mbar_wait(bar, parity, a.status);
+    got = __all_sync(0xffffffffu, got) && !__any_sync(0xffffffffu, abort_flag != 0);
+    if (!got && lane == 0) abort_flag = 1;
+    return got;
+  };
+  auto arrive = [&](uint64_t* bar) {
+    if (lane == 0) asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(bar)) : "memory");
+  };
+
+  if (warp == 0) {
+    // ------------------------------------------------------------ producer
+    long long g = 0;  // stages issued
+    for (long long i = 0; i < nl; ++i) {
+      const long long t0 = ((long long)cid + i * ncl) * TP_T;
+      bool ok = true;
+      for (int j = 0; j < NB; ++j, ++g) {
+        const int s = (int)(g % TP_NST);
+        if (!warp_wait(smem_u32(&empty_bar[s]), (uint32_t)((g / TP_NST) & 1) ^ 1u, false)) {
+          ok = false;
+          break;
+        }
+        const int pth = j / ngrp, grp = j - pth * ngrp;
+        if (lane == 0) {
+          const bool last = grp == ngrp - 1;
+          const uint32_t fb = smem_u32(&full_bar[s]);
+          mbar_arrive_expect_tx(fb, (last ? geo.tail : TP_C) * TP_PLANE);
+          tma_load_3d(smem_u32(ring + s * TP_SB), last ? &maps.tail : &maps.main, 0, (int)t0,
+                      (pth * d + (int)rank * ec) / 64 + grp * TP_C, fb);
+        }
+        __syncwarp();
+      }
+      if (!ok) break;
+    }
+    // no copy may still be landing when the CTA exits
+    for (long long k = g > TP_NST ? g - TP_NST : 0; k < g; ++k)
+      if (!mbar_wait(smem_u32(&full_bar[k % TP_NST]), (uint32_t)((k / TP_NST) & 1), a.status)) break;
+  } else if (warp <= TP_NGW) {
+    // --------------------------------------------------------------- gates
+    // warp (rt, hb): tokens 16*rt .. 16*rt + 15 of the boxes j with j % 2 == hb
+    const int gw = warp - 1, rt = gw & 1, hb = gw >> 1;
+    const int g8 = lane >> 2, q = lane & 3;
+    const __nv_bfloat16* wrowp = wsl + (size_t)(g8 < M ? g8 : 0) * geo.wrow + 2 * q;
+    const int row = rt * 16 + (lane & 15), hsel = lane >> 4;
+    for (long long i = 0; i < nl; ++i) {
+      float acc[2][4] = {{0.f, 0.f, 0.f, 0.f}, {0.f, 0.f, 0.f, 0.f}};  // two chains: plane parity
+      unsigned long long sq0[2] = {0ull, 0ull}, sq1[2] = {0ull, 0ull};
+      bool ok = true;
+      for (int j = hb; j < NB; j += 2) {
+        const long long gs = i * NB + j;  // stage counter
+        const int s = (int)(gs % TP_NST);
+        if (!warp_wait(smem_u32(&full_bar[s]), (uint32_t)((gs / TP_NST) & 1), false)) {
+          ok = false;
+          break;
+        }
+        const int pth = j / ngrp, grp = j - pth * ngrp;
+        const int nc = grp == ngrp - 1 ? geo.tail : TP_C;
+        const uint32_t sbase = smem_u32(ring + s * TP_SB);
+        const __nv_bfloat16* wk = wrowp + (pth * geo.nkb + grp * TP_C) * 64;
+#pragma unroll
+        for (int c = 0; c < TP_C; ++c) {
+          if (c < nc) {
+            // a plane's fragments first (loads in flight together), then its arithmetic
+            uint32_t af[4][4], bf[4][2];
+#pragma unroll
+            for (int kk = 0; kk < 4; ++kk) {
+              const int chunk = kk * 2 + hsel;
+              ldsm_x4(sbase + c * TP_PLANE + row * 128 + ((chunk ^ (row & 7)) << 4), af[kk][0], af[kk][1],
+                      af[kk][2], af[kk][3]);
+              bf[kk][0] = g8 < M ? *reinterpret_cast<const uint32_t*>(wk + c * 64 + kk * 16) : 0u;
+              bf[kk][1] = g8 < M ? *reinterpret_cast<const uint32_t*>(wk + c * 64 + kk * 16 + 8) : 0u;
+            }
+#pragma unroll
+            for (int kk = 0; kk < 4; ++kk) {
+              mma16816(acc[kk & 1], af[kk], bf[kk][0], bf[kk][1]);
+              sq_acc2(sq0[kk & 1], af[kk][0]);  // row g8
+              sq_acc2(sq0[kk & 1], af[kk][2]);
+              sq_acc2(sq1[kk & 1], af[kk][1]);  // row g8 + 8
+              sq_acc2(sq1[kk & 1], af[kk][3]);
+            }
+          }
+        }
+        __syncwarp();
+        arrive(&empty_bar[s]);
+      }
+      // this warp's [16 tokens][m + 1] partials into red[hb]; the hb = 0 warps
+      // add the hb = 1 halves and send one row per lane to every rank
+      float* rw = red + ((size_t)hb * TP_T + rt * 16) * TP_PS;
+      {
+        float s0 = sum2(sq0[0]) + sum2(sq0[1]), s1 = sum2(sq1[0]) + sum2(sq1[1]);
+        s0 += __shfl_xor_sync(0xffffffffu, s0, 1);
+        s0 += __shfl_xor_sync(0xffffffffu, s0, 2);
+        s1 += __shfl_xor_sync(0xffffffffu, s1, 1);
+        s1 += __shfl_xor_sync(0xffffffffu, s1, 2);
+        if (2 * q < M) {
+          rw[g8 * TP_PS + 2 * q] = acc[0][0] + acc[1][0];
+          rw[(g8 + 8) * TP_PS + 2 * q] = acc[0][2] + acc[1][2];
+        }
+        if (2 * q + 1 < M) {
+          rw[g8 * TP_PS + 2 * q + 1] = acc[0][1] + acc[1][1];
+          rw[(g8 + 8) * TP_PS + 2 * q + 1] = acc[0][3] + acc[1][3];
+        }
+        if (q == 0) {
+          rw[g8 * TP_PS + M] = s0;
+          rw[(g8 + 8) * TP_PS + M] = s1;
+        }
+      }
+      // one decision for the four gate warps (named barrier 3): all go on or all stop
+      uint32_t go;
+      asm volatile(
+          "{\n .reg .pred p, q;\n setp.ne.u32 q, %1, 0;\n bar.red.and.pred p, 3, %2, q;\n selp.u32 %0, 1, 0, p;\n}\n"
+          : "=r"(go)
+          : "r"((uint32_t)ok), "n"(32 * TP_NGW)
+          : "memory");
+      if (!go) break;
+      bool sent = true;
+      if (hb == 0) {
+        // credit: this rank's alpha warp has read tile i - LA, so every rank
+        // has read the buffer this tile's partials go to
+        if (i >= TP_LA) {
+          const long long c = i - TP_LA;
+          sent = warp_wait(smem_u32(&xdone[c % TP_NX]), (uint32_t)((c / TP_NX) & 1), false);
+        }
+        if (sent && lane < 16) {
+          const int b = (int)(i % TP_NX);
+          const float* r0 = red + (size_t)(rt * 16 + lane) * TP_PS;
+          const float* r1 = r0 + TP_T * TP_PS;
+          const float4 a0 = *reinterpret_cast<const float4*>(r0), a1 = *reinterpret_cast<const float4*>(r1);
+          const float4 lo = make_float4(a0.x + a1.x, a0.y + a1.y, a0.z + a1.z, a0.w + a1.w);
+          const float4 hi = make_float4(r0[4] + r1[4], 0.f, 0.f, 0.f);
+          const uint32_t lx = smem_u32(xbuf + (((size_t)b * TP_S + rank) * TP_T + rt * 16 + lane) * TP_PS);
+          const uint32_t lb = smem_u32(&xfull[b]);
+#pragma unroll
+          for (uint32_t r = 0; r < TP_S; ++r) {
+            st_async_v4(map_rank(lx, r), lo, map_rank(lb, r));
+            st_async_v4(map_rank(lx + 16, r), hi, map_rank(lb, r));
+          }
+        }
+        __syncwarp();
+      }
+      // red is rewritten only after every sender has read it
+      asm volatile(
+          "{\n .reg .pred p, q;\n setp.ne.u32 q, %1, 0;\n bar.red.and.pred p, 3, %2, q;\n selp.u32 %0, 1, 0, p;\n}\n"
+          : "=r"(go)
+          : "r"((uint32_t)sent), "n"(32 * TP_NGW)
+          : "memory");
+      if (!go) break;
+    }
+  } else if (warp == TP_NGW + 1) {
+    // ---------------------------------------------------------------- alpha
+    long long consumed = 0;
+    bool ok = true;
+    for (long long i = 0; i < nl; ++i) {
+      consumed = i;
+      const int b = (int)(i % TP_NX);
+      if (!warp_wait(smem_u32(&xfull[b]), (uint32_t)((i / TP_NX) & 1), true)) {
+        ok = false;
+        break;
+      }
+      // lane = token: its partials from the 8 ranks, summed in rank order
+      float v[5] = {0.f, 0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+      for (int r = 0; r < TP_S; ++r) {
+        const float* x = xbuf + (((size_t)b * TP_S + r) * TP_T + lane) * TP_PS;
+        const float4 lo = *reinterpret_cast<const float4*>(x);
+        v[0] += lo.x;
+        v[1] += lo.y;
+        v[2] += lo.z;
+        v[3] += lo.w;
+        v[4] += x[4];
+      }
+      __syncwarp();
+      // buffer b is read: arm it for tile i + NX (no rank sends that tile
+      // before this warp has read tile i + 2) and give the credit
+      if (lane == 0 && i + TP_NX < nl) mbar_arrive_expect_tx(smem_u32(&xfull[b]), TP_XBYTES);
+      arrive(&xdone[b]);
+      const int ab = (int)(i % TP_NAB);
+      if (i >= TP_NAB && !warp_wait(smem_u32(&alpha_free[ab]), (uint32_t)(((i / TP_NAB) - 1) & 1), false)) {
+        ok = false;
+        break;
+      }
+      const float r = rsqrtf(v[M] / (float)(M * d) + a.rms_eps);
+      float al[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+      for (int j = 0; j < M; ++j) al[j] = 1.0f / (1.0f + expf(-(a.gate_scale * r * v[j] + bias_s[j]))) + a.gate_offset;
+      *reinterpret_cast<float4*>(alpha_s + ((size_t)ab * TP_T + lane) * 4) = make_float4(al[0], al[1], al[2], al[3]);
+      const long long t = ((long long)cid + i * ncl) * TP_T + lane;
+      if (a.alpha_out && rank == 0 && t < N)
+#pragma unroll
+        for (int j = 0; j < M; ++j) a.alpha_out[t * M + j] = al[j];
+      __syncwarp();
+      arrive(&alpha_ready[ab]);
+    }
+    if (!ok && lane == 0) {
+      // abort: let the partials other ranks may still send land before the
+      // cluster exits (one shared time limit for all of them)
+      const unsigned long long tb = globaltimer_ns();
+      for (long long j = consumed; j < nl && j < consumed + TP_NX; ++j) {
+        const uint32_t bar = smem_u32(&xfull[j % TP_NX]), par = (uint32_t)((j / TP_NX) & 1);
+        while (!mbar_try_wait_cluster(bar, par) && globaltimer_ns() - tb < kWaitLimitNs) {
+        }
+      }
+    }
+  } else {
+    // ------------------------------------------------------- weighted warps
+    const int ww = warp - TP_NGW - 2;
+    const int vpt = ec / 8;            // 16-byte outputs per token in the slice
+    const int nitems = TP_T * vpt;
+    const __nv_bfloat16* H = reinterpret_cast<const __nv_bfloat16*>(a.H);
+    __nv_bfloat16* y = reinterpret_cast<__nv_bfloat16*>(a.y);
+    for (long long i = 0; i < nl; ++i) {
+      const int ab = (int)(i % TP_NAB);
+      if (!warp_wait(smem_u32(&alpha_ready[ab]), (uint32_t)((i / TP_NAB) & 1), false)) break;
+      const long long t0 = ((long long)cid + i * ncl) * TP_T;
+      const float* al_s = alpha_s + (size_t)ab * TP_T * 4;
+      for (int w0 = ww * 32 + lane; w0 < nitems; w0 += TP_NWW * 32 * TP_U) {
+        uint4 h[TP_U][M];
+        int tk[TP_U], col[TP_U];
+#pragma unroll
+        for (int r = 0; r < TP_U; ++r) {  // every load of the round before any arithmetic
+          const int w = w0 + r * TP_NWW * 32;
+          tk[r] = w / vpt;
+          col[r] = (int)rank * ec + (w - tk[r] * vpt) * 8;
+          const bool live = w < nitems && t0 + tk[r] < N;
+          if (!live) tk[r] = -1;
+#pragma unroll
+          for (int p = 0; p < M; ++p)
+            h[r][p] = live ? ld_stream16(H + ((t0 + tk[r]) * M + p) * d + col[r]) : make_uint4(0, 0, 0, 0);
+        }
+#pragma unroll
+        for (int r = 0; r < TP_U; ++r) {
+          if (tk[r] < 0) continue;
+          float out[8];
+#pragma unroll
+          for (int e = 0; e < 8; ++e) out[e] = 0.f;
+#pragma unroll
+          for (int p = 0; p < M; ++p) {
+            float x[8];
+            V16<__nv_bfloat16>::unpack(h[r][p], x);
+            const float al = al_s[tk[r] * 4 + p];
+#pragma unroll
+            for (int e = 0; e < 8; ++e) out[e] = fmaf(al, x[e], out[e]);
+          }
+          *reinterpret_cast<uint4*>(y + (t0 + tk[r]) * d + col[r]) = V16<__nv_bfloat16>::pack(out);
+        }
+      }
+      __syncwarp();  // alpha_s[ab] is free once every lane is past it
+      arrive(&alpha_free[ab]);
+    }
+  }
+  __syncthreads();
+  cluster_sync_all();  // no rank still writes into this CTA's shared memory
+}
+
+template <int M>
+cudaError_t launch_tile_m(const ReduceArgs& a, const TileGeo& geo, size_t smem, const TileMaps* maps,
+                          cudaStream_t s) {
+  auto k = gated_reduce_tile_kernel<M>;
+  static size_t cached_smem = 0;
+  static int cached_clusters = 0;
+  cudaError_t e;
+  int max_clusters = cached_smem == smem ? cached_clusters : 0;
+  if (!max_clusters) {
+    if ((e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem)) != cudaSuccess)
+      return e;
+    cudaLaunchConfig_t cfg = {};
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = TP_S;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    cfg.gridDim = dim3(TP_S);
+    cfg.blockDim = dim3(TP_THR);
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = s;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    if ((e = cudaOccupancyMaxActiveClusters(&max_clusters, k, &cfg)) != cudaSuccess) return e;
+    if (max_clusters < 1) return cudaErrorInvalidConfiguration;
+    cached_smem = smem;
+    cached_clusters = max_clusters;
+  }
+  const long long ncl = std::min<long long>(max_clusters, geo.ntiles);
+  return launch_kernel(k, dim3((unsigned)(ncl * TP_S)), dim3(TP_THR), smem, s, (unsigned)TP_S, a, *maps, geo);
+}
+
+bool tile_geometry(const ReduceArgs& a, int dtype, TileGeo* geo, size_t* smem) {
+  if (dtype != HDF_BF16 || a.alpha_override || a.path_norm_w) return false;
+  if (a.n_tokens <= 0 || a.n_tokens > (1ll << 31) - 64) return false;  // TMA coordinates are 32-bit
+  if (!(a.m == 1 || a.m == 2 || a.m == 4) || a.d % (TP_S * 64)) return false;
+  geo->ec = a.d / TP_S;
+  geo->nkb = geo->ec / 64;
+  geo->ngrp = (geo->nkb + TP_C - 1) / TP_C;
+  geo->tail = geo->nkb - (geo->ngrp - 1) * TP_C;
+  geo->wrow = a.m * geo->ec + 8;  // + 16 bytes: the gate rows of one B fragment sit in distinct banks
+  geo->ntiles = (a.n_tokens + TP_T - 1) / TP_T;
+  *smem = 1024 + (size_t)TP_NST * TP_SB + (size_t)TP_XBYTES * TP_NX + (size_t)2 * TP_T * TP_PS * 4 +
+          (size_t)TP_NAB * TP_T * 16 + (size_t)a.m * geo->wrow * 2;
+  return *smem <= 227 * 1024;
+}
+
+}  // namespace
+
+bool reduce_tile_boxes(const ReduceArgs& a, int dtype, unsigned box[3], unsigned tail_box[3]) {
+  TileGeo geo;
+  size_t smem;
+  if (!tile_geometry(a, dtype, &geo, &smem)) return false;
+  box[0] = tail_box[0] = 64;
+  box[1] = tail_box[1] = TP_T;
+  box[2] = (unsigned)std::min(TP_C, geo.nkb);
+  tail_box[2] = (unsigned)geo.tail;
+  return true;
+}
+
+cudaError_t launch_gated_reduce_tile(const ReduceArgs& a, const CUtensorMap* maps2, cudaStream_t s) {
+  TileGeo geo;
+  size_t smem;
+  if (!tile_geometry(a, HDF_BF16, &geo, &smem)) return cudaErrorInvalidValue;
+  TileMaps maps;
+  maps.main = maps2[0];
+  maps.tail = maps2[1];
+  switch (a.m) {
+    case 1: return launch_tile_m<1>(a, geo, smem, &maps, s);
+    case 2: return launch_tile_m<2>(a, geo, smem, &maps, s);
+    case 4: return launch_tile_m<4>(a, geo, smem, &maps, s);
+    default: return cudaErrorInvalidValue;
+  }
+}
+
 }  // namespace hdf

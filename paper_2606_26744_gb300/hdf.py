@@ -142,7 +142,7 @@ def device_status(reset: bool = True) -> int:
 
 
 # ----------------------------------------------------------------- reducer
-REDUCE_PATHS = {"auto": 0, "general": 1, "cluster": 2}
+REDUCE_PATHS = {"auto": 0, "general": 1, "cluster": 2, "tile": 3}
 
 
 def hdf_set_reduce_path(path: str) -> None:

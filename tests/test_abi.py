@@ -52,7 +52,8 @@ def test_reduce_host_validation(lib):
 
 
 def test_reduce_path_switch(lib):
-    assert lib.hdf_set_reduce_path(3) == 1            # HDF_ERR_INVALID_ARG
+    assert lib.hdf_set_reduce_path(3) == 0            # HDF_REDUCE_TILE
+    assert lib.hdf_set_reduce_path(4) == 1            # HDF_ERR_INVALID_ARG
     for path in (1, 2, 0):                            # general, cluster, auto (left at the default)
         assert lib.hdf_set_reduce_path(path) == 0
 

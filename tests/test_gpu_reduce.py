@@ -11,10 +11,11 @@ from _util import TOL_BF16, TOL_F32_REDUCE, exact_fraction, rowwise_rel, to64
 pytestmark = pytest.mark.gpu
 
 
-@pytest.fixture(params=["general", "cluster"])
+@pytest.fixture(params=["general", "cluster", "tile"])
 def reduce_path(request):
-    """Runs a test on each kernel of the reducer (the cluster kernel takes the
-    bf16 shapes it supports; the others fall back to the general kernel)."""
+    """Runs a test on each kernel of the reducer (the cluster and tile kernels
+    take the bf16 shapes they support; the others fall back to the general
+    kernel)."""
     hdf.hdf_set_reduce_path(request.param)
     yield request.param
     hdf.hdf_set_reduce_path("auto")
@@ -42,6 +43,9 @@ def _run(inp, **kw):
     (4099, 4, 2048, "bf16", 0.1),   # many batches per cluster: ring and exchange buffers wrap
     (50, 1, 1024, "bf16", 0.1),
     (777, 2, 7168, "bf16", 0.1),
+    (32, 4, 512, "bf16", 0.1),      # one whole 32-token tile, one 64-element block per CTA
+    (33, 1, 512, "bf16", 0.1),      # a tile of one token after a full one
+    (1000, 4, 7168, "bf16", 0.1),   # 56 k-blocks per CTA: the stage ring wraps in both passes
 ])
 def test_reduce_parity(N, m, d, dtype, std, reduce_path):
     inp = W.make_reduce_inputs(N, m, d, dtype, std, seed=N * 131 + d)
