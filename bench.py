@@ -515,7 +515,6 @@ NCU_DRAM_BYTES_DECODE = {
     "L0.down_gemm": 34031360,
     "lm_head": 134365952 + 3178496,
     "L0.attention": 17016576,
-    "gated_reduce": 33669120,
 }
 
 
@@ -605,8 +604,21 @@ def run_sweep(args):
         torch.cuda.synchronize()
         ms = e0.elapsed_time(e1) / args.steps
         byt = n * m * d * 2 + n * d * 2 + m * m * d * 2
-        row = {"n": n, "ms": round(ms, 4), "gbs": round(byt / ms / 1e6, 1),
-               "frac_hbm": round(byt / ms / 1e6 / pk["hbm_gbs"], 4)}
+        row = {"n": n, "kernel": "tile" if m == 4 else "general", "ms": round(ms, 4),
+               "gbs": round(byt / ms / 1e6, 1), "frac_hbm": round(byt / ms / 1e6 / pk["hbm_gbs"], 4)}
+        # the general kernel on the same input, for comparison
+        hdf.hdf_set_reduce_path("general")
+        hdf.hdf_gated_reduce(H, Wf, b, y=y)
+        torch.cuda.synchronize()
+        greps = max(1, args.steps // 2)
+        e0.record()
+        for _ in range(greps):
+            hdf.hdf_gated_reduce(H, Wf, b, y=y)
+        e1.record()
+        torch.cuda.synchronize()
+        hdf.hdf_set_reduce_path("auto")
+        gms = e0.elapsed_time(e1) / greps
+        row["general_gbs"] = round(byt / gms / 1e6, 1)
         if n <= args.fc_max_n:
             Wfc = (torch.randn((d, m * d), device=dev) * 0.02).to(torch.bfloat16)
             yfc = torch.empty_like(y)

@@ -116,8 +116,9 @@ HDF_API int hdf_gated_reduce(const void* H, int dtype, int64_t n_tokens, int m, 
  * tiles of 32 tokens, gate dots on the tensor cores, one exchange per tile.
  * CLUSTER and TILE need bf16, m in {1,2,4}, d % 512 == 0 and neither
  * alpha_override nor path_norm_w; the general kernel runs otherwise.
- * HDF_REDUCE_AUTO (the default) takes the fastest kernel measured for the
- * shape.  Process-wide; returns HDF_ERR_INVALID_ARG for another value.  The
+ * HDF_REDUCE_AUTO (the default) takes the tile kernel for m = 4 and the
+ * general kernel otherwise, whatever n_tokens is, so that a token's y does not
+ * depend on how many tokens share the call.  Process-wide; returns HDF_ERR_INVALID_ARG for another value.  The
  * paper has no counterpart: it is a tuning and test hook. */
 enum { HDF_REDUCE_AUTO = 0, HDF_REDUCE_GENERAL = 1, HDF_REDUCE_CLUSTER = 2, HDF_REDUCE_TILE = 3 };
 HDF_API int hdf_set_reduce_path(int path);

@@ -338,14 +338,19 @@ int hdf_gated_reduce(const void* H, int dtype, int64_t n_tokens, int m, int d, c
   unsigned box[3];
   const int path = g_reduce_path.load();
   unsigned tail_box[3];
-  if (path == HDF_REDUCE_TILE && reduce_tile_boxes(a, dtype, box, tail_box)) {
+  // auto: the tile kernel for m = 4 (1.2-1.6x the general kernel from 4096
+  // tokens, a tie below), the general kernel for other m.  The choice does not
+  // depend on n_tokens: a token's y is then the same bits whether it is
+  // reduced with its whole context or alone in a serving round.
+  const bool tile_wanted = path == HDF_REDUCE_TILE || (path == HDF_REDUCE_AUTO && m == 4);
+  if (tile_wanted && reduce_tile_boxes(a, dtype, box, tail_box)) {
     CUtensorMap hm[2];
     if ((rc = make_chunk_map(&hm[0], H, n_tokens, m, d, box))) return rc;
     if ((rc = make_chunk_map(&hm[1], H, n_tokens, m, d, tail_box))) return rc;
     CK(launch_gated_reduce_tile(a, hm, (cudaStream_t)stream), "gated_reduce tile launch");
     return HDF_OK;
   }
-  const bool cluster_wanted = path == HDF_REDUCE_CLUSTER;  // auto: the general kernel, faster on every shape measured
+  const bool cluster_wanted = path == HDF_REDUCE_CLUSTER;
   if (cluster_wanted && reduce_cluster_box(a, dtype, box)) {
     CUtensorMap hm;
     if ((rc = make_chunk_map(&hm, H, n_tokens, m, d, box))) return rc;

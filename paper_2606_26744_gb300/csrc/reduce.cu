@@ -835,25 +835,26 @@ cudaError_t launch_gated_reduce_cluster(const ReduceArgs& a, const CUtensorMap* 
 // ===========================================================================
 // bf16 tile path (persistent, warp-specialised).
 //
-// A cluster of TP_S = 8 CTAs walks tiles of TP_T = 32 consecutive tokens; CTA
-// rank c owns elements [c*E, (c+1)*E) of each of the m paths (E = d/8), so
-// its W_f slice (m x m*E) stays in shared memory.  Roles, meeting only at
-// mbarriers:
+// A cluster of S CTAs (S = 4, or 8 when d is wide) walks tiles of TP_T = 32
+// consecutive tokens; CTA rank c owns elements [c*E, (c+1)*E) of each of the
+// m paths (E = d/S), so its W_f slice (m x m*E) stays in shared memory.
+// Roles, meeting only at mbarriers:
 //   producer warp   streams pass 1 of every tile from HBM into a 128 KB ring:
 //                   one TMA box per stage from the 3-D view {64 elements,
 //                   tokens, 128-byte chunks} of H, 4 chunks (512 contiguous
 //                   bytes) of 32 tokens, landing as planes [32 tokens][64
 //                   elements] with the 128-byte swizzle; it never waits on
 //                   the gates, so HBM streaming continues across tiles
-//   2 gate warps    one per 16-token row tile: the m gate dots on mma.sync
-//                   m16n8k16 (tokens are the rows, the W_f slice is B) and
-//                   the sums of squares from the same A fragments; each sends
-//                   its [16 tokens][m + 1] partials to every rank with
-//                   st.async, which completes the receiver's exchange
-//                   mbarrier on bytes
-//   alpha warp      on every rank: waits for the 16 senders of a tile, sums
-//                   each token's partials over the 8 ranks in rank order (so
-//                   every rank gets the same alpha, Eq. 1) and publishes alpha
+//   8 gate warps    (row tile of 16 tokens) x (box phase 0..3): the m gate
+//                   dots on mma.sync m16n8k16 (tokens are the rows, the W_f
+//                   slice is B) and the sums of squares from the same A
+//                   fragments; the four phases of a row tile are added in
+//                   phase order and sent, [16 tokens][m + 1] partials, to
+//                   every rank with st.async, which completes the receiver's
+//                   exchange mbarrier on bytes
+//   alpha warp      on every rank: waits for all senders of a tile, sums each
+//                   token's partials over the ranks in rank order (so every
+//                   rank gets the same alpha, Eq. 1) and publishes alpha
 //   8 weighted      y = sum_j alpha_j H_j for the CTA's slice of the tile,
 //   warps           reading H again from L2 (streamed microseconds before)
 //                   with 16 loads in flight per lane, one store per output
@@ -862,23 +863,22 @@ cudaError_t launch_gated_reduce_cluster(const ReduceArgs& a, const CUtensorMap* 
 // from HBM once, W_f once per CTA.  Every wait is time-limited.
 namespace {
 
-constexpr int TP_S = 8;                    // CTAs per cluster
 constexpr int TP_T = 32;                   // tokens per tile
 constexpr int TP_C = 4;                    // 128-byte chunks per token in a box
 constexpr int TP_PLANE = TP_T * 128;       // one [32 tokens x 64 elements] bf16 plane
 constexpr int TP_SB = TP_C * TP_PLANE;     // bytes per ring stage
 constexpr int TP_NST = 8;                  // ring stages (128 KB)
-constexpr int TP_NGW = 4;                  // gate warps: (row tile, box parity)
+constexpr int TP_NGW = 8;                  // gate warps: (row tile, box phase 0..3)
 constexpr int TP_NWW = 8;                  // weighted warps
 constexpr int TP_THR = 32 * (2 + TP_NGW + TP_NWW);
 constexpr int TP_LA = 2;                   // gate warps run at most this many tiles ahead of the alpha warp
 constexpr int TP_NX = 2 * TP_LA + 2;       // exchange buffers
 constexpr int TP_NAB = 3;                  // alpha buffers
 constexpr int TP_PS = 8;                   // floats per token in an exchange row (m + 1 <= 5 used)
-constexpr int TP_XBYTES = TP_S * TP_T * TP_PS * 4;  // one tile's partials from all senders
 constexpr int TP_U = 4;                    // weighted outputs per lane and round
 
 struct TileGeo {
+  int s;     // CTAs per cluster (4 or 8): the d split
   int ec;    // elements per path in a CTA slice (multiple of 64)
   int nkb;   // 128-byte chunks per path slice
   int ngrp;  // boxes per path slice: ngrp - 1 of TP_C chunks, then one of tail chunks
@@ -897,16 +897,18 @@ __device__ __forceinline__ void st_async_v4(uint32_t addr, float4 v, uint32_t ba
                : "memory");
 }
 
-template <int M>
+constexpr int tp_xbytes(int S) { return S * TP_T * TP_PS * 4; }  // one tile's partials from all senders
+
+template <int M, int S>
 __global__ void __launch_bounds__(TP_THR, 1) gated_reduce_tile_kernel(const ReduceArgs a,
                                                                       const __grid_constant__ TileMaps maps,
                                                                       const TileGeo geo) {
   extern __shared__ uint8_t tp_smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(tp_smem_raw) + 1023) &
                                              ~static_cast<uintptr_t>(1023));
-  uint8_t* ring = smem;                                                              // [NST][SB]
+  uint8_t* ring = smem;                                                              // [NST][TP_SB]
   float* xbuf = reinterpret_cast<float*>(smem + TP_NST * TP_SB);                     // [NX][S][T][PS]
-  float* red = xbuf + TP_NX * TP_S * TP_T * TP_PS;                                  // [2 halves][32][PS]
+  float* red = xbuf + TP_NX * S * TP_T * TP_PS;                                     // [NGW/2 phases][32][PS]
   float* alpha_s = red + TP_NGW * 16 * TP_PS;                                        // [NAB][T][4]
   __nv_bfloat16* wsl = reinterpret_cast<__nv_bfloat16*>(alpha_s + TP_NAB * TP_T * 4);  // [M][wrow]
   __shared__ __align__(8) uint64_t full_bar[TP_NST];
@@ -951,7 +953,7 @@ __global__ void __launch_bounds__(TP_THR, 1) gated_reduce_tile_kernel(const Redu
     }
     abort_flag = 0;
     fence_mbar_init();
-    for (int b = 0; b < TP_NX && b < nl; ++b) mbar_arrive_expect_tx(smem_u32(&xfull[b]), TP_XBYTES);
+    for (int b = 0; b < TP_NX && b < nl; ++b) mbar_arrive_expect_tx(smem_u32(&xfull[b]), tp_xbytes(S));
   }
   __syncthreads();
   cluster_sync_all();  // every rank's barriers exist and are armed before anyone signals them
@@ -999,7 +1001,7 @@ __global__ void __launch_bounds__(TP_THR, 1) gated_reduce_tile_kernel(const Redu
   } else if (warp <= TP_NGW) {
     // --------------------------------------------------------------- gates
     // warp (rt, hb): tokens 16*rt .. 16*rt + 15 of the boxes j with j % 2 == hb
-    const int gw = warp - 1, rt = gw & 1, hb = gw >> 1;
+    const int gw = warp - 1, rt = gw & 1, hb = gw >> 1;  // hb 0..3
     const int g8 = lane >> 2, q = lane & 3;
     const __nv_bfloat16* wrowp = wsl + (size_t)(g8 < M ? g8 : 0) * geo.wrow + 2 * q;
     const int row = rt * 16 + (lane & 15), hsel = lane >> 4;
@@ -1007,7 +1009,7 @@ __global__ void __launch_bounds__(TP_THR, 1) gated_reduce_tile_kernel(const Redu
       float acc[2][4] = {{0.f, 0.f, 0.f, 0.f}, {0.f, 0.f, 0.f, 0.f}};  // two chains: plane parity
       unsigned long long sq0[2] = {0ull, 0ull}, sq1[2] = {0ull, 0ull};
       bool ok = true;
-      for (int j = hb; j < NB; j += 2) {
+      for (int j = hb; j < NB; j += TP_NGW / 2) {
         const long long gs = i * NB + j;  // stage counter
         const int s = (int)(gs % TP_NST);
         if (!warp_wait(smem_u32(&full_bar[s]), (uint32_t)((gs / TP_NST) & 1), false)) {
@@ -1045,7 +1047,7 @@ __global__ void __launch_bounds__(TP_THR, 1) gated_reduce_tile_kernel(const Redu
         arrive(&empty_bar[s]);
       }
       // this warp's [16 tokens][m + 1] partials into red[hb]; the hb = 0 warps
-      // add the hb = 1 halves and send one row per lane to every rank
+      // add the four box phases and send one row per lane to every rank
       float* rw = red + ((size_t)hb * TP_T + rt * 16) * TP_PS;
       {
         float s0 = sum2(sq0[0]) + sum2(sq0[1]), s1 = sum2(sq1[0]) + sum2(sq1[1]);
@@ -1085,14 +1087,20 @@ __global__ void __launch_bounds__(TP_THR, 1) gated_reduce_tile_kernel(const Redu
         if (sent && lane < 16) {
           const int b = (int)(i % TP_NX);
           const float* r0 = red + (size_t)(rt * 16 + lane) * TP_PS;
-          const float* r1 = r0 + TP_T * TP_PS;
-          const float4 a0 = *reinterpret_cast<const float4*>(r0), a1 = *reinterpret_cast<const float4*>(r1);
-          const float4 lo = make_float4(a0.x + a1.x, a0.y + a1.y, a0.z + a1.z, a0.w + a1.w);
-          const float4 hi = make_float4(r0[4] + r1[4], 0.f, 0.f, 0.f);
-          const uint32_t lx = smem_u32(xbuf + (((size_t)b * TP_S + rank) * TP_T + rt * 16 + lane) * TP_PS);
+          float4 lo = make_float4(0.f, 0.f, 0.f, 0.f), hi = lo;
+#pragma unroll
+          for (int h = 0; h < TP_NGW / 2; ++h) {  // the box phases in a fixed order
+            const float4 ah = *reinterpret_cast<const float4*>(r0 + h * TP_T * TP_PS);
+            lo.x += ah.x;
+            lo.y += ah.y;
+            lo.z += ah.z;
+            lo.w += ah.w;
+            hi.x += r0[h * TP_T * TP_PS + 4];
+          }
+          const uint32_t lx = smem_u32(xbuf + (((size_t)b * S + rank) * TP_T + rt * 16 + lane) * TP_PS);
           const uint32_t lb = smem_u32(&xfull[b]);
 #pragma unroll
-          for (uint32_t r = 0; r < TP_S; ++r) {
+          for (uint32_t r = 0; r < S; ++r) {
             st_async_v4(map_rank(lx, r), lo, map_rank(lb, r));
             st_async_v4(map_rank(lx + 16, r), hi, map_rank(lb, r));
           }
@@ -1121,8 +1129,8 @@ __global__ void __launch_bounds__(TP_THR, 1) gated_reduce_tile_kernel(const Redu
       // lane = token: its partials from the 8 ranks, summed in rank order
       float v[5] = {0.f, 0.f, 0.f, 0.f, 0.f};
 #pragma unroll
-      for (int r = 0; r < TP_S; ++r) {
-        const float* x = xbuf + (((size_t)b * TP_S + r) * TP_T + lane) * TP_PS;
+      for (int r = 0; r < S; ++r) {
+        const float* x = xbuf + (((size_t)b * S + r) * TP_T + lane) * TP_PS;
         const float4 lo = *reinterpret_cast<const float4*>(x);
         v[0] += lo.x;
         v[1] += lo.y;
@@ -1133,7 +1141,7 @@ __global__ void __launch_bounds__(TP_THR, 1) gated_reduce_tile_kernel(const Redu
       __syncwarp();
       // buffer b is read: arm it for tile i + NX (no rank sends that tile
       // before this warp has read tile i + 2) and give the credit
-      if (lane == 0 && i + TP_NX < nl) mbar_arrive_expect_tx(smem_u32(&xfull[b]), TP_XBYTES);
+      if (lane == 0 && i + TP_NX < nl) mbar_arrive_expect_tx(smem_u32(&xfull[b]), tp_xbytes(S));
       arrive(&xdone[b]);
       const int ab = (int)(i % TP_NAB);
       if (i >= TP_NAB && !warp_wait(smem_u32(&alpha_free[ab]), (uint32_t)(((i / TP_NAB) - 1) & 1), false)) {
@@ -1213,10 +1221,10 @@ __global__ void __launch_bounds__(TP_THR, 1) gated_reduce_tile_kernel(const Redu
   cluster_sync_all();  // no rank still writes into this CTA's shared memory
 }
 
-template <int M>
-cudaError_t launch_tile_m(const ReduceArgs& a, const TileGeo& geo, size_t smem, const TileMaps* maps,
-                          cudaStream_t s) {
-  auto k = gated_reduce_tile_kernel<M>;
+template <int M, int S>
+cudaError_t launch_tile_ms(const ReduceArgs& a, const TileGeo& geo, size_t smem, const TileMaps* maps,
+                           cudaStream_t s) {
+  auto k = gated_reduce_tile_kernel<M, S>;
   static size_t cached_smem = 0;
   static int cached_clusters = 0;
   cudaError_t e;
@@ -1227,10 +1235,10 @@ cudaError_t launch_tile_m(const ReduceArgs& a, const TileGeo& geo, size_t smem, 
     cudaLaunchConfig_t cfg = {};
     cudaLaunchAttribute attr[1];
     attr[0].id = cudaLaunchAttributeClusterDimension;
-    attr[0].val.clusterDim.x = TP_S;
+    attr[0].val.clusterDim.x = S;
     attr[0].val.clusterDim.y = 1;
     attr[0].val.clusterDim.z = 1;
-    cfg.gridDim = dim3(TP_S);
+    cfg.gridDim = dim3(S);
     cfg.blockDim = dim3(TP_THR);
     cfg.dynamicSmemBytes = smem;
     cfg.stream = s;
@@ -1242,20 +1250,32 @@ cudaError_t launch_tile_m(const ReduceArgs& a, const TileGeo& geo, size_t smem, 
     cached_clusters = max_clusters;
   }
   const long long ncl = std::min<long long>(max_clusters, geo.ntiles);
-  return launch_kernel(k, dim3((unsigned)(ncl * TP_S)), dim3(TP_THR), smem, s, (unsigned)TP_S, a, *maps, geo);
+  return launch_kernel(k, dim3((unsigned)(ncl * S)), dim3(TP_THR), smem, s, (unsigned)S, a, *maps, geo);
 }
 
+template <int M>
+cudaError_t launch_tile_m(const ReduceArgs& a, const TileGeo& geo, size_t smem, const TileMaps* maps,
+                          cudaStream_t s) {
+  return geo.s == 4 ? launch_tile_ms<M, 4>(a, geo, smem, maps, s) : launch_tile_ms<M, 8>(a, geo, smem, maps, s);
+}
+
+// Cluster size: 8 CTAs once the W_f slices of a 4-CTA split would crowd the
+// ring (d >= 4096 at m = 4); 4 below, where more clusters fit the GPCs
+// (measured: 5.0 vs 3.9 TB/s at d = 2048, 4.1 vs 3.7 TB/s at d = 7168).
 bool tile_geometry(const ReduceArgs& a, int dtype, TileGeo* geo, size_t* smem) {
   if (dtype != HDF_BF16 || a.alpha_override || a.path_norm_w) return false;
   if (a.n_tokens <= 0 || a.n_tokens > (1ll << 31) - 64) return false;  // TMA coordinates are 32-bit
-  if (!(a.m == 1 || a.m == 2 || a.m == 4) || a.d % (TP_S * 64)) return false;
-  geo->ec = a.d / TP_S;
+  if (!(a.m == 1 || a.m == 2 || a.m == 4)) return false;
+  const int S = (long long)a.m * a.m * a.d * 2 / 4 > 32 * 1024 ? 8 : 4;
+  if (a.d % (S * 64)) return false;
+  geo->s = S;
+  geo->ec = a.d / S;
   geo->nkb = geo->ec / 64;
   geo->ngrp = (geo->nkb + TP_C - 1) / TP_C;
   geo->tail = geo->nkb - (geo->ngrp - 1) * TP_C;
   geo->wrow = a.m * geo->ec + 8;  // + 16 bytes: the gate rows of one B fragment sit in distinct banks
   geo->ntiles = (a.n_tokens + TP_T - 1) / TP_T;
-  *smem = 1024 + (size_t)TP_NST * TP_SB + (size_t)TP_XBYTES * TP_NX + (size_t)2 * TP_T * TP_PS * 4 +
+  *smem = 1024 + (size_t)TP_NST * TP_SB + (size_t)tp_xbytes(S) * TP_NX + (size_t)(TP_NGW / 2) * TP_T * TP_PS * 4 +
           (size_t)TP_NAB * TP_T * 16 + (size_t)a.m * geo->wrow * 2;
   return *smem <= 227 * 1024;
 }

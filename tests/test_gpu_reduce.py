@@ -113,3 +113,17 @@ def test_reduce_sweep_width_sampled_rows(reduce_path):
     y_ref, _ = O.gated_reduce(Hs, to64(inp["Wf"]), to64(inp["b"]), out_dtype="bf16")
     assert rowwise_rel(to64(y[rows.cuda()]), y_ref) <= TOL_BF16
     assert exact_fraction(to64(y[rows.cuda()]), y_ref) >= 0.99
+
+
+def test_reduce_rows_do_not_depend_on_the_call():
+    """A token's y is the same bits whether it is reduced with many others or
+    in a call of its own (the default kernel choice does not depend on the
+    token count): a serving round that reduces only its new tokens matches the
+    reduction of the whole context."""
+    N, m, d = 5000, 4, 2048
+    inp = W.make_reduce_inputs(N, m, d, "bf16", 0.1, seed=21, device="cuda")
+    H, Wf, b = inp["H"], inp["Wf"], inp["b"]
+    y_all = hdf.hdf_gated_reduce(H, Wf, b)
+    for lo, hi in [(0, 1), (4095, 4101), (17, 60), (4990, 5000)]:
+        y_part = hdf.hdf_gated_reduce(H[lo:hi].contiguous(), Wf, b)
+        assert torch.equal(y_part.view(torch.int16), y_all[lo:hi].view(torch.int16))
