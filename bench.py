@@ -515,7 +515,14 @@ NCU_DRAM_BYTES_DECODE = {
     "L0.down_gemm": 34031360,
     "lm_head": 134365952 + 3178496,
     "L0.attention": 17016576,
+    "gated_reduce": 33675008,
 }
+
+
+# DRAM bytes (read + write) per token of the tile reducer at m = 4, d = 7168,
+# from the ncu capture summarised in profiles/gated_reduce_sweep.md (8192
+# tokens; traffic grows with the tokens)
+NCU_DRAM_BYTES_PER_TOKEN_SWEEP = (470288896 + 87983616) / 8192
 
 
 def roofline_of(cfg, res, pk):
@@ -645,7 +652,9 @@ def run_sweep(args):
             "config": {"workload": "reducer sweep", "m": m, "d": d, "n": big["n"],
                        "l2": "inputs larger than L2 for N >= 4096"},
             "roofline": {"kernel": "gated_reduce", "bound": "hbm", "achieved": big["gbs"], "peak": pk["hbm_gbs"],
-                         "unit": "GB/s", "frac": big["frac_hbm"], "traffic": None},
+                         "unit": "GB/s", "frac": big["frac_hbm"],
+                         "traffic": int(NCU_DRAM_BYTES_PER_TOKEN_SWEEP * big["n"]) if m == 4 and d == 7168 else None,
+                         "traffic_note": "ncu capture at 8192 tokens scaled to the launch by tokens"},
             "sweep": rows}
     print(json.dumps(line), flush=True)
     return 0
