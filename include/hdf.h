@@ -115,7 +115,8 @@ HDF_API int hdf_gated_reduce(const void* H, int dtype, int64_t n_tokens, int m, 
  * distributed shared memory.  HDF_REDUCE_TILE: 8-CTA clusters split d over
  * tiles of 32 tokens, gate dots on the tensor cores, one exchange per tile.
  * CLUSTER and TILE need bf16, m in {1,2,4}, d % 512 == 0 and neither
- * alpha_override nor path_norm_w; the general kernel runs otherwise.
+ * alpha_override nor path_norm_w (TILE also a whole number of its 4 box
+ * phases per tile, always so for m = 4); the general kernel runs otherwise.
  * HDF_REDUCE_AUTO (the default) takes the tile kernel for m = 4 and the
  * general kernel otherwise, whatever n_tokens is, so that a token's y does not
  * depend on how many tokens share the call.  Process-wide; returns HDF_ERR_INVALID_ARG for another value.  The

@@ -26,6 +26,11 @@ namespace {
 constexpr int KT = 64;       // keys per tile
 constexpr int NSTAGE = 4;
 constexpr int NCW = 4;       // consumer warps
+// Tile t goes to stage t % NSTAGE and to consumer warp t % NCW: with the two
+// equal, each warp waits only on its own stage, one fill at a time.  A warp
+// that could wait on a stage two fills ahead would pass the parity wait on
+// the older fill (mbarrier parity tells adjacent phases apart only).
+static_assert(NSTAGE == NCW, "stage / consumer-warp affinity");
 
 __device__ __forceinline__ void ldsm_x4(uint32_t addr, uint32_t& r0, uint32_t& r1, uint32_t& r2,
                                         uint32_t& r3) {

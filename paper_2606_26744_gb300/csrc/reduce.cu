@@ -869,6 +869,13 @@ constexpr int TP_PLANE = TP_T * 128;       // one [32 tokens x 64 elements] bf16
 constexpr int TP_SB = TP_C * TP_PLANE;     // bytes per ring stage
 constexpr int TP_NST = 8;                  // ring stages (128 KB)
 constexpr int TP_NGW = 8;                  // gate warps: (row tile, box phase 0..3)
+// Box j of tile i is stage g = i*NB + j of the ring, slot g % TP_NST, and is
+// read by the two gate warps of phase j % 4.  With NB a multiple of 4 (the
+// tile geometry requires it), slot g % 8 only ever holds boxes of phase g % 4,
+// and the box a gate warp waits for comes 8 stages after one it read itself:
+// no waiter is more than one fill ahead of a slot's barrier (an mbarrier
+// parity wait tells adjacent phases apart only).
+static_assert(TP_NST == 2 * (TP_NGW / 2), "each slot serves one box phase");
 constexpr int TP_NWW = 8;                  // weighted warps
 constexpr int TP_THR = 32 * (2 + TP_NGW + TP_NWW);
 constexpr int TP_LA = 2;                   // gate warps run at most this many tiles ahead of the alpha warp
@@ -1273,6 +1280,7 @@ bool tile_geometry(const ReduceArgs& a, int dtype, TileGeo* geo, size_t* smem) {
   geo->nkb = geo->ec / 64;
   geo->ngrp = (geo->nkb + TP_C - 1) / TP_C;
   geo->tail = geo->nkb - (geo->ngrp - 1) * TP_C;
+  if ((a.m * geo->ngrp) % (TP_NGW / 2)) return false;  // boxes per tile: a multiple of the 4 phases
   geo->wrow = a.m * geo->ec + 8;  // + 16 bytes: the gate rows of one B fragment sit in distinct banks
   geo->ntiles = (a.n_tokens + TP_T - 1) / TP_T;
   *smem = 1024 + (size_t)TP_NST * TP_SB + (size_t)tp_xbytes(S) * TP_NX + (size_t)(TP_NGW / 2) * TP_T * TP_PS * 4 +
