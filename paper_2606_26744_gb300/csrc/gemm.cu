@@ -249,6 +249,62 @@ __device__ __forceinline__ void epilogue_chunk(const GemmArgs& g, int tile_m, in
       __syncthreads();
       return;
     }
+    case kEpiLmHead: {  // rows = tokens, columns = vocabulary entries
+      // Each thread owns one token and scans the tile's columns in increasing
+      // order, chunk after chunk; its running max, first argmax and sum of
+      // exp((z - max) * inv_temp) stay in a private shared-memory slot
+      // between chunks, and the last chunk writes the tile's partials.
+      float* st = reinterpret_cast<float*>(smem) + row * 4;
+      const long long t = (long long)tile_m * BM + row;
+      const long long V = g.N;
+      const int jb = tile_n * BN + c0;
+      const float it = E.inv_temp;
+      float m = -INFINITY, sum = 0.f;
+      int a = INT_MAX;
+      if (c0 > 0) {
+        m = st[0];
+        sum = st[1];
+        a = __float_as_int(st[2]);
+      }
+      if (t < g.M) {
+        if (E.logsoftmax) {
+          float* dst = E.logsoftmax + t * V + jb;
+          if (jb + 16 <= V && ((V & 3) == 0)) {
+#pragma unroll
+            for (int i = 0; i < 4; ++i)
+              reinterpret_cast<float4*>(dst)[i] =
+                  make_float4(v[4 * i] * it, v[4 * i + 1] * it, v[4 * i + 2] * it, v[4 * i + 3] * it);
+          } else {
+#pragma unroll
+            for (int k = 0; k < 16; ++k)
+              if (jb + k < V) dst[k] = v[k] * it;
+          }
+        }
+#pragma unroll
+        for (int k = 0; k < 16; ++k) {
+          if (jb + k >= V) break;
+          const float x = v[k];
+          if (x > m) {
+            sum = (m == -INFINITY ? 0.f : sum * expf((m - x) * it)) + 1.f;
+            m = x;
+            a = jb + k;
+          } else if (x != -INFINITY) {
+            sum += expf((x - m) * it);
+          }
+        }
+      }
+      if (c0 + 16 < BN) {
+        st[0] = m;
+        st[1] = sum;
+        st[2] = __int_as_float(a);
+      } else if (t < g.M) {
+        const size_t o = (size_t)tile_n * g.M + t;
+        E.part_max[o] = m;
+        E.part_arg[o] = a;
+        E.part_sum[o] = sum;
+      }
+      return;
+    }
     case kEpiLmHeadT: {  // rows = vocabulary entries, columns = tokens
       // Per (tile, token): max, first argmax and sum of exp((z - max) * inv_temp)
       // over the tile's 128 rows.  The chunk goes through shared memory token-

@@ -777,13 +777,23 @@ int hdf_ctx_append(const hdf_drafter_weights* w, const hdf_draft_shape* sh, cons
 namespace {
 struct LmLayout {
   SplitPlan p;
+  bool token_major;
+  int tiles;    // vocabulary tiles the partials come from
   int tiles_m;
   size_t pmax, parg, psum, total;
 };
+// Token-major LM head (tokens on the GEMM rows, vocabulary 256 columns per
+// tile) from this many tokens: each CTA then streams 1.5 bytes per weight
+// byte instead of 2 (the swapped tile re-reads a token tile as large as its
+// weight tile)
+constexpr int64_t kLmTokenMajorFrom = 64;
+
 LmLayout lm_layout(int64_t M, int64_t V, int dtype, int d) {
   LmLayout L;
-  L.p = plan_swap(dtype, V, M, d);
-  L.tiles_m = (int)((V + 127) / 128);
+  L.token_major = M >= kLmTokenMajorFrom;
+  L.p = L.token_major ? SplitPlan{256, 1, (int)(((M + 127) / 128) * ((V + 255) / 256))} : plan_swap(dtype, V, M, d);
+  L.tiles_m = (int)((V + 127) / 128);  // partial rows reserved: enough for either orientation
+  L.tiles = L.token_major ? (int)((V + 255) / 256) : L.tiles_m;
   size_t off = 0;
   auto take = [&](size_t b) {
     const size_t o = off;
@@ -795,6 +805,37 @@ LmLayout lm_layout(int64_t M, int64_t V, int dtype, int d) {
   L.psum = take((size_t)L.tiles_m * M * 4);
   L.total = off;
   return L;
+}
+
+// LM-head GEMM with the argmax / sum-exp epilogue, then the cross-tile reduce.
+int lm_head_launch(const LmLayout& L, const void* h, int dtype, int64_t M, int d, const void* W_lm, int64_t V,
+                   float inv_temp, int32_t* tok, float* zmax, float* logsoftmax, char* W, cudaStream_t s) {
+  GemmArgs g;
+  int rc;
+  if (L.token_major) {
+    init_gemm(g, dtype, M, V, d, L.p);
+    g.group_n = 8;  // the token tiles of one weight tile run together
+    if ((rc = make_map(&g.A.map[0], h, dtype, M, d, d, 64))) return rc;
+    if ((rc = make_map(&g.B.map[0], W_lm, dtype, V, d, d, L.p.bn))) return rc;
+    g.pre_operand = 2;  // the LM head weight
+    g.epi.kind = kEpiLmHead;
+  } else {
+    init_gemm(g, dtype, V, M, d, L.p);
+    if ((rc = make_map(&g.A.map[0], W_lm, dtype, V, d, d, 64))) return rc;
+    if ((rc = make_map(&g.B.map[0], h, dtype, M, d, d, L.p.bn))) return rc;
+    g.pre_operand = 1;  // the LM head weight
+    g.epi.kind = kEpiLmHeadT;
+  }
+  g.epi.inv_temp = inv_temp;
+  g.epi.logsoftmax = logsoftmax;
+  g.epi.part_max = reinterpret_cast<float*>(W + L.pmax);
+  g.epi.part_arg = reinterpret_cast<int*>(W + L.parg);
+  g.epi.part_sum = reinterpret_cast<float*>(W + L.psum);
+  CK(launch_gemm(g, s), "lm head gemm");
+  CK(launch_lm_reduce(g.epi.part_max, g.epi.part_arg, g.epi.part_sum, L.tiles, M, V, inv_temp, tok, zmax,
+                      logsoftmax, s),
+     "lm reduce");
+  return HDF_OK;
 }
 }  // namespace
 
@@ -818,25 +859,8 @@ int hdf_lm_head_argmax(const void* h, int dtype, int64_t M, int d, const void* W
   const LmLayout L = lm_layout(M, V, dtype, d);
   if (!ws || ws_bytes < L.total || (reinterpret_cast<uintptr_t>(ws) & 255))
     return fail(HDF_ERR_WORKSPACE, "workspace %zu bytes (need %zu, 256-byte aligned)", ws_bytes, L.total);
-  cudaStream_t s = (cudaStream_t)stream;
-  char* W = static_cast<char*>(ws);
-  GemmArgs g;
-  init_gemm(g, dtype, V, M, d, L.p);
-  int rc;
-  if ((rc = make_map(&g.A.map[0], W_lm, dtype, V, d, d, 64))) return rc;
-  if ((rc = make_map(&g.B.map[0], h, dtype, M, d, d, L.p.bn))) return rc;
-  g.pre_operand = 1;  // the LM head weight
-  g.epi.kind = kEpiLmHeadT;
-  g.epi.inv_temp = inv_temp;
-  g.epi.logsoftmax = logsoftmax;
-  g.epi.part_max = reinterpret_cast<float*>(W + L.pmax);
-  g.epi.part_arg = reinterpret_cast<int*>(W + L.parg);
-  g.epi.part_sum = reinterpret_cast<float*>(W + L.psum);
-  CK(launch_gemm(g, s), "lm head gemm");
-  CK(launch_lm_reduce(g.epi.part_max, g.epi.part_arg, g.epi.part_sum, L.tiles_m, M, V, inv_temp, tok, zmax,
-                      logsoftmax, s),
-     "lm reduce");
-  return HDF_OK;
+  return lm_head_launch(L, h, dtype, M, d, W_lm, V, inv_temp, tok, zmax, logsoftmax, static_cast<char*>(ws),
+                        (cudaStream_t)stream);
 }
 
 // ------------------------------------------------ T = 1 verification

@@ -82,6 +82,7 @@ enum EpiKind {
   kEpiResidT = 2,   // resid[col, row] += D  (fp32 residual)
   kEpiSwigluT = 3,  // pair tile: act[col, f] = silu(g) * u
   kEpiLmHeadT = 4,  // rows = vocab, cols = tokens: argmax / sum-exp partials
+  kEpiLmHead = 5,   // rows = tokens, cols = vocab: the same partials, one per (column tile, token)
 };
 
 struct Epilogue {
