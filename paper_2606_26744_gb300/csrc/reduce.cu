@@ -835,8 +835,8 @@ cudaError_t launch_gated_reduce_cluster(const ReduceArgs& a, const CUtensorMap* 
 // ===========================================================================
 // bf16 tile path (persistent, warp-specialised).
 //
-// A cluster of S CTAs (S = 4, or 8 when d is wide) walks tiles of TP_T = 32
-// consecutive tokens; CTA rank c owns elements [c*E, (c+1)*E) of each of the
+// A cluster of S CTAs (S = 4, or 8 when d is wide) walks tiles of T = 32 (or
+// 16, for wide slices) consecutive tokens; CTA rank c owns elements [c*E, (c+1)*E) of each of the
 // m paths (E = d/S), so its W_f slice (m x m*E) stays in shared memory.
 // Roles, meeting only at mbarriers:
 //   producer warp   streams pass 1 of every tile from HBM into a 128 KB ring:
@@ -863,19 +863,17 @@ cudaError_t launch_gated_reduce_cluster(const ReduceArgs& a, const CUtensorMap* 
 // from HBM once, W_f once per CTA.  Every wait is time-limited.
 namespace {
 
-constexpr int TP_T = 32;                   // tokens per tile
 constexpr int TP_C = 4;                    // 128-byte chunks per token in a box
-constexpr int TP_PLANE = TP_T * 128;       // one [32 tokens x 64 elements] bf16 plane
-constexpr int TP_SB = TP_C * TP_PLANE;     // bytes per ring stage
-constexpr int TP_NST = 8;                  // ring stages (128 KB)
-constexpr int TP_NGW = 8;                  // gate warps: (row tile, box phase 0..3)
-// Box j of tile i is stage g = i*NB + j of the ring, slot g % TP_NST, and is
-// read by the two gate warps of phase j % 4.  With NB a multiple of 4 (the
-// tile geometry requires it), slot g % 8 only ever holds boxes of phase g % 4,
-// and the box a gate warp waits for comes 8 stages after one it read itself:
-// no waiter is more than one fill ahead of a slot's barrier (an mbarrier
-// parity wait tells adjacent phases apart only).
-static_assert(TP_NST == 2 * (TP_NGW / 2), "each slot serves one box phase");
+constexpr int TP_RING = 128 * 1024;        // ring bytes
+constexpr int TP_MAXST = 16;               // ring slots at most (16-token tiles)
+constexpr int TP_NGW = 8;                  // gate warps: (sub, box phase 0..3)
+constexpr int TP_NPH = TP_NGW / 2;         // box phases
+// Box j of tile i is stage g = i*NB + j of the ring, slot g % NST, and is
+// read by the two gate warps of phase j % 4.  With NB and NST multiples of 4
+// (the tile geometry requires the first), slot g % NST only ever holds boxes
+// of phase g % 4, and the box a gate warp waits for comes NST stages after
+// one it read itself: no waiter is more than one fill ahead of a slot's
+// barrier (an mbarrier parity wait tells adjacent phases apart only).
 constexpr int TP_NWW = 8;                  // weighted warps
 constexpr int TP_THR = 32 * (2 + TP_NGW + TP_NWW);
 constexpr int TP_LA = 2;                   // gate warps run at most this many tiles ahead of the alpha warp
@@ -886,6 +884,7 @@ constexpr int TP_U = 4;                    // weighted outputs per lane and roun
 
 struct TileGeo {
   int s;     // CTAs per cluster (4 or 8): the d split
+  int t;     // tokens per tile (16 or 32)
   int ec;    // elements per path in a CTA slice (multiple of 64)
   int nkb;   // 128-byte chunks per path slice
   int ngrp;  // boxes per path slice: ngrp - 1 of TP_C chunks, then one of tail chunks
@@ -904,22 +903,35 @@ __device__ __forceinline__ void st_async_v4(uint32_t addr, float4 v, uint32_t ba
                : "memory");
 }
 
-constexpr int tp_xbytes(int S) { return S * TP_T * TP_PS * 4; }  // one tile's partials from all senders
+// one tile's partials from all senders
+constexpr int tp_xbytes(int S, int T) { return S * T * TP_PS * 4; }
+constexpr size_t tp_smem(int S, int T, int m, int wrow) {
+  return 1024 + (size_t)TP_RING + (size_t)tp_xbytes(S, T) * TP_NX + (size_t)TP_NPH * 32 * TP_PS * 4 +
+         (size_t)TP_NAB * T * 16 + (size_t)m * wrow * 2;
+}
 
-template <int M, int S>
+// T tokens per tile: 32 (two 16-row tiles; the two gate warps of a phase
+// take one each) or 16 (one row tile; the two gate warps of a phase take the
+// even and the odd planes of every box).
+template <int M, int S, int T>
 __global__ void __launch_bounds__(TP_THR, 1) gated_reduce_tile_kernel(const ReduceArgs a,
                                                                       const __grid_constant__ TileMaps maps,
                                                                       const TileGeo geo) {
+  static_assert(T == 16 || T == 32, "tokens per tile");
+  constexpr int PLANE = T * 128;      // one [T tokens x 64 elements] bf16 plane
+  constexpr int SB = TP_C * PLANE;    // bytes per ring slot (one box)
+  constexpr int NST = TP_RING / SB;   // ring slots
+  static_assert(NST % TP_NPH == 0 && NST <= TP_MAXST, "each slot serves one box phase");
   extern __shared__ uint8_t tp_smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(tp_smem_raw) + 1023) &
                                              ~static_cast<uintptr_t>(1023));
-  uint8_t* ring = smem;                                                              // [NST][TP_SB]
-  float* xbuf = reinterpret_cast<float*>(smem + TP_NST * TP_SB);                     // [NX][S][T][PS]
-  float* red = xbuf + TP_NX * S * TP_T * TP_PS;                                     // [NGW/2 phases][32][PS]
-  float* alpha_s = red + TP_NGW * 16 * TP_PS;                                        // [NAB][T][4]
-  __nv_bfloat16* wsl = reinterpret_cast<__nv_bfloat16*>(alpha_s + TP_NAB * TP_T * 4);  // [M][wrow]
-  __shared__ __align__(8) uint64_t full_bar[TP_NST];
-  __shared__ __align__(8) uint64_t empty_bar[TP_NST];
+  uint8_t* ring = smem;                                                              // [NST][SB]
+  float* xbuf = reinterpret_cast<float*>(smem + TP_RING);                            // [NX][S][T][PS]
+  float* red = xbuf + TP_NX * S * T * TP_PS;                                         // [phases][32][PS]
+  float* alpha_s = red + TP_NPH * 32 * TP_PS;                                        // [NAB][T][4]
+  __nv_bfloat16* wsl = reinterpret_cast<__nv_bfloat16*>(alpha_s + TP_NAB * T * 4);   // [M][wrow]
+  __shared__ __align__(8) uint64_t full_bar[TP_MAXST];
+  __shared__ __align__(8) uint64_t empty_bar[TP_MAXST];
   __shared__ __align__(8) uint64_t xfull[TP_NX];
   __shared__ __align__(8) uint64_t xdone[TP_NX];
   __shared__ __align__(8) uint64_t alpha_ready[TP_NAB];
@@ -946,9 +958,9 @@ __global__ void __launch_bounds__(TP_THR, 1) gated_reduce_tile_kernel(const Redu
   }
   if (tid < M) bias_s[tid] = a.b[tid];
   if (tid == 0) {
-    for (int i = 0; i < TP_NST; ++i) {
+    for (int i = 0; i < NST; ++i) {
       mbar_init(smem_u32(&full_bar[i]), 1);
-      mbar_init(smem_u32(&empty_bar[i]), 2);  // the two gate warps (row tiles) of the box's parity
+      mbar_init(smem_u32(&empty_bar[i]), 2);  // the two gate warps of the box's phase
     }
     for (int i = 0; i < TP_NX; ++i) {
       mbar_init(smem_u32(&xfull[i]), 1);  // completes on the bytes of every sender
@@ -960,7 +972,7 @@ __global__ void __launch_bounds__(TP_THR, 1) gated_reduce_tile_kernel(const Redu
     }
     abort_flag = 0;
     fence_mbar_init();
-    for (int b = 0; b < TP_NX && b < nl; ++b) mbar_arrive_expect_tx(smem_u32(&xfull[b]), tp_xbytes(S));
+    for (int b = 0; b < TP_NX && b < nl; ++b) mbar_arrive_expect_tx(smem_u32(&xfull[b]), tp_xbytes(S, T));
   }
   __syncthreads();
   cluster_sync_all();  // every rank's barriers exist and are armed before anyone signals them
@@ -982,11 +994,11 @@ __global__ void __launch_bounds__(TP_THR, 1) gated_reduce_tile_kernel(const Redu
     // ------------------------------------------------------------ producer
     long long g = 0;  // stages issued
     for (long long i = 0; i < nl; ++i) {
-      const long long t0 = ((long long)cid + i * ncl) * TP_T;
+      const long long t0 = ((long long)cid + i * ncl) * T;
       bool ok = true;
       for (int j = 0; j < NB; ++j, ++g) {
-        const int s = (int)(g % TP_NST);
-        if (!warp_wait(smem_u32(&empty_bar[s]), (uint32_t)((g / TP_NST) & 1) ^ 1u, false)) {
+        const int s = (int)(g % NST);
+        if (!warp_wait(smem_u32(&empty_bar[s]), (uint32_t)((g / NST) & 1) ^ 1u, false)) {
           ok = false;
           break;
         }
@@ -994,8 +1006,8 @@ __global__ void __launch_bounds__(TP_THR, 1) gated_reduce_tile_kernel(const Redu
         if (lane == 0) {
           const bool last = grp == ngrp - 1;
           const uint32_t fb = smem_u32(&full_bar[s]);
-          mbar_arrive_expect_tx(fb, (last ? geo.tail : TP_C) * TP_PLANE);
-          tma_load_3d(smem_u32(ring + s * TP_SB), last ? &maps.tail : &maps.main, 0, (int)t0,
+          mbar_arrive_expect_tx(fb, (last ? geo.tail : TP_C) * PLANE);
+          tma_load_3d(smem_u32(ring + s * SB), last ? &maps.tail : &maps.main, 0, (int)t0,
                       (pth * d + (int)rank * ec) / 64 + grp * TP_C, fb);
         }
         __syncwarp();
@@ -1003,39 +1015,41 @@ __global__ void __launch_bounds__(TP_THR, 1) gated_reduce_tile_kernel(const Redu
       if (!ok) break;
     }
     // no copy may still be landing when the CTA exits
-    for (long long k = g > TP_NST ? g - TP_NST : 0; k < g; ++k)
-      if (!mbar_wait(smem_u32(&full_bar[k % TP_NST]), (uint32_t)((k / TP_NST) & 1), a.status)) break;
+    for (long long k = g > NST ? g - NST : 0; k < g; ++k)
+      if (!mbar_wait(smem_u32(&full_bar[k % NST]), (uint32_t)((k / NST) & 1), a.status)) break;
   } else if (warp <= TP_NGW) {
     // --------------------------------------------------------------- gates
-    // warp (rt, hb): tokens 16*rt .. 16*rt + 15 of the boxes j with j % 2 == hb
-    const int gw = warp - 1, rt = gw & 1, hb = gw >> 1;  // hb 0..3
+    // warp (sub, hb) reads the boxes j with j % 4 == hb: with 32-token tiles
+    // the 16 tokens 16*sub .. 16*sub + 15 of every plane, with 16-token tiles
+    // all tokens of the planes c with c % 2 == sub
+    const int gw = warp - 1, sub = gw & 1, hb = gw >> 1;  // hb 0..3
     const int g8 = lane >> 2, q = lane & 3;
     const __nv_bfloat16* wrowp = wsl + (size_t)(g8 < M ? g8 : 0) * geo.wrow + 2 * q;
-    const int row = rt * 16 + (lane & 15), hsel = lane >> 4;
+    const int row = (T == 32 ? sub * 16 : 0) + (lane & 15), hsel = lane >> 4;
     for (long long i = 0; i < nl; ++i) {
       float acc[2][4] = {{0.f, 0.f, 0.f, 0.f}, {0.f, 0.f, 0.f, 0.f}};  // two chains: plane parity
       unsigned long long sq0[2] = {0ull, 0ull}, sq1[2] = {0ull, 0ull};
       bool ok = true;
-      for (int j = hb; j < NB; j += TP_NGW / 2) {
+      for (int j = hb; j < NB; j += TP_NPH) {
         const long long gs = i * NB + j;  // stage counter
-        const int s = (int)(gs % TP_NST);
-        if (!warp_wait(smem_u32(&full_bar[s]), (uint32_t)((gs / TP_NST) & 1), false)) {
+        const int s = (int)(gs % NST);
+        if (!warp_wait(smem_u32(&full_bar[s]), (uint32_t)((gs / NST) & 1), false)) {
           ok = false;
           break;
         }
         const int pth = j / ngrp, grp = j - pth * ngrp;
         const int nc = grp == ngrp - 1 ? geo.tail : TP_C;
-        const uint32_t sbase = smem_u32(ring + s * TP_SB);
+        const uint32_t sbase = smem_u32(ring + s * SB);
         const __nv_bfloat16* wk = wrowp + (pth * geo.nkb + grp * TP_C) * 64;
 #pragma unroll
         for (int c = 0; c < TP_C; ++c) {
-          if (c < nc) {
+          if (c < nc && (T == 32 || (c & 1) == sub)) {
             // a plane's fragments first (loads in flight together), then its arithmetic
             uint32_t af[4][4], bf[4][2];
 #pragma unroll
             for (int kk = 0; kk < 4; ++kk) {
               const int chunk = kk * 2 + hsel;
-              ldsm_x4(sbase + c * TP_PLANE + row * 128 + ((chunk ^ (row & 7)) << 4), af[kk][0], af[kk][1],
+              ldsm_x4(sbase + c * PLANE + row * 128 + ((chunk ^ (row & 7)) << 4), af[kk][0], af[kk][1],
                       af[kk][2], af[kk][3]);
               bf[kk][0] = g8 < M ? *reinterpret_cast<const uint32_t*>(wk + c * 64 + kk * 16) : 0u;
               bf[kk][1] = g8 < M ? *reinterpret_cast<const uint32_t*>(wk + c * 64 + kk * 16 + 8) : 0u;
@@ -1053,9 +1067,10 @@ __global__ void __launch_bounds__(TP_THR, 1) gated_reduce_tile_kernel(const Redu
         __syncwarp();
         arrive(&empty_bar[s]);
       }
-      // this warp's [16 tokens][m + 1] partials into red[hb]; the hb = 0 warps
-      // add the four box phases and send one row per lane to every rank
-      float* rw = red + ((size_t)hb * TP_T + rt * 16) * TP_PS;
+      // this warp's [16 tokens][m + 1] partials into rows 16*sub.. of red[hb];
+      // sender warps add the box phases (and with 16-token tiles the two plane
+      // halves) in a fixed order and send one token row per lane to every rank
+      float* rw = red + ((size_t)hb * 32 + sub * 16) * TP_PS;
       {
         float s0 = sum2(sq0[0]) + sum2(sq0[1]), s1 = sum2(sq1[0]) + sum2(sq1[1]);
         s0 += __shfl_xor_sync(0xffffffffu, s0, 1);
@@ -1084,7 +1099,7 @@ __global__ void __launch_bounds__(TP_THR, 1) gated_reduce_tile_kernel(const Redu
           : "memory");
       if (!go) break;
       bool sent = true;
-      if (hb == 0) {
+      if (hb == 0 && (T == 32 || sub == 0)) {
         // credit: this rank's alpha warp has read tile i - LA, so every rank
         // has read the buffer this tile's partials go to
         if (i >= TP_LA) {
@@ -1093,18 +1108,22 @@ __global__ void __launch_bounds__(TP_THR, 1) gated_reduce_tile_kernel(const Redu
         }
         if (sent && lane < 16) {
           const int b = (int)(i % TP_NX);
-          const float* r0 = red + (size_t)(rt * 16 + lane) * TP_PS;
+          const int tok = (T == 32 ? sub * 16 : 0) + lane;
+          const float* r0 = red + (size_t)(T == 32 ? sub * 16 + lane : lane) * TP_PS;
           float4 lo = make_float4(0.f, 0.f, 0.f, 0.f), hi = lo;
 #pragma unroll
-          for (int h = 0; h < TP_NGW / 2; ++h) {  // the box phases in a fixed order
-            const float4 ah = *reinterpret_cast<const float4*>(r0 + h * TP_T * TP_PS);
-            lo.x += ah.x;
-            lo.y += ah.y;
-            lo.z += ah.z;
-            lo.w += ah.w;
-            hi.x += r0[h * TP_T * TP_PS + 4];
-          }
-          const uint32_t lx = smem_u32(xbuf + (((size_t)b * S + rank) * TP_T + rt * 16 + lane) * TP_PS);
+          for (int h = 0; h < TP_NPH; ++h)  // the box phases in a fixed order
+#pragma unroll
+            for (int hs = 0; hs < (T == 32 ? 1 : 2); ++hs) {  // then the plane halves
+              const float* rr = r0 + (h * 32 + hs * 16) * TP_PS;
+              const float4 ah = *reinterpret_cast<const float4*>(rr);
+              lo.x += ah.x;
+              lo.y += ah.y;
+              lo.z += ah.z;
+              lo.w += ah.w;
+              hi.x += rr[4];
+            }
+          const uint32_t lx = smem_u32(xbuf + (((size_t)b * S + rank) * T + tok) * TP_PS);
           const uint32_t lb = smem_u32(&xfull[b]);
 #pragma unroll
           for (uint32_t r = 0; r < S; ++r) {
@@ -1133,11 +1152,12 @@ __global__ void __launch_bounds__(TP_THR, 1) gated_reduce_tile_kernel(const Redu
         ok = false;
         break;
       }
-      // lane = token: its partials from the 8 ranks, summed in rank order
+      // lane = token: its partials from the ranks, summed in rank order
       float v[5] = {0.f, 0.f, 0.f, 0.f, 0.f};
+      const int tl = lane < T ? lane : 0;  // lanes past the tile repeat token 0 and store nothing
 #pragma unroll
       for (int r = 0; r < S; ++r) {
-        const float* x = xbuf + (((size_t)b * S + r) * TP_T + lane) * TP_PS;
+        const float* x = xbuf + (((size_t)b * S + r) * T + tl) * TP_PS;
         const float4 lo = *reinterpret_cast<const float4*>(x);
         v[0] += lo.x;
         v[1] += lo.y;
@@ -1148,7 +1168,7 @@ __global__ void __launch_bounds__(TP_THR, 1) gated_reduce_tile_kernel(const Redu
       __syncwarp();
       // buffer b is read: arm it for tile i + NX (no rank sends that tile
       // before this warp has read tile i + 2) and give the credit
-      if (lane == 0 && i + TP_NX < nl) mbar_arrive_expect_tx(smem_u32(&xfull[b]), tp_xbytes(S));
+      if (lane == 0 && i + TP_NX < nl) mbar_arrive_expect_tx(smem_u32(&xfull[b]), tp_xbytes(S, T));
       arrive(&xdone[b]);
       const int ab = (int)(i % TP_NAB);
       if (i >= TP_NAB && !warp_wait(smem_u32(&alpha_free[ab]), (uint32_t)(((i / TP_NAB) - 1) & 1), false)) {
@@ -1159,9 +1179,10 @@ __global__ void __launch_bounds__(TP_THR, 1) gated_reduce_tile_kernel(const Redu
       float al[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
       for (int j = 0; j < M; ++j) al[j] = 1.0f / (1.0f + expf(-(a.gate_scale * r * v[j] + bias_s[j]))) + a.gate_offset;
-      *reinterpret_cast<float4*>(alpha_s + ((size_t)ab * TP_T + lane) * 4) = make_float4(al[0], al[1], al[2], al[3]);
-      const long long t = ((long long)cid + i * ncl) * TP_T + lane;
-      if (a.alpha_out && rank == 0 && t < N)
+      if (lane < T)
+        *reinterpret_cast<float4*>(alpha_s + ((size_t)ab * T + lane) * 4) = make_float4(al[0], al[1], al[2], al[3]);
+      const long long t = ((long long)cid + i * ncl) * T + lane;
+      if (a.alpha_out && rank == 0 && lane < T && t < N)
 #pragma unroll
         for (int j = 0; j < M; ++j) a.alpha_out[t * M + j] = al[j];
       __syncwarp();
@@ -1181,14 +1202,14 @@ __global__ void __launch_bounds__(TP_THR, 1) gated_reduce_tile_kernel(const Redu
     // ------------------------------------------------------- weighted warps
     const int ww = warp - TP_NGW - 2;
     const int vpt = ec / 8;            // 16-byte outputs per token in the slice
-    const int nitems = TP_T * vpt;
+    const int nitems = T * vpt;
     const __nv_bfloat16* H = reinterpret_cast<const __nv_bfloat16*>(a.H);
     __nv_bfloat16* y = reinterpret_cast<__nv_bfloat16*>(a.y);
     for (long long i = 0; i < nl; ++i) {
       const int ab = (int)(i % TP_NAB);
       if (!warp_wait(smem_u32(&alpha_ready[ab]), (uint32_t)((i / TP_NAB) & 1), false)) break;
-      const long long t0 = ((long long)cid + i * ncl) * TP_T;
-      const float* al_s = alpha_s + (size_t)ab * TP_T * 4;
+      const long long t0 = ((long long)cid + i * ncl) * T;
+      const float* al_s = alpha_s + (size_t)ab * T * 4;
       for (int w0 = ww * 32 + lane; w0 < nitems; w0 += TP_NWW * 32 * TP_U) {
         uint4 h[TP_U][M];
         int tk[TP_U], col[TP_U];
@@ -1228,10 +1249,10 @@ __global__ void __launch_bounds__(TP_THR, 1) gated_reduce_tile_kernel(const Redu
   cluster_sync_all();  // no rank still writes into this CTA's shared memory
 }
 
-template <int M, int S>
-cudaError_t launch_tile_ms(const ReduceArgs& a, const TileGeo& geo, size_t smem, const TileMaps* maps,
-                           cudaStream_t s) {
-  auto k = gated_reduce_tile_kernel<M, S>;
+template <int M, int S, int T>
+cudaError_t launch_tile_mst(const ReduceArgs& a, const TileGeo& geo, size_t smem, const TileMaps* maps,
+                            cudaStream_t s) {
+  auto k = gated_reduce_tile_kernel<M, S, T>;
   static size_t cached_smem = 0;
   static int cached_clusters = 0;
   cudaError_t e;
@@ -1263,29 +1284,41 @@ cudaError_t launch_tile_ms(const ReduceArgs& a, const TileGeo& geo, size_t smem,
 template <int M>
 cudaError_t launch_tile_m(const ReduceArgs& a, const TileGeo& geo, size_t smem, const TileMaps* maps,
                           cudaStream_t s) {
-  return geo.s == 4 ? launch_tile_ms<M, 4>(a, geo, smem, maps, s) : launch_tile_ms<M, 8>(a, geo, smem, maps, s);
+  if (geo.s == 4)
+    return geo.t == 32 ? launch_tile_mst<M, 4, 32>(a, geo, smem, maps, s) : launch_tile_mst<M, 4, 16>(a, geo, smem, maps, s);
+  return geo.t == 32 ? launch_tile_mst<M, 8, 32>(a, geo, smem, maps, s) : launch_tile_mst<M, 8, 16>(a, geo, smem, maps, s);
 }
 
-// Cluster size: 8 CTAs once the W_f slices of a 4-CTA split would crowd the
-// ring (d >= 4096 at m = 4); 4 below, where more clusters fit the GPCs
-// (measured: 5.0 vs 3.9 TB/s at d = 2048, 4.1 vs 3.7 TB/s at d = 7168).
+// The weighted pass re-reads a CTA's slice of a tile from L2, so the slice
+// must stay in it: with 4-CTA clusters and 32 tokens at m = 4, d = 7168 (459 KB
+// slices) the launch read 800 MB from DRAM for 470 MB of H.  The geometry is
+// the first of (4 CTAs, 32 tokens), (8, 32), (4, 16), (8, 16) whose slice is
+// at most 300 KB, whose boxes per tile are a whole number of phases and
+// whose shared memory fits: 4-CTA clusters fit more SMs (5.0 vs 3.9 TB/s at
+// d = 2048), 16-token tiles pay twice the per-box and exchange overhead (3.2
+// vs 4.1 TB/s at d = 7168).
 bool tile_geometry(const ReduceArgs& a, int dtype, TileGeo* geo, size_t* smem) {
   if (dtype != HDF_BF16 || a.alpha_override || a.path_norm_w) return false;
   if (a.n_tokens <= 0 || a.n_tokens > (1ll << 31) - 64) return false;  // TMA coordinates are 32-bit
   if (!(a.m == 1 || a.m == 2 || a.m == 4)) return false;
-  const int S = (long long)a.m * a.m * a.d * 2 / 4 > 32 * 1024 ? 8 : 4;
-  if (a.d % (S * 64)) return false;
-  geo->s = S;
-  geo->ec = a.d / S;
-  geo->nkb = geo->ec / 64;
-  geo->ngrp = (geo->nkb + TP_C - 1) / TP_C;
-  geo->tail = geo->nkb - (geo->ngrp - 1) * TP_C;
-  if ((a.m * geo->ngrp) % (TP_NGW / 2)) return false;  // boxes per tile: a multiple of the 4 phases
-  geo->wrow = a.m * geo->ec + 8;  // + 16 bytes: the gate rows of one B fragment sit in distinct banks
-  geo->ntiles = (a.n_tokens + TP_T - 1) / TP_T;
-  *smem = 1024 + (size_t)TP_NST * TP_SB + (size_t)tp_xbytes(S) * TP_NX + (size_t)(TP_NGW / 2) * TP_T * TP_PS * 4 +
-          (size_t)TP_NAB * TP_T * 16 + (size_t)a.m * geo->wrow * 2;
-  return *smem <= 227 * 1024;
+  const int order[4][2] = {{4, 32}, {8, 32}, {4, 16}, {8, 16}};
+  for (const auto& st : order) {
+    const int S = st[0];
+    if (a.d % (S * 64)) continue;
+    geo->s = S;
+    geo->ec = a.d / S;
+    geo->t = st[1];
+    if ((size_t)geo->t * a.m * geo->ec * 2 > 300 * 1024) continue;
+    geo->nkb = geo->ec / 64;
+    geo->ngrp = (geo->nkb + TP_C - 1) / TP_C;
+    geo->tail = geo->nkb - (geo->ngrp - 1) * TP_C;
+    if ((a.m * geo->ngrp) % TP_NPH) continue;  // boxes per tile: a multiple of the 4 phases
+    geo->wrow = a.m * geo->ec + 8;  // + 16 bytes: the gate rows of one B fragment sit in distinct banks
+    geo->ntiles = (a.n_tokens + geo->t - 1) / geo->t;
+    *smem = tp_smem(S, geo->t, a.m, geo->wrow);
+    if (*smem <= 227 * 1024) return true;
+  }
+  return false;
 }
 
 }  // namespace
@@ -1295,7 +1328,7 @@ bool reduce_tile_boxes(const ReduceArgs& a, int dtype, unsigned box[3], unsigned
   size_t smem;
   if (!tile_geometry(a, dtype, &geo, &smem)) return false;
   box[0] = tail_box[0] = 64;
-  box[1] = tail_box[1] = TP_T;
+  box[1] = tail_box[1] = (unsigned)geo.t;
   box[2] = (unsigned)std::min(TP_C, geo.nkb);
   tail_box[2] = (unsigned)geo.tail;
   return true;

@@ -46,6 +46,8 @@ def _run(inp, **kw):
     (32, 4, 512, "bf16", 0.1),      # one whole 32-token tile, one 64-element block per CTA
     (33, 1, 512, "bf16", 0.1),      # a tile of one token after a full one
     (1000, 4, 7168, "bf16", 0.1),   # 56 k-blocks per CTA: the stage ring wraps in both passes
+    (300, 4, 16384, "bf16", 0.1),   # the widest d: 16-token tiles in 8-CTA clusters
+    (333, 2, 7168, "bf16", 0.1),    # m = 2 at the sweep width: 8-CTA clusters
 ])
 def test_reduce_parity(N, m, d, dtype, std, reduce_path):
     inp = W.make_reduce_inputs(N, m, d, dtype, std, seed=N * 131 + d)
