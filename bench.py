@@ -508,21 +508,21 @@ def measure_warm(cfg, inp, drafter, y, tok_cold, tgt, stream, steps, dev, pk):
 # profiles/*_decode.md, decode workload only; an entry must be removed when
 # its kernel changes.
 NCU_DRAM_BYTES_DECODE = {
-    "L0.ctx_kv_gemm": 26288384 + 2816,
-    "L0.qkv_gemm": 25340160,
-    "L0.o_gemm": 8668928,
-    "L0.gate_up_gemm": 67264512 + 452864,
-    "L0.down_gemm": 34031360,
-    "lm_head": 134365952 + 3178496,
+    "L0.ctx_kv_gemm": 26287616 + 1280,
+    "L0.qkv_gemm": 25341696,
+    "L0.o_gemm": 8667136,
+    "L0.gate_up_gemm": 67264768 + 301568,
+    "L0.down_gemm": 34029312,
+    "lm_head": 134369536 + 3009280,
     "L0.attention": 17016576,
-    "gated_reduce": 33675008,
+    "gated_reduce": 33675264,
 }
 
 
 # DRAM bytes (read + write) per token of the tile reducer at m = 4, d = 7168,
 # from the ncu capture summarised in profiles/gated_reduce_sweep.md (8192
 # tokens; traffic grows with the tokens)
-NCU_DRAM_BYTES_PER_TOKEN_SWEEP = (470288896 + 87983616) / 8192
+NCU_DRAM_BYTES_PER_TOKEN_SWEEP = (470209024 + 87422976) / 8192
 
 
 def roofline_of(cfg, res, pk):
