@@ -205,7 +205,11 @@ def run_ours(args, rank, world, local_rank):
     for e in [x for row in evs + outer for x in row]:
         e.record(stream)
     stream.synchronize()
-    graph = staged = None
+    graph = staged = stepped = None
+    step_marks = [ev() for _ in range(K + 1)]
+    for e in step_marks:
+        e.record(stream)
+    stream.synchronize()
     if not args.eager:
         # the K timed steps are captured once and replayed as one graph, so the
         # host's launch rate does not gate the GPU; a second graph of the same
@@ -219,6 +223,14 @@ def run_ours(args, rank, world, local_rank):
         with torch.cuda.graph(staged, stream=stream):
             for k in range(K):
                 step(tgt, events=evs[k], outer=outer[k])
+        # a third capture with one event between consecutive steps: the
+        # distribution of step times (one record per step)
+        stepped = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(stepped, stream=stream):
+            for k in range(K):
+                step_marks[k].record(stream)
+                step(tgt)
+            step_marks[K].record(stream)
         with torch.cuda.stream(stream):  # replay() launches on the current stream
             graph.replay()  # warm replays (untimed)
             staged.replay()
@@ -257,6 +269,17 @@ def run_ours(args, rank, world, local_rank):
         ms_staged = t0.elapsed_time(t1) / K
     else:
         ms_staged = ms
+    if stepped is not None:
+        with torch.cuda.stream(stream):
+            stepped.replay()
+        stream.synchronize()
+        with torch.cuda.stream(stream):
+            stepped.replay()
+        stream.synchronize()
+        per_step = sorted(step_marks[k].elapsed_time(step_marks[k + 1]) for k in range(K))
+    else:
+        per_step = [ms] * K
+    pct = {f"p{q}": round(float(np.percentile(per_step, q)), 5) for q in (10, 50, 90)}
 
     # per-stage durations over the timed region
     names = ["gated_reduce", "ctx_norm"]
@@ -327,6 +350,35 @@ def run_ours(args, rank, world, local_rank):
                  "mean_accept": round(float(va.float().mean()), 3), "launches": 1}
     del pv, qv
 
+    # ------------------------------------ acceptance kernel at 2^20 blocks
+    # the real sizes are launch-bound (one latency in "stages"); this is the
+    # bandwidth view: drafts and targets [2^20, B-1] int32 with a prefix of
+    # random length matching, every row read up to its first mismatch
+    nb = 1 << 20
+    ga = torch.Generator(device=dev).manual_seed(seed + 11)
+    dr_b = torch.randint(0, V, (nb, nd), device=dev, dtype=torch.int32, generator=ga)
+    keep = torch.randint(0, nd + 1, (nb, 1), device=dev, generator=ga)
+    tg_b = torch.where(torch.arange(nd, device=dev)[None, :] < keep, dr_b, (dr_b + 1) % V)
+    acc_b = torch.empty(nb, dtype=torch.int32, device=dev)
+    for _ in range(3):
+        hdf.hdf_accept_len(dr_b, tg_b, n_draft=nd, draft_stride=nd, batch=nb, accept=acc_b, stream=stream)
+    stream.synchronize()
+    k0.record(stream)
+    for _ in range(20):
+        hdf.hdf_accept_len(dr_b, tg_b, n_draft=nd, draft_stride=nd, batch=nb, accept=acc_b, stream=stream)
+    k1.record(stream)
+    stream.synchronize()
+    a_us = k0.elapsed_time(k1) / 20 * 1000
+    # algorithmic bytes as in the stage table: both rows of every block (a
+    # row ends inside one or two 32-byte sectors whatever its first
+    # mismatch), plus the lengths written
+    a_bytes = 2 * nb * nd * 4 + nb * 4
+    if not torch.equal(acc_b, keep[:, 0].to(torch.int32)):
+        raise RuntimeError("acceptance sweep: lengths differ from the planted prefixes")
+    accept_sweep = {"batch": nb, "n_draft": nd, "us": round(a_us, 2), "bytes": a_bytes,
+                    "gbs": round(a_bytes / a_us / 1e3, 1), "launches": 1}
+    del dr_b, tg_b, keep, acc_b
+
     # ------------------------------------------- warm (incremental) step
     warm = None
     if not args.no_warm:
@@ -369,7 +421,7 @@ def run_ours(args, rank, world, local_rank):
         torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
         ms, e2e_ms = float(t[0]), float(t[1])
     return dict(cfg=cfg, ms=ms, ms_staged=ms_staged, e2e_ms=e2e_ms, dur=dur, clk=clk, kl=kl, verify_t1=verify_t1,
-                warm=warm, batch=batch, n_ctx=n_ctx, lens=lens,
+                warm=warm, pct=pct, accept_sweep=accept_sweep, batch=batch, n_ctx=n_ctx, lens=lens,
                 h2d=h2d, d2h=d2h, acc_mean=acc_mean, tok=tok, y=y, inputs=inp, tgt=tgt)
 
 
@@ -766,10 +818,13 @@ def main():
                                   "; stage times from a second replay of the same steps with an event record "
                                   "between stages (ms_per_step_instrumented)")},
             "ms_per_step_instrumented": round(res["ms_staged"], 5),
+            "step_ms_percentiles": res["pct"],
+            "blocks_per_s_at_median": round(res["batch"] * world / (res["pct"]["p50"] / 1e3), 2),
             "roofline": rf,
             "reducer": {"gbs": red.get("gbs"), "frac_hbm": red.get("frac"), "us": red["us"]},
             "kl_target": dict(res["kl"], frac_hbm=round(res["kl"]["gbs"] / pk["hbm_gbs"], 3)),
             "verify_t1": res["verify_t1"],
+            "accept_sweep": dict(res["accept_sweep"], frac_hbm=round(res["accept_sweep"]["gbs"] / pk["hbm_gbs"], 3)),
             "warm_step": res["warm"],
             "stages": stages,
             "e2e": {"value": round(e2e_val, 2), "unit": "blocks/s", "h2d_bytes_per_step": res["h2d"],

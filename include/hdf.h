@@ -328,6 +328,8 @@ HDF_API int hdf_lm_head_argmax_static(const void* h, int dtype, int64_t M, int d
  * so the drafts can be read straight out of hdf_lm_head_argmax's tok
  * (draft = tok + 1, draft_stride = B).  tau = mean(accept + 1) counts the
  * bonus token (Table 2 prints tau above the number of drafted steps).
+ * 0 <= n_draft <= 47 (HDF_ERR_UNSUPPORTED above: the rows of 128 sequences
+ * are staged in 48 KB of shared memory).
  * ---------------------------------------------------------------------- */
 HDF_API int hdf_accept_len(const int32_t* draft, int64_t draft_stride,
                    const int32_t* target, int64_t target_stride,

@@ -962,6 +962,7 @@ int hdf_accept_len(const int32_t* draft, int64_t draft_stride, const int32_t* ta
                    int batch, int n_draft, int32_t* accept, hdf_stream_t stream) {
   g_err.clear();
   if (batch < 0 || n_draft < 0) return fail(HDF_ERR_SHAPE, "batch/n_draft");
+  if (n_draft > 47) return fail(HDF_ERR_UNSUPPORTED, "n_draft %d > 47", n_draft);
   if (batch == 0) return HDF_OK;
   if (!draft || !target || !accept) return fail(HDF_ERR_INVALID_ARG, "null pointer");
   if (draft_stride < n_draft || target_stride < n_draft) return fail(HDF_ERR_SHAPE, "stride < n_draft");

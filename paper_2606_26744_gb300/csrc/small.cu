@@ -127,15 +127,57 @@ cudaError_t launch_norm_t(const void* x, const void* w, void* y, long long rows,
   return cudaErrorInvalidValue;
 }
 
-__global__ void accept_kernel(const int* __restrict__ draft, long long ds, const int* __restrict__ target,
-                              long long ts, int batch, int nd, int* __restrict__ accept) {
+// Accepted-prefix length (Sec. 3.4): n_i = the number of leading draft
+// tokens equal to the target's.  A CTA stages the rows of ACC_ROWS sequences
+// of both inputs in shared memory with coalesced loads (consecutive threads,
+// consecutive entries), then each thread scans its own row there.
+constexpr int ACC_ROWS = 128;
+__global__ void __launch_bounds__(ACC_ROWS) accept_kernel(const int* __restrict__ draft, long long ds,
+                                                          const int* __restrict__ target, long long ts, int batch,
+                                                          int nd, int* __restrict__ accept) {
+  extern __shared__ int acc_sm[];  // [2][ACC_ROWS][nd]
   pdl_launch_dependents();
   pdl_wait();
-  const int i = blockIdx.x * blockDim.x + threadIdx.x;
-  if (i >= batch) return;
+  const long long r0 = (long long)blockIdx.x * ACC_ROWS;
+  const int rows = (int)min((long long)ACC_ROWS, (long long)batch - r0);
+  int* sd = acc_sm;
+  int* st = acc_sm + ACC_ROWS * nd;
+  const int total = rows * nd;
+  if (nd > 0) {
+    // entry e = r * nd + k, advanced by ACC_ROWS entries a step without a division
+    const int rstep = ACC_ROWS / nd, kstep = ACC_ROWS - rstep * nd;
+    int r = threadIdx.x / nd, k = threadIdx.x - r * nd;
+    for (int base = threadIdx.x; base < total; base += 8 * ACC_ROWS) {
+      int vd[8], vt[8];
+#pragma unroll
+      for (int u = 0; u < 8; ++u) {  // eight pairs of loads in flight before any store
+        if (base + u * ACC_ROWS < total) {
+          vd[u] = __ldcs(draft + (r0 + r) * ds + k);
+          vt[u] = __ldcs(target + (r0 + r) * ts + k);
+        }
+        r += rstep;
+        k += kstep;
+        if (k >= nd) {
+          k -= nd;
+          ++r;
+        }
+      }
+#pragma unroll
+      for (int u = 0; u < 8; ++u) {
+        const int e = base + u * ACC_ROWS;
+        if (e < total) {
+          sd[e] = vd[u];
+          st[e] = vt[u];
+        }
+      }
+    }
+  }
+  __syncthreads();
+  const int i = threadIdx.x;
+  if (i >= rows) return;
   int n = 0;
-  while (n < nd && draft[(long long)i * ds + n] == target[(long long)i * ts + n]) ++n;
-  accept[i] = n;
+  while (n < nd && sd[i * nd + n] == st[i * nd + n]) ++n;
+  accept[r0 + i] = n;
 }
 
 // Cache length update after an append: len[b] += n_b (n_b = cu[b+1] - cu[b]),
@@ -246,8 +288,8 @@ cudaError_t launch_embed_norm(const void* embed, const void* mask_vec, const int
 cudaError_t launch_accept(const int* draft, long long ds, const int* target, long long ts, int batch, int nd,
                           int* accept, cudaStream_t s) {
   if (batch == 0) return cudaSuccess;
-  return launch_kernel(accept_kernel, dim3((batch + 127) / 128), dim3(128), 0, s, 1u, draft, ds, target, ts, batch,
-                       nd, accept);
+  return launch_kernel(accept_kernel, dim3((unsigned)((batch + ACC_ROWS - 1) / ACC_ROWS)), dim3(ACC_ROWS),
+                       (size_t)2 * ACC_ROWS * nd * sizeof(int), s, 1u, draft, ds, target, ts, batch, nd, accept);
 }
 
 cudaError_t launch_cache_advance(int* len, const int* cu, int batch, long long cap, int* status, cudaStream_t s) {

@@ -84,6 +84,7 @@ def test_lm_head_and_accept_host_validation(lib):
     assert lib.hdf_accept_len(v(16), 3, v(16), 7, 2, 7, v(16), None) == 2   # stride < n_draft
     assert lib.hdf_accept_len(None, 7, v(16), 7, 2, 7, v(16), None) == 1
     assert lib.hdf_accept_len(None, 7, None, 7, 0, 7, None, None) == 0      # empty batch
+    assert lib.hdf_accept_len(v(16), 48, v(16), 48, 2, 48, v(16), None) == 7  # n_draft above 47
 
 
 def test_draft_block_host_validation(lib):

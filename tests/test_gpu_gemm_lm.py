@@ -102,3 +102,18 @@ def test_rope_table_matches_definition():
     ang = pos[:, None] * 10000.0 ** (-2.0 * i / hd)[None, :]
     np.testing.assert_allclose(to64(c[pos]), np.cos(ang), rtol=0, atol=2e-7)
     np.testing.assert_allclose(to64(s[pos]), np.sin(ang), rtol=0, atol=2e-7)
+
+
+@pytest.mark.parametrize("batch,nd,ds,ts", [(1000, 15, 16, 15), (129, 47, 50, 47), (1 << 17, 7, 7, 9)])
+def test_accept_len_staged_rows(batch, nd, ds, ts):
+    """Ragged CTAs of 128 sequences, strides above n_draft, the largest n_draft."""
+    g = torch.Generator().manual_seed(batch + nd)
+    draft = torch.randint(0, 1000, (batch, ds), generator=g, dtype=torch.int32)
+    keep = torch.randint(0, nd + 1, (batch,), generator=g)
+    target = torch.randint(0, 1000, (batch, ts), generator=g, dtype=torch.int32)
+    k = torch.arange(ts)[None, :]
+    target = torch.where(k < keep[:, None], torch.nn.functional.pad(draft, (0, max(0, ts - ds)))[:, :ts], (target % 997) + 1001)
+    acc = hdf.hdf_accept_len(draft.cuda(), target.cuda(), n_draft=nd, draft_stride=ds, batch=batch)
+    ref = O.accept_len(draft[:, :nd].numpy(), target[:, :nd].numpy())
+    assert np.array_equal(acc.cpu().numpy(), ref)
+    assert np.array_equal(ref, keep.numpy())
