@@ -111,6 +111,15 @@ __device__ __forceinline__ long long ctx_store_row(const Epilogue& E, long long 
   return (long long)lo * E.cache_cap + p;
 }
 
+// Token column j of a kEpiStoreT GEMM: its output row (or -1: not stored)
+// and its RoPE position.  Context rows (modes 1 and 3) as ctx_store_row;
+// block rows land at row j, at their block position.
+__device__ __forceinline__ long long column_target(const Epilogue& E, long long j, int* pos, int* status) {
+  if (E.pos_mode == 1 || E.pos_mode == 3) return ctx_store_row(E, j, pos, status);
+  *pos = E.pos_mode == 0 ? 0 : block_position(E, (int)j);
+  return j;
+}
+
 template <typename T>
 __device__ __forceinline__ void store16(T* dst, const float* v);
 template <>
@@ -176,18 +185,27 @@ __device__ __forceinline__ void epilogue_chunk(const GemmArgs& g, int tile_m, in
     }
     case kEpiStoreT: {  // rows = output features, columns = tokens
       const int f = tile_m * BM + row;
-      const int seg = f / E.seg_width;
+      const int seg = f / E.seg_width;  // one segment per tile: seg_width is a multiple of 128
       const int fl = f - seg * E.seg_width;
       const int jb = tile_n * BN + c0;
-      if ((E.rope_mask >> seg) & 1) {  // pair (2i, 2i+1) lives in lanes (l, l^1)
+      const bool rope = (E.rope_mask >> seg) & 1;
+      // lane k of each warp finds the output row and RoPE position of token
+      // jb + (k & 15) and the warp shares them: one round trip, not one per token
+      const int kk = lane & 15;
+      int my_pos = 0;
+      const long long my_row = jb + kk < g.N ? column_target(E, jb + kk, &my_pos, g.status) : -1;
+      my_pos = (int)min((long long)my_pos, E.rope_rows - 1);
+      long long orow[16];
+#pragma unroll
+      for (int k = 0; k < 16; ++k) orow[k] = __shfl_sync(0xffffffffu, my_row, k);
+      if (rope) {  // pair (2i, 2i+1) lives in lanes (l, l^1)
         const bool even = (fl & 1) == 0;
         const int hh = E.head_dim >> 1;
         const int pi = (fl % E.head_dim) >> 1;
-        // all 16 positions and table entries first: independent loads in flight together
         int pos[16];
 #pragma unroll
-        for (int k = 0; k < 16; ++k)
-          pos[k] = jb + k < g.N ? (int)min((long long)block_position(E, jb + k), E.rope_rows - 1) : 0;
+        for (int k = 0; k < 16; ++k) pos[k] = __shfl_sync(0xffffffffu, my_pos, k);
+        // all 16 table entries of each table: independent loads in flight together
         float cs[16], sn[16];
 #pragma unroll
         for (int k = 0; k < 16; ++k) {
@@ -203,10 +221,8 @@ __device__ __forceinline__ void epilogue_chunk(const GemmArgs& g, int tile_m, in
       if (f >= g.M) return;
       T* out = reinterpret_cast<T*>(E.out[seg]);
 #pragma unroll
-      for (int k = 0; k < 16; ++k) {
-        const int j = jb + k;
-        if (j < g.N) out[(long long)j * E.ld + fl] = from_f32<T>(v[k]);
-      }
+      for (int k = 0; k < 16; ++k)
+        if (orow[k] >= 0) out[orow[k] * E.ld + fl] = from_f32<T>(v[k]);
       return;
     }
     case kEpiResidT: {

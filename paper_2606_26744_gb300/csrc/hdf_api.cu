@@ -442,26 +442,56 @@ size_t cache_layer_offset(const hdf_draft_shape* sh, const hdf_ctx_cache* cache,
   return (size_t)l * sh->batch * (size_t)cache->capacity * sh->d * esize(sh->dtype);
 }
 
-// [K_c | V_c] = c [W_k; W_v]^T with RoPE on K_c (context rows as GEMM rows,
-// no K split, so every row's sums run in the same order whatever the launch).
+// Context rows up to which the K/V projection runs weights-as-A: the
+// weight rows fill the 128-row tiles and the few context rows ride in one
+// narrow column tile, instead of a 128-row tile of mostly absent rows that
+// every CTA of the grid reads at once.
+constexpr long long kCtxKvSwapRows = 256;
+
+// Tile width of the row-major context K/V GEMM: 256 columns when a 256-wide
+// grid covers every SM (the projection of a whole context is compute-bound);
+// otherwise the widest tile that still gives two CTAs per SM, down to 16.
+int ctx_kv_bn(const hdf_draft_shape* sh, long long rows) {
+  const long long row_tiles = (rows + 127) / 128;
+  if (sh->d % 256 == 0 && row_tiles * (2LL * sh->d / 256) >= num_sms()) return 256;
+  int bn = 128;
+  while (bn > 16 && row_tiles * (2LL * sh->d / bn) < 2LL * num_sms()) bn >>= 1;
+  return bn;
+}
+
+// [K_c | V_c] = c [W_k; W_v]^T with RoPE on K_c.  Never a K split: each
+// output element is one K-ordered accumulation whatever the orientation or
+// tile width, so a row's K / V do not depend on the launch that made them.
 // pos_mode 1: rows land packed in kout / vout; pos_mode 3: rows are appended
 // to a cache (cu = cu_new, len, cap).
 int launch_ctx_kv(const hdf_drafter_weights* w, const hdf_layer_weights& Lw, const hdf_draft_shape* sh,
-                  const void* c, long long rows, int bn, void* kout, void* vout, const int32_t* cu, int pos_mode,
+                  const void* c, long long rows, void* kout, void* vout, const int32_t* cu, int pos_mode,
                   const int32_t* len, long long cap, cudaStream_t s) {
   const int dt = sh->dtype;
   const long long d = sh->d;
-  SplitPlan p{bn, 1, 0};
+  const bool swap = rows <= kCtxKvSwapRows;
   GemmArgs g;
-  init_gemm(g, dt, rows, 2 * d, d, p);
-  g.group_n = 8;
   int rc;
-  if ((rc = make_map(&g.A.map[0], c, dt, rows, d, d, 64))) return rc;
-  if ((rc = make_map(&g.B.map[0], Lw.wk, dt, d, d, d, p.bn))) return rc;
-  if ((rc = make_map(&g.B.map[1], Lw.wv, dt, d, d, d, p.bn))) return rc;
-  g.pre_operand = 2;  // weights: loaded before the context norm has finished
-  g.B.rows_per_map = (int)d;
-  g.epi.kind = kEpiStore;
+  if (swap) {  // rows = output features of [W_k; W_v], columns = context rows
+    const SplitPlan p{pick_bn(rows), 1, 0};
+    init_gemm(g, dt, 2 * d, rows, d, p);
+    if ((rc = make_map(&g.A.map[0], Lw.wk, dt, d, d, d, 64))) return rc;
+    if ((rc = make_map(&g.A.map[1], Lw.wv, dt, d, d, d, 64))) return rc;
+    g.A.rows_per_map = (int)d;
+    if ((rc = make_map(&g.B.map[0], c, dt, rows, d, d, p.bn))) return rc;
+    g.pre_operand = 1;  // weights: loaded before the context norm has finished
+    g.epi.kind = kEpiStoreT;
+  } else {
+    const SplitPlan p{ctx_kv_bn(sh, rows), 1, 0};
+    init_gemm(g, dt, rows, 2 * d, d, p);
+    g.group_n = 8;
+    if ((rc = make_map(&g.A.map[0], c, dt, rows, d, d, 64))) return rc;
+    if ((rc = make_map(&g.B.map[0], Lw.wk, dt, d, d, d, p.bn))) return rc;
+    if ((rc = make_map(&g.B.map[1], Lw.wv, dt, d, d, d, p.bn))) return rc;
+    g.pre_operand = 2;
+    g.B.rows_per_map = (int)d;
+    g.epi.kind = kEpiStore;
+  }
   g.epi.out[0] = kout;
   g.epi.out[1] = vout;
   g.epi.seg_width = (int)d;
@@ -479,14 +509,6 @@ int launch_ctx_kv(const hdf_drafter_weights* w, const hdf_layer_weights& Lw, con
   g.epi.cache_cap = cap;
   CK(launch_gemm(g, s), "ctx kv gemm");
   return HDF_OK;
-}
-
-// Tile width of the context K/V GEMM: 256 columns, or 128 when a 256-wide
-// grid would leave most SMs idle (few new rows in an append).
-int ctx_kv_bn(const hdf_draft_shape* sh, long long rows) {
-  if (sh->d % 256) return 128;
-  const long long tiles = ((rows + 127) / 128) * (2LL * sh->d / 256);
-  return tiles >= num_sms() ? 256 : 128;
 }
 
 // The block forward of hdf_draft_block.  Context from packed rows (ctx,
@@ -547,7 +569,7 @@ int draft_forward(const hdf_drafter_weights* w, const hdf_draft_shape* sh, const
     // ---- conditioning projection: [K_c | V_c] = c [W_k; W_v]^T, RoPE on K_c
     if ((rc = mark())) return rc;
     if (n_ctx > 0 &&
-        (rc = launch_ctx_kv(w, Lw, sh, c, n_ctx, d % 256 == 0 ? 256 : 128, kc, vc, cu_ctx, 1, nullptr, 0, s)))
+        (rc = launch_ctx_kv(w, Lw, sh, c, n_ctx, kc, vc, cu_ctx, 1, nullptr, 0, s)))
       return rc;
     // context K / V of this layer: the workspace, or the cache
     const void* kctx = kc;
@@ -761,11 +783,10 @@ int hdf_ctx_append(const hdf_drafter_weights* w, const hdf_draft_shape* sh, cons
   const long long d = sh->d;
   void* c = ws;
   CK(launch_rmsnorm(ctx_new, 0, w->ctx_norm, c, sh->dtype, sh->n_ctx, (int)d, sh->norm_eps, s), "ctx norm");
-  const int bn = ctx_kv_bn(sh, sh->n_ctx);
   for (int l = 0; l < sh->n_layers; ++l) {
     char* kl = static_cast<char*>(cache->k) + cache_layer_offset(sh, cache, l);
     char* vl = static_cast<char*>(cache->v) + cache_layer_offset(sh, cache, l);
-    if ((rc = launch_ctx_kv(w, w->layers[l], sh, c, sh->n_ctx, bn, kl, vl, cu_new, 3, cache->len,
+    if ((rc = launch_ctx_kv(w, w->layers[l], sh, c, sh->n_ctx, kl, vl, cu_new, 3, cache->len,
                             cache->capacity, s)))
       return rc;
   }
