@@ -10,11 +10,14 @@
 // 4-stage ring; tile i lands in stage i % 4 and is consumed by warp i % 4,
 // which runs S = Q K^T and O += P V on mma.sync m16n8k16 (the B <= 16 queries
 // are one m16 row tile) with an fp32 online softmax in the log2 domain.  The
-// four warps merge in shared memory; a sequence that fits one chunk writes
-// its output directly, otherwise each CTA writes an fp32 partial (m, l, O)
-// and the last chunk to finish (atomic ticket) merges them.
+// four warps merge in shared memory.  With one chunk per (sequence, head)
+// that is the output; with several (at most 8) the chunks of one (sequence,
+// head) are one thread-block cluster: each CTA leaves its fp32 partial
+// (m, l, O) in its shared memory and, after a cluster barrier, each merges a
+// slice of the block rows over all chunks in chunk order, over DSMEM.
 // With B queries per key the kernel does ~B flops per byte of K/V, so it is
 // bound by HBM, not by the tensor pipe.
+#include <atomic>
 #include <cmath>
 
 #include "common.cuh"
@@ -105,8 +108,9 @@ __global__ void __launch_bounds__(160, 1)
   pdl_wait();  // Q, the block / context K, V and the cache lengths come from the kernels before
   int c0, T;
   context_span(a, b, chunk_id == 0 && h == 0 && tid == 0, &c0, &T);
+  // chunks past the sequence's keys hold no tiles: in a cluster they still
+  // join its barriers, with an empty partial (m = -inf, l = 0)
   const int nc_b = min(a.n_chunks, T > 0 ? (T + a.chunk - 1) / a.chunk : 1);
-  if (chunk_id >= nc_b) return;
   const int kbeg = chunk_id * a.chunk;
   const int kend = min(T, kbeg + a.chunk);
   const int n_ctx_tiles = kend > kbeg ? (kend - kbeg + KT - 1) / KT : 0;
@@ -286,71 +290,93 @@ __global__ void __launch_bounds__(160, 1)
   if (warp == NCW) __syncthreads();  // matches (A)
   __syncthreads();
 
-  // merge the four warps into this chunk's (m, l, O)
-  const float* ow = reinterpret_cast<const float*>(smem);
-  __nv_bfloat16* out = reinterpret_cast<__nv_bfloat16*>(a.out);
-  const size_t base = ((size_t)b * a.n_heads + h) * a.n_chunks;
-  const size_t pidx = (base + chunk_id) * a.block;
-  for (int i = tid; i < B * HD; i += blockDim.x) {
-    const int r = i / HD, col = i - r * HD;
-    float mstar = -INFINITY;
-#pragma unroll
-    for (int w = 0; w < NCW; ++w) mstar = fmaxf(mstar, wm[w][r]);
-    float acc = 0.f, lsum = 0.f;
-#pragma unroll
-    for (int w = 0; w < NCW; ++w) {
-      const float f = wm[w][r] == -INFINITY ? 0.f : exp2f(wm[w][r] - mstar);
-      acc += ow[(w * 16 + r) * HD + col] * f;
-      lsum += wl[w][r] * f;
-    }
-    if (nc_b == 1) {  // the whole sequence in one CTA: final output
-      out[((size_t)b * B + r) * a.d + h * HD + col] = __float2bfloat16_rn(acc / lsum);
-    } else {
-      __stcg(a.part_o + (pidx + r) * HD + col, acc);
-      if (col == 0) {
-        __stcg(a.part_ml + (pidx + r) * 2, mstar);
-        __stcg(a.part_ml + (pidx + r) * 2 + 1, lsum);
-      }
-    }
-  }
-  if (nc_b == 1) return;
-
-  // The last chunk of (sequence, head) to finish merges all chunks (atomic
-  // ticket, nobody waits): O = sum_c O_c 2^(m_c - m*) / sum_c l_c 2^(m_c - m*).
-  // Per-(row, chunk) factors go to shared memory first, so the element loop
-  // issues independent loads.
-  __shared__ int last;
-  __threadfence();
-  __syncthreads();
-  if (tid == 0) last = atomicAdd(a.counters + b * a.n_heads + h, 1) == nc_b - 1;
-  __syncthreads();
-  if (!last) return;
-  __threadfence();
-  float* fac = reinterpret_cast<float*>(smem + NCW * 16 * HD * 4);  // [B][nc_b]
+  // merge the four warps into this chunk's (m, l, O): one factor per (warp,
+  // row), then the element sums over the warps in order, 4 columns per thread
+  __shared__ float fw[NCW][16], pm[16], pl[16];
   if (tid < B) {
     float mstar = -INFINITY;
-    for (int c = 0; c < nc_b; ++c) mstar = fmaxf(mstar, __ldcg(a.part_ml + ((base + c) * a.block + tid) * 2));
-    float l = 0.f;
-    for (int c = 0; c < nc_b; ++c) {
-      const size_t pi = (base + c) * a.block + tid;
-      const float mc = __ldcg(a.part_ml + pi * 2);
-      const float f = mc == -INFINITY ? 0.f : exp2f(mc - mstar);
-      fac[tid * nc_b + c] = f;
-      l += __ldcg(a.part_ml + pi * 2 + 1) * f;
+#pragma unroll
+    for (int w = 0; w < NCW; ++w) mstar = fmaxf(mstar, wm[w][tid]);
+    float lsum = 0.f;
+#pragma unroll
+    for (int w = 0; w < NCW; ++w) {
+      const float f = wm[w][tid] == -INFINITY ? 0.f : exp2f(wm[w][tid] - mstar);
+      fw[w][tid] = f;
+      lsum += wl[w][tid] * f;
     }
-    const float inv = 1.0f / l;
-    for (int c = 0; c < nc_b; ++c) fac[tid * nc_b + c] *= inv;
+    pm[tid] = mstar;
+    pl[tid] = lsum;
   }
   __syncthreads();
-  for (int i = tid; i < B * HD; i += blockDim.x) {
-    const int r = i / HD, col = i - r * HD;
-    float acc = 0.f;
-#pragma unroll 4
-    for (int c = 0; c < nc_b; ++c)
-      acc += __ldcg(a.part_o + ((base + c) * a.block + r) * HD + col) * fac[r * nc_b + c];
-    out[((size_t)b * B + r) * a.d + h * HD + col] = __float2bfloat16_rn(acc);
+  const float* ow = reinterpret_cast<const float*>(smem);
+  __nv_bfloat16* out = reinterpret_cast<__nv_bfloat16*>(a.out);
+  const int nc = (int)gridDim.x;  // chunks per (sequence, head): the cluster size
+  float* po = reinterpret_cast<float*>(smem + NCW * 16 * HD * 4);  // [16][HD] partial O, unnormalised
+  constexpr int C4 = HD / 4;
+  for (int i = tid; i < B * C4; i += blockDim.x) {
+    const int r = i / C4, c4 = i - r * C4;
+    float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+    for (int w = 0; w < NCW; ++w) {
+      const float4 x = *reinterpret_cast<const float4*>(ow + (w * 16 + r) * HD + 4 * c4);
+      const float f = fw[w][r];
+      acc.x += x.x * f;
+      acc.y += x.y * f;
+      acc.z += x.z * f;
+      acc.w += x.w * f;
+    }
+    if (nc == 1) {
+      const float l = pl[r];
+      uint2 pk;
+      pk.x = pack_bf16x2(acc.x / l, acc.y / l);
+      pk.y = pack_bf16x2(acc.z / l, acc.w / l);
+      *reinterpret_cast<uint2*>(out + ((size_t)b * B + r) * a.d + h * HD + 4 * c4) = pk;
+    } else {
+      *reinterpret_cast<float4*>(po + r * HD + 4 * c4) = acc;
+    }
   }
-  if (tid == 0) a.counters[b * a.n_heads + h] = 0;
+  if (nc == 1) return;
+
+  // O = sum_c O_c 2^(m_c - m*) / sum_c l_c 2^(m_c - m*) over the chunks c of
+  // the cluster, in chunk order; rank r merges block rows [r * rpr, (r+1) * rpr)
+  cluster_sync_all();  // every chunk's partial is in its shared memory
+  {
+    const int rank = (int)cluster_rank();
+    const int rpr = (B + nc - 1) / nc;
+    const int r0 = rank * rpr, nr = max(0, min(B, r0 + rpr) - r0);
+    for (int it = tid; it < nr * C4; it += blockDim.x) {
+      const int r = r0 + it / C4, c4 = it - (it / C4) * C4;
+      float mc[8], lc[8];
+#pragma unroll
+      for (int c = 0; c < 8; ++c)
+        if (c < nc) {
+          mc[c] = ld_dsmem_f32(map_rank(smem_u32(&pm[r]), (uint32_t)c));
+          lc[c] = ld_dsmem_f32(map_rank(smem_u32(&pl[r]), (uint32_t)c));
+        }
+      float mstar = -INFINITY;
+#pragma unroll
+      for (int c = 0; c < 8; ++c)
+        if (c < nc) mstar = fmaxf(mstar, mc[c]);
+      float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+      float l = 0.f;
+#pragma unroll
+      for (int c = 0; c < 8; ++c)
+        if (c < nc && mc[c] != -INFINITY) {  // -inf: a chunk without keys of this sequence
+          const float f = exp2f(mc[c] - mstar);
+          const float4 q = ld_dsmem_v4(map_rank(smem_u32(po + r * HD + 4 * c4), (uint32_t)c));
+          acc.x += q.x * f;
+          acc.y += q.y * f;
+          acc.z += q.z * f;
+          acc.w += q.w * f;
+          l += lc[c] * f;
+        }
+      uint2 pk;
+      pk.x = pack_bf16x2(acc.x / l, acc.y / l);
+      pk.y = pack_bf16x2(acc.z / l, acc.w / l);
+      *reinterpret_cast<uint2*>(out + ((size_t)b * B + r) * a.d + h * HD + 4 * c4) = pk;
+    }
+  }
+  cluster_sync_all();  // no CTA leaves while another still reads its shared memory
 }
 
 // fp32 path (tiny correctness workloads): one warp per (sequence, head, query),
@@ -417,12 +443,45 @@ cudaError_t launch_hd(const AttnArgs& a, const AttnTmaps* tm, cudaStream_t s) {
       return e;
     attr_set = true;
   }
-  return launch_kernel(k, dim3(a.n_chunks, a.n_heads, a.batch), dim3(160), attn_smem<HD>(), s, 1u, a, *tm);
+  if (a.n_chunks < 1 || a.n_chunks > 8) return cudaErrorInvalidValue;
+  // the chunks of one (sequence, head) are one cluster
+  return launch_kernel(k, dim3(a.n_chunks, a.n_heads, a.batch), dim3(160), attn_smem<HD>(), s,
+                       (unsigned)a.n_chunks, a, *tm);
 }
 
 }  // namespace
 
 size_t attention_smem_bytes(int head_dim) { return head_dim == 64 ? attn_smem<64>() : attn_smem<128>(); }
+
+// Clusters of `cluster` attention CTAs resident at once (occupancy API), or
+// -1 if it cannot be asked.  Cached per head_dim and cluster size.
+int attention_max_clusters(int head_dim, int cluster) {
+  if ((head_dim != 64 && head_dim != 128) || cluster < 1 || cluster > 8) return -1;
+  static std::atomic<int> cache[2][9];
+  const int hi = head_dim == 128;
+  const int v = cache[hi][cluster].load();
+  if (v != 0) return v;
+  auto k = hi ? attn_bf16_kernel<128> : attn_bf16_kernel<64>;
+  const size_t smem = hi ? attn_smem<128>() : attn_smem<64>();
+  int n = -1;
+  if (cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) == cudaSuccess) {
+    cudaLaunchConfig_t cfg = {};
+    cudaLaunchAttribute attr;
+    attr.id = cudaLaunchAttributeClusterDimension;
+    attr.val.clusterDim.x = (unsigned)cluster;
+    attr.val.clusterDim.y = 1;
+    attr.val.clusterDim.z = 1;
+    cfg.gridDim = dim3((unsigned)cluster * 64);
+    cfg.blockDim = dim3(160);
+    cfg.dynamicSmemBytes = smem;
+    cfg.attrs = &attr;
+    cfg.numAttrs = 1;
+    if (cudaOccupancyMaxActiveClusters(&n, k, &cfg) != cudaSuccess) n = -1;
+  }
+  cudaGetLastError();
+  cache[hi][cluster].store(n);
+  return n;
+}
 
 cudaError_t launch_attention(const AttnArgs& a, const AttnTmaps* tm, int dtype, cudaStream_t s) {
   if (a.batch == 0) return cudaSuccess;

@@ -172,6 +172,12 @@ __device__ __forceinline__ uint32_t map_rank(uint32_t local, uint32_t rank) {
 __device__ __forceinline__ void cluster_sync_all() {
   asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::: "memory");
 }
+// 4-byte load from another CTA's shared memory (address from map_rank)
+__device__ __forceinline__ float ld_dsmem_f32(uint32_t addr) {
+  float v;
+  asm volatile("ld.shared::cluster.f32 %0, [%1];" : "=f"(v) : "r"(addr) : "memory");
+  return v;
+}
 // 16-byte load from another CTA's shared memory (address from map_rank)
 __device__ __forceinline__ float4 ld_dsmem_v4(uint32_t addr) {
   float4 v;

@@ -13,6 +13,7 @@
 #include <atomic>
 #include <mutex>
 #include <string>
+#include <vector>
 
 #include "common.cuh"
 #include "kernels.h"
@@ -188,17 +189,41 @@ void init_gemm(GemmArgs& g, int dtype, long long M, long long N, long long K, co
 
 // ---------------------------------------------------- draft-block layout
 struct DraftLayout {
-  size_t c, kc, vc, h, x, q, kb, vb, o, act, part_o, part_ml, counters, counters_bytes, total;
+  size_t c, kc, vc, h, x, q, kb, vb, o, act, total;
   int chunk, n_chunks;
   SplitPlan qkv, oproj, gu, down;
 };
 
+// Context keys per attention CTA.  The chunks of one (sequence, head) are one
+// thread-block cluster of at most 8 CTAs, each chunk at least 256 keys.  The
+// count is the one with the least waves x (rounds + 2): waves of clusters
+// from the resident clusters the occupancy API gives, rounds of the four
+// consumer warps over the 64-key tiles of the longest chunk (the last one
+// also holds the block's keys), 2 for the fixed cost of a wave; ties go to
+// more chunks.
 int attn_chunk(const hdf_draft_shape* sh, int* n_chunks) {
-  const int per = std::max(1, (2 * num_sms() + sh->batch * sh->n_heads - 1) / (sh->batch * sh->n_heads));
-  int chunk = (sh->max_ctx + per - 1) / per;
-  chunk = std::max(256, ((chunk + 63) / 64) * 64);
-  *n_chunks = std::max(1, (sh->max_ctx + chunk - 1) / chunk);
-  return chunk;
+  const long long bh = std::max(1LL, (long long)sh->batch * sh->n_heads);
+  const int T = sh->max_ctx;
+  int best_chunk = std::max(256, ((T + 63) / 64) * 64), best_nc = 1;
+  long long best_cost = LLONG_MAX;
+  for (int per = 1; per <= 8; ++per) {
+    const int chunk = std::max(256, (((T + per - 1) / per + 63) / 64) * 64);
+    const int nc = std::max(1, (T + chunk - 1) / chunk);
+    if (nc != per) continue;  // the same split as a smaller count
+    const int maxc = attention_max_clusters(sh->head_dim, nc);
+    const long long slots = std::max(1, maxc > 0 ? maxc : num_sms() / nc);
+    const long long waves = (bh + slots - 1) / slots;
+    const int last = (T - (nc - 1) * chunk + 63) / 64 + 1;
+    const int tiles = std::max(chunk / 64, last);
+    const long long cost = waves * ((tiles + 3) / 4 + 2);
+    if (cost <= best_cost) {
+      best_cost = cost;
+      best_chunk = chunk;
+      best_nc = nc;
+    }
+  }
+  *n_chunks = best_nc;
+  return best_chunk;
 }
 
 DraftLayout draft_layout(const hdf_draft_shape* sh) {
@@ -223,16 +248,10 @@ DraftLayout draft_layout(const hdf_draft_shape* sh) {
   L.o = take(M * d * es);
   L.act = take(M * F * es);
   L.chunk = attn_chunk(sh, &L.n_chunks);
-  const size_t np = (size_t)sh->batch * sh->n_heads * L.n_chunks * sh->block;
-  L.part_o = take(np * sh->head_dim * 4);
-  L.part_ml = take(np * 2 * 4);
   L.qkv = plan_swap(sh->dtype, 3 * d, M, d);
   L.oproj = plan_swap(sh->dtype, d, M, d);
   L.gu = plan_swap(sh->dtype, 2 * F, M, d);
   L.down = plan_swap(sh->dtype, d, M, F);
-  // attention merge tickets [batch * heads]
-  L.counters_bytes = up256((size_t)sh->batch * sh->n_heads * 4);
-  L.counters = take(L.counters_bytes);
   L.total = off;
   return L;
 }
@@ -511,6 +530,37 @@ int launch_ctx_kv(const hdf_drafter_weights* w, const hdf_layer_weights& Lw, con
   return HDF_OK;
 }
 
+// Second stream of the calling thread on the current device, with events
+// for fork / join points.  Created once, in relaxed capture mode so that a
+// first call made under stream capture may create it.  nullptr on failure.
+struct SideStream {
+  cudaStream_t s = nullptr;
+  std::vector<cudaEvent_t> ev;
+};
+SideStream* side_stream(size_t n_events) {
+  thread_local SideStream per_dev[64];
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return nullptr;
+  SideStream& ss = per_dev[dev];
+  if (ss.s && ss.ev.size() >= n_events) return &ss;
+  cudaStreamCaptureMode mode = cudaStreamCaptureModeRelaxed;
+  cudaThreadExchangeStreamCaptureMode(&mode);
+  bool ok = true;
+  if (!ss.s) ok = cudaStreamCreateWithFlags(&ss.s, cudaStreamNonBlocking) == cudaSuccess;
+  while (ok && ss.ev.size() < n_events) {
+    cudaEvent_t e;
+    ok = cudaEventCreateWithFlags(&e, cudaEventDisableTiming) == cudaSuccess;
+    if (ok) ss.ev.push_back(e);
+  }
+  cudaThreadExchangeStreamCaptureMode(&mode);
+  if (!ok) {
+    if (ss.s) cudaStreamDestroy(ss.s);
+    ss.s = nullptr;
+    return nullptr;
+  }
+  return &ss;
+}
+
 // The block forward of hdf_draft_block.  Context from packed rows (ctx,
 // cu_ctx: normed and projected here) or from a K/V cache (cache != null).
 int draft_forward(const hdf_drafter_weights* w, const hdf_draft_shape* sh, const void* ctx, const int32_t* cu_ctx,
@@ -537,7 +587,6 @@ int draft_forward(const hdf_drafter_weights* w, const hdf_draft_shape* sh, const
   void* vbk = W + Lo.vb;
   void* o = W + Lo.o;
   void* act = W + Lo.act;
-  int* counters = reinterpret_cast<int*>(W + Lo.counters);
   const long long n_ctx = cached ? 0 : sh->n_ctx;
 
   const int n_ev = trace ? trace->n_events : 0;
@@ -558,19 +607,32 @@ int draft_forward(const hdf_drafter_weights* w, const hdf_draft_shape* sh, const
     return HDF_OK;
   };
 
-  CK(cudaMemsetAsync(counters, 0, Lo.counters_bytes, s), "memset counters");
-  int* attn_counters = counters;
+  // The context path (RMSNorm, then each layer's K/V projection: compute-
+  // bound) runs on a second stream beside the block path (weight-streaming
+  // GEMMs): layer l's projection joins before layer l's attention and starts
+  // once layer l-1's attention has read the shared K/V buffers.  Serial when
+  // stage times are traced.
+  cudaStream_t sc = s;
+  SideStream* side = nullptr;
+  if (!trace && n_ctx > 0) side = side_stream(2 * (size_t)sh->n_layers + 1);
+  if (side) {
+    sc = side->s;
+    CK(cudaEventRecord(side->ev[0], s), "fork record");
+    CK(cudaStreamWaitEvent(sc, side->ev[0], 0), "fork wait");
+  }
   // ---- context RMSNorm
   if ((rc = mark())) return rc;
-  if (n_ctx > 0) CK(launch_rmsnorm(ctx, 0, w->ctx_norm, c, dt, n_ctx, (int)d, sh->norm_eps, s), "ctx norm");
+  if (n_ctx > 0) CK(launch_rmsnorm(ctx, 0, w->ctx_norm, c, dt, n_ctx, (int)d, sh->norm_eps, sc), "ctx norm");
 
   for (int l = 0; l < sh->n_layers; ++l) {
     const hdf_layer_weights& Lw = w->layers[l];
     // ---- conditioning projection: [K_c | V_c] = c [W_k; W_v]^T, RoPE on K_c
     if ((rc = mark())) return rc;
+    if (side && l > 0) CK(cudaStreamWaitEvent(sc, side->ev[2 * l], 0), "attention-done wait");
     if (n_ctx > 0 &&
-        (rc = launch_ctx_kv(w, Lw, sh, c, n_ctx, kc, vc, cu_ctx, 1, nullptr, 0, s)))
+        (rc = launch_ctx_kv(w, Lw, sh, c, n_ctx, kc, vc, cu_ctx, 1, nullptr, 0, sc)))
       return rc;
+    if (side) CK(cudaEventRecord(side->ev[2 * l + 1], sc), "join record");
     // context K / V of this layer: the workspace, or the cache
     const void* kctx = kc;
     const void* vctx = vc;
@@ -632,8 +694,6 @@ int draft_forward(const hdf_drafter_weights* w, const hdf_draft_shape* sh, const
       a.ctx_stride = cached ? cache->capacity : 0;
       a.max_len = sh->max_ctx;
       a.out = o;
-      a.part_o = reinterpret_cast<float*>(W + Lo.part_o);
-      a.part_ml = reinterpret_cast<float*>(W + Lo.part_ml);
       a.batch = sh->batch;
       a.block = sh->block;
       a.n_heads = sh->n_heads;
@@ -642,7 +702,6 @@ int draft_forward(const hdf_drafter_weights* w, const hdf_draft_shape* sh, const
       a.n_ctx = ctx_rows;
       a.chunk = Lo.chunk;
       a.n_chunks = Lo.n_chunks;
-      a.counters = attn_counters;
       a.status = device_status_ptr();
       AttnTmaps tm;
       if (dt == HDF_BF16) {
@@ -654,7 +713,9 @@ int draft_forward(const hdf_drafter_weights* w, const hdf_draft_shape* sh, const
         if ((rc = make_map(&tm.kb, kbk, dt, M, d, d, 64))) return rc;
         if ((rc = make_map(&tm.vb, vbk, dt, M, d, d, 64))) return rc;
       }
+      if (side) CK(cudaStreamWaitEvent(s, side->ev[2 * l + 1], 0), "join wait");
       CK(launch_attention(a, &tm, dt, s), "attention");
+      if (side && l + 1 < sh->n_layers) CK(cudaEventRecord(side->ev[2 * l + 2], s), "attention-done record");
     }
     // ---- h += O W_o^T
     if ((rc = mark())) return rc;

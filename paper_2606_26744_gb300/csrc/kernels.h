@@ -173,13 +173,10 @@ struct AttnArgs {
   long long ctx_stride;
   int max_len;         // with ctx_len: keys past max_len are not attended (status recorded)
   void* out;           // [M, d]
-  float* part_o;       // [batch, heads, chunks, block, hd]
-  float* part_ml;      // [batch, heads, chunks, block, 2]
   int batch, block, n_heads, head_dim, d;
   long long n_ctx;
   int chunk;           // context keys per split
-  int n_chunks;        // splits per (sequence, head) = ceil(max_ctx / chunk) (>= 1)
-  int* counters;       // [batch * n_heads], zero on entry, left zero on exit
+  int n_chunks;        // splits per (sequence, head) = ceil(max_ctx / chunk), 1..8: one cluster
   int* status;
 };
 // bf16 path: TMA maps over context K/V and block K/V, box {64 cols, 64 rows}
@@ -188,5 +185,7 @@ struct AttnTmaps {
 };
 cudaError_t launch_attention(const AttnArgs& a, const AttnTmaps* tm, int dtype, cudaStream_t s);
 size_t attention_smem_bytes(int head_dim);
+// clusters of `cluster` (1..8) attention CTAs resident at once; -1 if unknown
+int attention_max_clusters(int head_dim, int cluster);
 
 }  // namespace hdf
