@@ -22,7 +22,13 @@
  *   - Every call is asynchronous on the caller's CUDA stream (a cudaStream_t
  *     passed as hdf_stream_t; NULL = legacy default stream).  No call
  *     synchronises, and there is no host fallback: if the CUDA kernels cannot
- *     run the call returns HDF_ERR_CUDA.
+ *     run the call returns HDF_ERR_CUDA.  hdf_draft_block (without a trace)
+ *     runs its context projection on a second stream that the library keeps
+ *     per host thread and device (created on first use, with a few events):
+ *     forked from the caller's stream by an event when the call starts and
+ *     joined back into it before the call's later kernels, so the call's work
+ *     is still ordered after earlier work on the caller's stream and before
+ *     later work, and the pair captures into one CUDA graph.
  *   - Arguments are validated on the host before any launch; a rejected call
  *     launches nothing and returns a non-zero status.  hdf_last_error() gives
  *     a human-readable reason (thread-local, valid until the next call).
@@ -197,7 +203,8 @@ typedef struct {
  * n_events = 3 + HDF_DRAFT_STAGES_PER_LAYER * n_layers (or pass NULL).
  * Stages: context norm, then per layer {context K/V GEMM, block
  * norm (+embedding), QKV GEMM, attention (+combine), O GEMM, MLP norm,
- * gate/up GEMM, down GEMM}, then the final norm. */
+ * gate/up GEMM, down GEMM}, then the final norm.  With a trace every stage
+ * runs on the caller's stream, in this order (no second stream). */
 #define HDF_DRAFT_STAGES_PER_LAYER 8
 typedef struct {
   void* const* events;
