@@ -148,3 +148,84 @@ def test_batch6_block16_96_tokens_fp32():
     cfg = W.DraftConfig("b6f32", m=4, d=256, block=16, n_layers=1, n_heads=2, head_dim=128, ffn=1024,
                         vocab=2048, batch=6, ctx_len=70, dtype="f32")
     run_step(cfg, seed=12, ctx_lens=[70, 1, 5, 64, 33, 17])
+
+
+def _fork_setup():
+    cfg = W.DraftConfig("fork", m=4, d=512, block=16, n_layers=2, n_heads=4, head_dim=128, ffn=1024,
+                        vocab=4096, batch=3, ctx_len=700)
+    lens = [700, 333, 1]
+    inp = W.make_draft_inputs(cfg, 3001)
+    cu = torch.tensor(np.concatenate([[0], np.cumsum(lens)]).astype(np.int32)).cuda()
+    red = W.make_reduce_inputs(sum(lens), cfg.m, cfg.d, cfg.dtype, cfg.wf_std, seed=3001)
+    wc = _to_cuda(inp["weights"])
+    drafter = hdf.Drafter(wc, n_heads=cfg.n_heads, head_dim=cfg.head_dim, rope_theta=cfg.rope_theta,
+                          rope_max_pos=max(lens) + cfg.block, norm_eps=cfg.norm_eps)
+    y = hdf.hdf_gated_reduce(red["H"].cuda(), red["Wf"].cuda(), red["b"].cuda())
+    return cfg, drafter, y, cu, inp["anchor"].cuda(), max(lens)
+
+
+def test_two_stream_step_is_graph_capturable_and_matches_one_stream():
+    """Without a trace the context projection runs on a second stream, forked
+    and joined with events.  Eager, traced (one stream) and captured-then-
+    replayed steps give the same h_out bit for bit (two layers, ragged
+    contexts, so some attention chunks of the short sequences are empty)."""
+    cfg, drafter, y, cu, anchor, max_ctx = _fork_setup()
+    kw = dict(block=cfg.block, max_ctx=max_ctx)
+    h_eager = drafter.hdf_draft_block(y, cu, anchor, **kw)
+    events = [torch.cuda.Event(enable_timing=True) for _ in range(drafter.n_trace_events())]
+    for e in events:  # a torch event creates its CUDA event at its first record
+        e.record()
+    h_traced = drafter.hdf_draft_block(y, cu, anchor, events=events, **kw)
+    torch.cuda.synchronize()
+    assert torch.equal(h_eager.view(torch.int16), h_traced.view(torch.int16))
+
+    s = torch.cuda.Stream()
+    h_graph = torch.zeros_like(h_eager)
+    ws = torch.empty(drafter.workspace_size(anchor.shape[0], cfg.block, y.shape[0], max_ctx), dtype=torch.uint8,
+                     device="cuda")
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g, stream=s):
+        drafter.hdf_draft_block(y, cu, anchor, h_out=h_graph, ws=ws, stream=s, **kw)
+    for _ in range(2):
+        h_graph.zero_()
+        torch.cuda.synchronize()
+        with torch.cuda.stream(s):
+            g.replay()
+        s.synchronize()
+        assert torch.equal(h_eager.view(torch.int16), h_graph.view(torch.int16))
+    assert hdf.device_status() == 0
+
+
+def test_first_call_of_a_thread_under_capture():
+    """The second stream is per host thread and created on first use; a
+    thread whose first call is made under stream capture still captures a
+    step that replays to the eager result."""
+    import threading
+    cfg, drafter, y, cu, anchor, max_ctx = _fork_setup()
+    kw = dict(block=cfg.block, max_ctx=max_ctx)
+    h_eager = drafter.hdf_draft_block(y, cu, anchor, **kw)
+    torch.cuda.synchronize()
+    ws = torch.empty(drafter.workspace_size(anchor.shape[0], cfg.block, y.shape[0], max_ctx), dtype=torch.uint8,
+                     device="cuda")
+    h_graph = torch.zeros_like(h_eager)
+    errors = []
+
+    def worker():
+        try:
+            torch.cuda.set_device(0)
+            s = torch.cuda.Stream()
+            g = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(g, stream=s):
+                drafter.hdf_draft_block(y, cu, anchor, h_out=h_graph, ws=ws, stream=s, **kw)
+            with torch.cuda.stream(s):
+                g.replay()
+            s.synchronize()
+        except Exception as e:  # reported on the main thread
+            errors.append(e)
+
+    t = threading.Thread(target=worker)
+    t.start()
+    t.join()
+    assert not errors, errors
+    assert torch.equal(h_eager.view(torch.int16), h_graph.view(torch.int16))
+    assert hdf.device_status() == 0
