@@ -115,6 +115,31 @@ def gated_reduce(H, Wf, b, *, rms_eps: float = 1e-6, gate_scale: float = 1.0,
     return store(y, out_dtype), alpha
 
 
+def gated_reduce_backward(H, Wf, b, dy, *, rms_eps: float = 1e-6, gate_scale: float = 1.0):
+    """Gradient of Eq. 1 with respect to the reducer's trainable parameters,
+    the gate W_f and b (the 65K parameters of Table 1), for the loss
+    L = sum_t dy_t . y_t, with H held fixed (the frozen target's residual),
+    no per-path norm and no gate override.  The chain rule written out:
+        g_tj   = s * r_t * (W_f vec H_t)_j + b_j        (gate_logits)
+        a_tj   = dL/dalpha_tj = dy_t . H_tj
+        dg_tj  = a_tj * sigmoid(g_tj) * (1 - sigmoid(g_tj))
+        dL/db_j    = sum_t dg_tj
+        dL/dW_f[j] = sum_t dg_tj * s * r_t * vec(H_t)
+    The offset eps_alpha does not enter.  Returns (dW_f [m, m*d], db [m]),
+    fp64."""
+    H = np.asarray(H, dtype=np.float64)
+    N, m, d = H.shape
+    dy = np.asarray(dy, dtype=np.float64).reshape(N, d)
+    x = H.reshape(N, m * d)
+    r = 1.0 / np.sqrt(np.mean(x * x, axis=1) + rms_eps)
+    sg = sigmoid(gate_logits(H, Wf, b, rms_eps, gate_scale))
+    a = np.einsum("nd,njd->nj", dy, H)
+    dg = a * sg * (1.0 - sg)
+    db = dg.sum(axis=0)
+    dWf = (gate_scale * r[:, None] * dg).T @ x
+    return dWf, db
+
+
 def hc_gate_param_count(m: int, d: int) -> int:
     """Trainable parameters of W_f in Eq. 1 (W_f in R^{m x md})."""
     return m * (m * d)

@@ -117,6 +117,54 @@ def test_reduce_scale_invariance():
     np.testing.assert_allclose(y2, 3.5 * y1, rtol=1e-12)
 
 
+def _reduce_loss(H, Wf, b, dy, s, eps):
+    y, _ = O.gated_reduce(H, Wf, b, rms_eps=eps, gate_scale=s, gate_offset=0.25, out_dtype="f64")
+    return float(np.sum(np.asarray(dy) * y))
+
+
+def test_reduce_backward_matches_central_differences():
+    """dL/dW_f and dL/db of L = sum dy . y (Eq. 1, forward oracle in fp64)
+    against central differences of that loss, entry by entry; the offset
+    (0.25 here) must not enter."""
+    N, m, d, s, eps = 5, 3, 8, 1.7, 1e-3
+    H = rng.standard_normal((N, m, d))
+    Wf = rng.standard_normal((m, m * d)) * 0.3
+    b = rng.standard_normal(m) * 0.5
+    dy = rng.standard_normal((N, d))
+    dWf, db = O.gated_reduce_backward(H, Wf, b, dy, rms_eps=eps, gate_scale=s)
+    assert dWf.shape == (m, m * d) and db.shape == (m,)
+    h = 1e-6
+    fd = np.zeros_like(Wf)
+    for j in range(m):
+        for k in range(m * d):
+            Wp, Wm = Wf.copy(), Wf.copy()
+            Wp[j, k] += h
+            Wm[j, k] -= h
+            fd[j, k] = (_reduce_loss(H, Wp, b, dy, s, eps) - _reduce_loss(H, Wm, b, dy, s, eps)) / (2 * h)
+    fdb = np.zeros(m)
+    for j in range(m):
+        bp, bm = b.copy(), b.copy()
+        bp[j] += h
+        bm[j] -= h
+        fdb[j] = (_reduce_loss(H, Wf, bp, dy, s, eps) - _reduce_loss(H, Wf, bm, dy, s, eps)) / (2 * h)
+    scale = max(np.abs(fd).max(), 1.0)
+    assert np.abs(dWf - fd).max() <= 1e-7 * scale
+    assert np.abs(db - fdb).max() <= 1e-7 * max(np.abs(fdb).max(), 1.0)
+
+
+def test_reduce_backward_zero_cotangent_and_bias_is_gate_sum():
+    H = _H(6, 4, 16)
+    Wf = rng.standard_normal((4, 64)) * 0.1
+    b = rng.standard_normal(4)
+    dWf, db = O.gated_reduce_backward(H, Wf, b, np.zeros((6, 16)))
+    assert not dWf.any() and not db.any()
+    # W_f = 0: every gate is sigmoid(b), so dL/db_j = sigmoid'(b_j) * sum_t dy_t . H_tj
+    dy = rng.standard_normal((6, 16))
+    _, db0 = O.gated_reduce_backward(H, np.zeros((4, 64)), b, dy)
+    sg = 1.0 / (1.0 + np.exp(-b))
+    np.testing.assert_allclose(db0, sg * (1 - sg) * np.einsum("nd,njd->j", dy, H), rtol=1e-13)
+
+
 def test_reduce_gates_are_not_a_softmax():
     H = _H(16, 4, 32)
     _, a = O.gated_reduce(H, rng.standard_normal((4, 128)) * 0.1, np.zeros(4), out_dtype="f64")
