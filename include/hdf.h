@@ -130,6 +130,31 @@ HDF_API int hdf_gated_reduce(const void* H, int dtype, int64_t n_tokens, int m, 
 enum { HDF_REDUCE_AUTO = 0, HDF_REDUCE_GENERAL = 1, HDF_REDUCE_CLUSTER = 2, HDF_REDUCE_TILE = 3 };
 HDF_API int hdf_set_reduce_path(int path);
 
+/* Gradient of the reducer (Eq. 1) with respect to its trainable gate
+ * parameters W_f and b (Table 1's 65K parameters), for the loss
+ * L = sum_t dy_t . y_t, with H held fixed (the frozen target's residual),
+ * gate_offset not entering, no per-path norm and no gate override:
+ *   a_tj   = dy_t . H_tj                                 (dL/dalpha_tj)
+ *   dg_tj  = a_tj * sigmoid(g_tj) * (1 - sigmoid(g_tj))  (g_tj as above)
+ *   db_j   = sum_t dg_tj
+ *   dWf[j] = sum_t gate_scale * r_t * dg_tj * vec(H_t)
+ *
+ *   H, Wf, b, rms_eps, gate_scale   as in hdf_gated_reduce
+ *   dy   [n_tokens, d]  dtype   dL/dy (the upstream gradient)
+ *   dWf  [m, m*d]       fp32    out, overwritten (16-byte aligned)
+ *   db   [m]            fp32    out, overwritten
+ *   ws   caller workspace of hdf_gated_reduce_backward_workspace_size()
+ *        bytes (256-byte aligned; 0 bytes when n_tokens == 0)
+ * Every sum runs in a fixed order: the result is bitwise reproducible.
+ * Same m, d and dtype support as hdf_gated_reduce; n_tokens == 0 writes
+ * zero gradients.  The paper trains the reducer but prints no backward; this
+ * is the chain rule of Eq. 1. */
+HDF_API size_t hdf_gated_reduce_backward_workspace_size(int64_t n_tokens, int m, int d, int dtype);
+HDF_API int hdf_gated_reduce_backward(const void* H, int dtype, int64_t n_tokens, int m, int d,
+                              const void* Wf, const float* b, float rms_eps, float gate_scale,
+                              const void* dy, float* dWf, float* db, void* ws, size_t ws_bytes,
+                              hdf_stream_t stream);
+
 /* Generic fc reducer of vanilla DFlash (Sec. 2.2, Table 1 "generic fc"),
  * kept as the comparison path and the fallback the paper names:
  *   y_t = W_fc vec(H_t),   W_fc [d, m*d] dtype, y [n_tokens, d] dtype.

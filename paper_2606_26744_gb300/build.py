@@ -24,7 +24,7 @@ LIB = os.path.join(PKG, "libhdf.so")
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-std=c++17", "-lineinfo", "-Xcompiler", "-fPIC", "--expt-relaxed-constexpr",
          "-Xcompiler", "-fvisibility=hidden"]
-SOURCES = ["hdf_api.cu", "reduce.cu", "gemm.cu", "attention.cu", "small.cu", "kl.cu", "verify.cu"]
+SOURCES = ["hdf_api.cu", "reduce.cu", "reduce_bwd.cu", "gemm.cu", "attention.cu", "small.cu", "kl.cu", "verify.cu"]
 
 
 def nvcc() -> str:

@@ -308,6 +308,85 @@ int hdf_device_status(int reset) {
   return v;
 }
 
+// ---------------------------------------------------- reducer backward
+namespace {
+struct ReduceBwdLayout {
+  size_t u, dg, part, dbpart, total;
+};
+ReduceBwdLayout reduce_bwd_layout(const ReduceBwdPlan& p, long long n, int m, int d) {
+  ReduceBwdLayout L;
+  size_t off = 0;
+  auto take = [&](size_t bytes) {
+    const size_t o = off;
+    off += up256(bytes);
+    return o;
+  };
+  L.u = take((size_t)n * m * 4);
+  L.dg = take((size_t)n * m * 4);
+  L.part = take((size_t)p.splits * m * m * d * 4);
+  L.dbpart = take((size_t)p.splits * m * 4);
+  L.total = n > 0 ? off : 0;
+  return L;
+}
+int check_reduce_bwd(int dtype, int64_t n_tokens, int m, int d) {
+  if (dtype != HDF_BF16 && dtype != HDF_F32) return fail(HDF_ERR_DTYPE, "dtype %d", dtype);
+  if (n_tokens < 0) return fail(HDF_ERR_SHAPE, "n_tokens < 0");
+  if (!(m == 1 || m == 2 || m == 3 || m == 4 || m == 8)) return fail(HDF_ERR_UNSUPPORTED, "m=%d", m);
+  const int vec = dtype == HDF_BF16 ? 8 : 4;
+  if (d <= 0 || d % vec || d > 16384) return fail(HDF_ERR_SHAPE, "d=%d (multiple of %d, <= 16384)", d, vec);
+  return HDF_OK;
+}
+}  // namespace
+
+size_t hdf_gated_reduce_backward_workspace_size(int64_t n_tokens, int m, int d, int dtype) {
+  if (check_reduce_bwd(dtype, n_tokens, m, d)) return 0;
+  return reduce_bwd_layout(reduce_bwd_plan(n_tokens, m, d, dtype, num_sms()), n_tokens, m, d).total;
+}
+
+int hdf_gated_reduce_backward(const void* H, int dtype, int64_t n_tokens, int m, int d, const void* Wf,
+                              const float* b, float rms_eps, float gate_scale, const void* dy, float* dWf,
+                              float* db, void* ws, size_t ws_bytes, hdf_stream_t stream) {
+  g_err.clear();
+  int rc;
+  if ((rc = check_reduce_bwd(dtype, n_tokens, m, d))) return rc;
+  if (!dWf || !db) return fail(HDF_ERR_INVALID_ARG, "dWf and db are required");
+  if (!aligned16(dWf)) return fail(HDF_ERR_ALIGNMENT, "dWf must be 16-byte aligned");
+  const cudaStream_t s = (cudaStream_t)stream;
+  if (n_tokens == 0) {  // empty sums
+    CK(cudaMemsetAsync(dWf, 0, (size_t)m * m * d * 4, s), "memset dWf");
+    CK(cudaMemsetAsync(db, 0, (size_t)m * 4, s), "memset db");
+    return HDF_OK;
+  }
+  if (!H || !Wf || !b || !dy) return fail(HDF_ERR_INVALID_ARG, "H, Wf, b and dy are required");
+  if (!aligned16(H) || !aligned16(Wf) || !aligned16(dy))
+    return fail(HDF_ERR_ALIGNMENT, "H, Wf and dy must be 16-byte aligned");
+  if (!std::isfinite(rms_eps) || !std::isfinite(gate_scale) || rms_eps < 0)
+    return fail(HDF_ERR_INVALID_ARG, "non-finite or negative scalar");
+  const ReduceBwdPlan p = reduce_bwd_plan(n_tokens, m, d, dtype, num_sms());
+  const ReduceBwdLayout L = reduce_bwd_layout(p, n_tokens, m, d);
+  if (!ws || ws_bytes < L.total || (reinterpret_cast<uintptr_t>(ws) & 255))
+    return fail(HDF_ERR_WORKSPACE, "workspace %zu bytes (need %zu, 256-byte aligned)", ws_bytes, L.total);
+  char* W = static_cast<char*>(ws);
+  ReduceBwdArgs a;
+  a.H = H;
+  a.Wf = Wf;
+  a.b = b;
+  a.dy = dy;
+  a.dWf = dWf;
+  a.db = db;
+  a.u = reinterpret_cast<float*>(W + L.u);
+  a.dg = reinterpret_cast<float*>(W + L.dg);
+  a.part = reinterpret_cast<float*>(W + L.part);
+  a.dbpart = reinterpret_cast<float*>(W + L.dbpart);
+  a.n_tokens = n_tokens;
+  a.m = m;
+  a.d = d;
+  a.rms_eps = rms_eps;
+  a.gate_scale = gate_scale;
+  CK(launch_gated_reduce_backward(a, dtype, p, s), "gated_reduce backward launch");
+  return HDF_OK;
+}
+
 // ------------------------------------------------------------- reducer
 static std::atomic<int> g_reduce_path{HDF_REDUCE_AUTO};
 

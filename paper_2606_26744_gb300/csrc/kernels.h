@@ -51,6 +51,29 @@ struct ReduceArgs {
   int* status;
 };
 cudaError_t launch_gated_reduce(const ReduceArgs& a, int dtype, cudaStream_t s);
+
+// Gradient of the reducer with respect to W_f and b (reduce_bwd.cu).
+struct ReduceBwdArgs {
+  const void* H;      // [N, m, d] dtype
+  const void* Wf;     // [m, m*d] dtype
+  const float* b;     // [m]
+  const void* dy;     // [N, d] dtype: dL/dy
+  float* dWf;         // [m, m*d] out
+  float* db;          // [m] out
+  float* u;           // [N, m] workspace: s * r_t * dg_tj
+  float* dg;          // [N, m] workspace: dL/dg_tj
+  float* part;        // [splits, m, m*d] workspace: per-split weight-gradient sums
+  float* dbpart;      // [splits, m] workspace
+  long long n_tokens;
+  int m, d;
+  float rms_eps, gate_scale;
+};
+struct ReduceBwdPlan {
+  int slices = 1, splits = 1, gate_ctas = 1;  // weight-gradient grid (slices x splits), gate-pass CTAs
+  long long tok_per = 0;                       // tokens per split
+};
+ReduceBwdPlan reduce_bwd_plan(long long n_tokens, int m, int d, int dtype, int n_sm);
+cudaError_t launch_gated_reduce_backward(const ReduceBwdArgs& a, int dtype, const ReduceBwdPlan& p, cudaStream_t s);
 // bf16 cluster path: box {64, rb, E/64} of the 3-D view {64 elements, tokens,
 // 128-byte chunks} of H (128-byte swizzle) that the caller encodes; false
 // when the shape or options need the general kernel above.

@@ -66,6 +66,9 @@ _SIGS = {
     "hdf_device_status": (c_int, [c_int]),
     "hdf_gated_reduce": (c_int, [c_vp, c_int, c_i64, c_int, c_int, c_vp, c_vp, c_float, c_float,
                                  c_float, c_vp, c_float, c_vp, c_vp, c_vp, c_vp]),
+    "hdf_gated_reduce_backward_workspace_size": (c_size, [c_i64, c_int, c_int, c_int]),
+    "hdf_gated_reduce_backward": (c_int, [c_vp, c_int, c_i64, c_int, c_int, c_vp, c_vp, c_float, c_float,
+                                          c_vp, c_vp, c_vp, c_vp, c_size, c_vp]),
     "hdf_fc_reduce_workspace_size": (c_size, [c_i64, c_int, c_int, c_int]),
     "hdf_fc_reduce": (c_int, [c_vp, c_int, c_i64, c_int, c_int, c_vp, c_vp, c_vp, c_size, c_vp]),
     "hdf_draft_block_workspace_size": (c_size, [ctypes.POINTER(DraftShape)]),
@@ -148,6 +151,26 @@ REDUCE_PATHS = {"auto": 0, "general": 1, "cluster": 2, "tile": 3}
 def hdf_set_reduce_path(path: str) -> None:
     """Kernel choice of hdf_gated_reduce: "auto", "general" or "cluster"."""
     _check(load().hdf_set_reduce_path(REDUCE_PATHS[path]))
+
+
+def hdf_gated_reduce_backward(H: torch.Tensor, Wf: torch.Tensor, b: torch.Tensor, dy: torch.Tensor, *,
+                              rms_eps: float = 1e-6, gate_scale: float = 1.0, dWf: Optional[torch.Tensor] = None,
+                              db: Optional[torch.Tensor] = None, ws: Optional[torch.Tensor] = None,
+                              stream=None):
+    """Gradient of Eq. 1 with respect to W_f and b for the upstream dy
+    (H fixed): returns (dWf [m, m*d] fp32, db [m] fp32)."""
+    N, m, d = H.shape
+    lib = load()
+    if dWf is None:
+        dWf = torch.empty((m, m * d), dtype=torch.float32, device=H.device)
+    if db is None:
+        db = torch.empty(m, dtype=torch.float32, device=H.device)
+    if ws is None:
+        need = lib.hdf_gated_reduce_backward_workspace_size(N, m, d, _dtype(H))
+        ws = torch.empty(max(need, 1), dtype=torch.uint8, device=H.device)
+    _check(lib.hdf_gated_reduce_backward(_p(H), _dtype(H), N, m, d, _p(Wf), _p(b), rms_eps, gate_scale, _p(dy),
+                                         _p(dWf), _p(db), _p(ws), ws.numel(), _stream(stream)))
+    return dWf, db
 
 
 def hdf_gated_reduce(H: torch.Tensor, Wf: Optional[torch.Tensor], b: Optional[torch.Tensor], *,

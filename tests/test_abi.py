@@ -51,6 +51,32 @@ def test_reduce_host_validation(lib):
     assert b"aligned" in lib.hdf_last_error()
 
 
+def _reduce_bwd(lib, **kw):
+    a = dict(H=16, dtype=1, n=4, m=4, d=64, Wf=16, b=16, dy=16, dWf=16, db=16, ws=256, ws_bytes=1 << 20)
+    a.update(kw)
+    p = lambda v: None if v is None else ctypes.c_void_p(v)
+    return lib.hdf_gated_reduce_backward(p(a["H"]), a["dtype"], a["n"], a["m"], a["d"], p(a["Wf"]), p(a["b"]),
+                                         1e-6, 1.0, p(a["dy"]), p(a["dWf"]), p(a["db"]), p(a["ws"]),
+                                         a["ws_bytes"], None)
+
+
+def test_reduce_backward_host_validation(lib):
+    assert _reduce_bwd(lib, dtype=7) == 3             # HDF_ERR_DTYPE
+    assert _reduce_bwd(lib, m=5) == 7                 # HDF_ERR_UNSUPPORTED
+    assert _reduce_bwd(lib, d=60) == 2                # d % 8 for bf16
+    assert _reduce_bwd(lib, n=-1) == 2
+    assert _reduce_bwd(lib, dWf=None) == 1            # outputs required, even for n = 0
+    assert _reduce_bwd(lib, n=0, db=None) == 1
+    assert _reduce_bwd(lib, dy=None) == 1
+    assert _reduce_bwd(lib, H=24) == 4                # HDF_ERR_ALIGNMENT
+    assert _reduce_bwd(lib, dWf=40) == 4
+    assert _reduce_bwd(lib, ws=None) == 5             # HDF_ERR_WORKSPACE
+    assert _reduce_bwd(lib, ws=300) == 5              # not 256-byte aligned
+    assert lib.hdf_gated_reduce_backward_workspace_size(4, 4, 64, 1) > 0
+    assert lib.hdf_gated_reduce_backward_workspace_size(0, 4, 64, 1) == 0
+    assert lib.hdf_gated_reduce_backward_workspace_size(4, 5, 64, 1) == 0   # unsupported m
+
+
 def test_reduce_path_switch(lib):
     assert lib.hdf_set_reduce_path(3) == 0            # HDF_REDUCE_TILE
     assert lib.hdf_set_reduce_path(4) == 1            # HDF_ERR_INVALID_ARG

@@ -6,7 +6,7 @@ import torch
 import oracle as O
 from paper_2606_26744_gb300 import hdf
 from paper_2606_26744_gb300 import workloads as W
-from _util import TOL_BF16, TOL_F32_REDUCE, exact_fraction, rowwise_rel, to64
+from _util import TOL_BF16, TOL_F32_REDUCE, TOL_F32_REDUCE_BWD, exact_fraction, rowwise_rel, to64
 
 pytestmark = pytest.mark.gpu
 
@@ -129,3 +129,60 @@ def test_reduce_rows_do_not_depend_on_the_call():
     for lo, hi in [(0, 1), (4095, 4101), (17, 60), (4990, 5000)]:
         y_part = hdf.hdf_gated_reduce(H[lo:hi].contiguous(), Wf, b)
         assert torch.equal(y_part.view(torch.int16), y_all[lo:hi].view(torch.int16))
+
+
+# ------------------------------------------------ gradient w.r.t. W_f and b
+def _bwd_inputs(N, m, d, dtype, std, seed):
+    inp = W.make_reduce_inputs(N, m, d, dtype, std, seed=seed)
+    g = torch.Generator().manual_seed(seed + 7)
+    dy = torch.randn((N, d), generator=g).to(inp["H"].dtype)
+    b = torch.randn(m, generator=g) * 0.5
+    return inp["H"], inp["Wf"], b, dy
+
+
+@pytest.mark.parametrize("N,m,d,dtype,std", [
+    (1, 4, 2048, "bf16", 0.1),      # one token
+    (37, 4, 512, "bf16", 0.1),      # ragged token count
+    (2048, 4, 2048, "bf16", 0.1),   # the decode workload's context
+    (300, 2, 256, "bf16", 0.1),
+    (100, 8, 128, "bf16", 0.1),
+    (1001, 3, 384, "bf16", 0.05),
+    (64, 4, 256, "f32", 0.02),      # the tiny workload
+    (5, 1, 64, "f32", 0.3),
+    (3, 4, 7168, "bf16", 0.1),      # the large width
+])
+def test_reduce_backward_parity(N, m, d, dtype, std):
+    H, Wf, b, dy = _bwd_inputs(N, m, d, dtype, std, seed=4000 + N + m)
+    dWf, db = hdf.hdf_gated_reduce_backward(H.cuda(), Wf.cuda(), b.cuda(), dy.cuda(), rms_eps=1e-6, gate_scale=1.0)
+    torch.cuda.synchronize()
+    assert hdf.device_status() == 0
+    dWf_ref, db_ref = O.gated_reduce_backward(to64(H), to64(Wf), to64(b), to64(dy), rms_eps=1e-6, gate_scale=1.0)
+    assert dWf.shape == (m, m * d) and db.shape == (m,)
+    err_w = rowwise_rel(to64(dWf), dWf_ref)
+    err_b = np.abs(to64(db) - db_ref).max() / max(np.abs(db_ref).max(), 1e-30)
+    assert err_w <= TOL_F32_REDUCE_BWD, f"dW_f row-normwise error {err_w}"
+    assert err_b <= TOL_F32_REDUCE_BWD, f"db error {err_b}"
+
+
+def test_reduce_backward_gate_scale_and_reproducible():
+    H, Wf, b, dy = _bwd_inputs(513, 4, 1024, "bf16", 0.05, seed=4100)
+    args = (H.cuda(), Wf.cuda(), b.cuda(), dy.cuda())
+    dW1, db1 = hdf.hdf_gated_reduce_backward(*args, rms_eps=1e-3, gate_scale=0.7)
+    dW2, db2 = hdf.hdf_gated_reduce_backward(*args, rms_eps=1e-3, gate_scale=0.7)
+    torch.cuda.synchronize()
+    assert torch.equal(dW1, dW2) and torch.equal(db1, db2)   # fixed summation order
+    dWf_ref, db_ref = O.gated_reduce_backward(to64(H), to64(Wf), to64(b), to64(dy), rms_eps=1e-3, gate_scale=0.7)
+    assert rowwise_rel(to64(dW1), dWf_ref) <= TOL_F32_REDUCE_BWD
+    assert np.abs(to64(db1) - db_ref).max() <= TOL_F32_REDUCE_BWD * np.abs(db_ref).max()
+
+
+def test_reduce_backward_no_tokens_gives_zero_gradients():
+    m, d = 4, 256
+    dWf = torch.full((m, m * d), 7.0, device="cuda")
+    db = torch.full((m,), 7.0, device="cuda")
+    H = torch.empty((0, m, d), dtype=torch.bfloat16, device="cuda")
+    hdf.hdf_gated_reduce_backward(H, torch.zeros((m, m * d), dtype=torch.bfloat16, device="cuda"),
+                                  torch.zeros(m, device="cuda"), torch.empty((0, d), dtype=torch.bfloat16,
+                                                                             device="cuda"), dWf=dWf, db=db)
+    torch.cuda.synchronize()
+    assert not dWf.any() and not db.any()
