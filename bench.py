@@ -326,6 +326,31 @@ def run_ours(args, rank, world, local_rank):
           "gbs": round(2 * kl_rows_n * V * 4 / kl_us / 1e3, 1), "launches": 2}
     del ls_t, ls_s
 
+    # -------------------- reducer gradient w.r.t. W_f and b (training-time)
+    # over this workload's context residual, upstream dy ~ N(0, 1); timed
+    # alone like the KL target.  HBM-bound: H twice, dy once, W_f once.
+    n_tok = H.shape[0]
+    dy_r = torch.randn((n_tok, cfg.d), device=dev, generator=gk).to(H.dtype)
+    dwf = torch.empty((cfg.m, cfg.m * cfg.d), dtype=torch.float32, device=dev)
+    dbv = torch.empty(cfg.m, dtype=torch.float32, device=dev)
+    rbws = torch.empty(max(1, hdf.load().hdf_gated_reduce_backward_workspace_size(n_tok, cfg.m, cfg.d,
+                                                                                  hdf._dtype(H))),
+                       dtype=torch.uint8, device=dev)
+    for _ in range(3):
+        hdf.hdf_gated_reduce_backward(H, Wf, b, dy_r, dWf=dwf, db=dbv, ws=rbws, stream=stream)
+    stream.synchronize()
+    k0.record(stream)
+    for _ in range(20):
+        hdf.hdf_gated_reduce_backward(H, Wf, b, dy_r, dWf=dwf, db=dbv, ws=rbws, stream=stream)
+    k1.record(stream)
+    stream.synchronize()
+    rb_us = k0.elapsed_time(k1) / 20 * 1000
+    es = H.element_size()
+    rb_bytes = 2 * H.numel() * es + dy_r.numel() * es + Wf.numel() * es + cfg.m * cfg.m * cfg.d * 4
+    reduce_bwd = {"tokens": n_tok, "us": round(rb_us, 2), "bytes": int(rb_bytes),
+                  "gbs": round(rb_bytes / rb_us / 1e3, 1), "launches": 3}
+    del dy_r, rbws
+
     # ------------------------------------ T = 1 verification (speculative sampling)
     # target / draft probabilities of every block slot, drafts sampled from q,
     # uniforms as 32-bit integers; timed alone like the KL target
@@ -421,6 +446,7 @@ def run_ours(args, rank, world, local_rank):
         torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
         ms, e2e_ms = float(t[0]), float(t[1])
     return dict(cfg=cfg, ms=ms, ms_staged=ms_staged, e2e_ms=e2e_ms, dur=dur, clk=clk, kl=kl, verify_t1=verify_t1,
+                reduce_bwd=reduce_bwd,
                 warm=warm, pct=pct, accept_sweep=accept_sweep, batch=batch, n_ctx=n_ctx, lens=lens,
                 h2d=h2d, d2h=d2h, acc_mean=acc_mean, tok=tok, y=y, inputs=inp, tgt=tgt)
 
@@ -823,6 +849,7 @@ def main():
             "roofline": rf,
             "reducer": {"gbs": red.get("gbs"), "frac_hbm": red.get("frac"), "us": red["us"]},
             "kl_target": dict(res["kl"], frac_hbm=round(res["kl"]["gbs"] / pk["hbm_gbs"], 3)),
+            "reducer_backward": dict(res["reduce_bwd"], frac_hbm=round(res["reduce_bwd"]["gbs"] / pk["hbm_gbs"], 3)),
             "verify_t1": res["verify_t1"],
             "accept_sweep": dict(res["accept_sweep"], frac_hbm=round(res["accept_sweep"]["gbs"] / pk["hbm_gbs"], 3)),
             "warm_step": res["warm"],
