@@ -454,7 +454,8 @@ cudaError_t launch_hd(const AttnArgs& a, const AttnTmaps* tm, cudaStream_t s) {
 size_t attention_smem_bytes(int head_dim) { return head_dim == 64 ? attn_smem<64>() : attn_smem<128>(); }
 
 // Clusters of `cluster` attention CTAs resident at once (occupancy API), or
-// -1 if it cannot be asked.  Cached per head_dim and cluster size.
+// -1 if it cannot be asked (or answers none).  Cached per head_dim and
+// cluster size (0: not asked yet).
 int attention_max_clusters(int head_dim, int cluster) {
   if ((head_dim != 64 && head_dim != 128) || cluster < 1 || cluster > 8) return -1;
   static std::atomic<int> cache[2][9];
@@ -479,6 +480,7 @@ int attention_max_clusters(int head_dim, int cluster) {
     if (cudaOccupancyMaxActiveClusters(&n, k, &cfg) != cudaSuccess) n = -1;
   }
   cudaGetLastError();
+  if (n <= 0) n = -1;  // unknown or none: the caller falls back to SMs / cluster size
   cache[hi][cluster].store(n);
   return n;
 }
