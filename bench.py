@@ -650,14 +650,26 @@ def oracle_step_fn(cfg, inp, tgt=None):
     anchor = inp["anchor"].tolist()
     tgt_np = None if tgt is None else tgt.cpu().numpy()
 
-    def run():
+    def run(times=None):
+        """One step; with a dict, adds each stage's seconds to times[stage]."""
+        clock = [time.perf_counter()]
+
+        def lap(name):
+            if times is not None:
+                now = time.perf_counter()
+                times[name] = times.get(name, 0.0) + now - clock[0]
+                clock[0] = now
         y, _ = O.gated_reduce(H64, Wf64, b64, out_dtype=cfg.dtype)
+        lap("gated_reduce")
         h = O.draft_block(w64, y, cu, anchor, block=cfg.block, n_heads=cfg.n_heads, head_dim=cfg.head_dim,
                           rope_theta=cfg.rope_theta, norm_eps=cfg.norm_eps, act_dtype=cfg.dtype)
+        lap("draft_block")
         lm = O.lm_head(h, w64["lm_head"], logsoftmax=cfg.logsoftmax)
+        lap("lm_head")
         drafts = O.draft_tokens(lm["tok"], cfg.batch, cfg.block)
         if tgt_np is not None:
             O.accept_len(drafts, tgt_np)
+        lap("accept")
         return lm
     return run
 
@@ -748,15 +760,17 @@ def host_cores():
 def cpu_baseline(cfg, inp, tgt, budget_s=15.0):
     run = oracle_step_fn(cfg, inp, tgt)
     n = 0
+    times = {}
     t0 = time.perf_counter()
     while True:
-        run()
+        run(times)
         n += 1
         if time.perf_counter() - t0 > budget_s or n >= 20:
             break
     el = time.perf_counter() - t0
     return {"value": round(n * cfg.batch / el, 4), "unit": METRIC, "cores": host_cores(), "kind": "oracle",
-            "sample": f"{n} full {cfg.name} steps (batch {cfg.batch}) of the fp64 numpy oracle, {el:.1f} s"}
+            "sample": f"{n} full {cfg.name} steps (batch {cfg.batch}) of the fp64 numpy oracle, {el:.1f} s",
+            "stages_ms": {k: round(v / n * 1e3, 3) for k, v in times.items()}}
 
 
 def run_reference(args):
