@@ -206,7 +206,7 @@ def context_kv(c, wk, wv, pos, *, n_heads: int, head_dim: int, theta: float,
     for already-normalised context rows c [n, d] at positions pos [n]."""
     n = c.shape[0]
     K = (_f64(c) @ _f64(wk).T).reshape(n, n_heads, head_dim)
-    K = store(rope(K, pos, theta), act_dtype).reshape(n, -1)
+    K = store(rope(K, pos, theta), act_dtype).reshape(n, n_heads * head_dim)
     V = store(_f64(c) @ _f64(wv).T, act_dtype)
     return K, V
 

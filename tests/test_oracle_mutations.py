@@ -1,0 +1,144 @@
+"""Planted mistakes in the oracle must each turn a pin red.
+
+Each entry below is a plausible slip in ``oracle/hdf_oracle.py`` (a swapped
+operand, a dropped term or weight, a rotation in the wrong place, an index
+off by one).  The test plants it in a copy of the oracle source, on the CPU,
+loads ``tests/test_oracle_pins.py`` against that copy and runs every pin:
+at least one must fail.  The unmutated source must pass them all, so the
+harness itself is checked too.  Nothing here touches the CUDA library."""
+import importlib.util
+import os
+import sys
+import types
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+ORACLE_SRC = os.path.join(ROOT, "oracle", "hdf_oracle.py")
+PINS = os.path.join(ROOT, "tests", "test_oracle_pins.py")
+
+# name -> (text in the oracle source, replacement)
+MUTATIONS = {
+    # ---------------------------------------------------------- drafter block
+    "swiglu gate and up projections swapped": (
+        'act = store(silu(x2 @ _f64(lw["wg"]).T) * (x2 @ _f64(lw["wu"]).T), A)',
+        'act = store(silu(x2 @ _f64(lw["wu"]).T) * (x2 @ _f64(lw["wg"]).T), A)'),
+    "rotary embedding applied to the context values": (
+        "V = store(_f64(c) @ _f64(wv).T, act_dtype)",
+        "V = store(rope((_f64(c) @ _f64(wv).T).reshape(n, n_heads, head_dim), pos, theta),"
+        " act_dtype).reshape(n, n_heads * head_dim)"),
+    "rotary embedding dropped from the context keys": (
+        "K = store(rope(K, pos, theta), act_dtype).reshape(n, n_heads * head_dim)",
+        "K = store(K, act_dtype).reshape(n, n_heads * head_dim)"),
+    "block slot k placed at T + 1 + k": (
+        "pos_blk = np.concatenate([lens[i] + np.arange(B) for i in range(batch)])",
+        "pos_blk = np.concatenate([lens[i] + 1 + np.arange(B) for i in range(batch)])"),
+    "context row t placed at t + 1": (
+        "pos_ctx = np.concatenate([np.arange(t) for t in lens]) if cu[-1] else np.zeros(0)",
+        "pos_ctx = np.concatenate([np.arange(t) + 1 for t in lens]) if cu[-1] else np.zeros(0)"),
+    "context norm weight dropped": (
+        'c = store(rmsnorm(ctx, W["ctx_norm"], norm_eps), A)',
+        "c = store(rmsnorm(ctx, np.ones(d), norm_eps), A)"),
+    "rotary embedding applied to the block values": (
+        'Vb = store(x @ _f64(lw["wv"]).T, A)',
+        'Vb = store(rope((x @ _f64(lw["wv"]).T).reshape(M, n_heads, head_dim), pos_blk, rope_theta),'
+        " A).reshape(M, d)"),
+    "block queries not rotated": (
+        'Q = store(rope((x @ _f64(lw["wq"]).T).reshape(M, n_heads, head_dim),\n'
+        "                       pos_blk, rope_theta), A).reshape(M, d)",
+        'Q = store((x @ _f64(lw["wq"]).T), A).reshape(M, d)'),
+    "block keys not rotated": (
+        'Kb = store(rope((x @ _f64(lw["wk"]).T).reshape(M, n_heads, head_dim),\n'
+        "                        pos_blk, rope_theta), A).reshape(M, d)",
+        'Kb = store((x @ _f64(lw["wk"]).T), A).reshape(M, d)'),
+    "attention keys and values swapped": (
+        "O[rows, cols] = softmax_attention(Q[rows, cols], k_all, v_all)",
+        "O[rows, cols] = softmax_attention(Q[rows, cols], v_all, k_all)"),
+    "attention 1/sqrt(head_dim) scale dropped": (
+        "s = (q @ k.T) / math.sqrt(q.shape[-1])",
+        "s = q @ k.T"),
+    "attention residual dropped": (
+        'h = store(h + O @ _f64(lw["wo"]).T, "f32")',
+        'h = store(O @ _f64(lw["wo"]).T, "f32")'),
+    "MLP residual dropped": (
+        'h = store(h + act @ _f64(lw["wd"]).T, "f32")',
+        'h = store(act @ _f64(lw["wd"]).T, "f32")'),
+    "MLP norm takes the attention norm weight": (
+        'x2 = store(rmsnorm(h, lw["mlp_norm"], norm_eps), A)',
+        'x2 = store(rmsnorm(h, lw["attn_norm"], norm_eps), A)'),
+    "final norm dropped": (
+        'return store(rmsnorm(h, W["final_norm"], norm_eps), A)',
+        "return store(h, A)"),
+    "anchor slot gets the mask vector": (
+        'h[i * B] = _f64(W["embed"])[int(anchor[i])]',
+        'h[i * B] = _f64(W["mask_vec"])'),
+    # ---------------------------------------------------------------- reducer
+    "gate computed from the per-path-normed residual": (
+        "        alpha = sigmoid(gate_logits(H, Wf, b, rms_eps, gate_scale)) + gate_offset\n",
+        "        Hg = H if path_norm_w is None else (H / np.sqrt(np.mean(H * H, axis=2, keepdims=True)"
+        " + path_norm_eps) * np.asarray(path_norm_w, np.float64)[None])\n"
+        "        alpha = sigmoid(gate_logits(Hg, Wf, b, rms_eps, gate_scale)) + gate_offset\n"),
+    "vec() taken element-major": (
+        "x = H.reshape(N, m * d)                              # vec(H_t), path-major",
+        "x = H.transpose(0, 2, 1).reshape(N, m * d)"),
+    "gate bias dropped": (
+        "return gate_scale * (x_tilde @ np.asarray(Wf, np.float64).T) + np.asarray(b, np.float64)[None, :]",
+        "return gate_scale * (x_tilde @ np.asarray(Wf, np.float64).T)"),
+    # ---------------------------------------------------------------- LM head
+    "log-softmax temperature ignored": (
+        "s = z * inv_temp",
+        "s = z"),
+    "argmax takes the last index on ties": (
+        "tok = np.argmax(z, axis=1)          # numpy returns the first maximiser",
+        "tok = z.shape[1] - 1 - np.argmax(z[:, ::-1], axis=1)"),
+    # --------------------------------------------------------------------- KL
+    "KL direction reversed": (
+        "return float(t_kd * t_kd / P * np.sum(p * (lp - lq)))",
+        "return float(t_kd * t_kd / P * np.sum(np.exp(lq) * (lq - lp)))"),
+    "KL temperature-squared factor dropped": (
+        "return float(t_kd * t_kd / P * np.sum(p * (lp - lq)))",
+        "return float(1.0 / P * np.sum(p * (lp - lq)))"),
+}
+
+
+def _load_oracle(src: str) -> types.ModuleType:
+    mod = types.ModuleType("oracle")
+    mod.__file__ = ORACLE_SRC
+    exec(compile(src, ORACLE_SRC, "exec"), mod.__dict__)
+    return mod
+
+
+def _red_pins(oracle_mod: types.ModuleType):
+    """Names of the pins that fail against ``oracle_mod``."""
+    saved = sys.modules.get("oracle")
+    sys.modules["oracle"] = oracle_mod
+    try:
+        spec = importlib.util.spec_from_file_location("_pins_against_planted_oracle", PINS)
+        pins = importlib.util.module_from_spec(spec)
+        spec.loader.exec_module(pins)
+    finally:
+        if saved is not None:
+            sys.modules["oracle"] = saved
+        else:
+            del sys.modules["oracle"]
+    red = []
+    for name in sorted(n for n in dir(pins) if n.startswith("test_")):
+        try:
+            getattr(pins, name)()
+        except Exception:  # an assertion, or the slip breaking a shape
+            red.append(name)
+    return red
+
+
+def test_unplanted_oracle_passes_every_pin():
+    assert _red_pins(_load_oracle(open(ORACLE_SRC).read())) == []
+
+
+@pytest.mark.parametrize("name", sorted(MUTATIONS))
+def test_planted_mistake_turns_a_pin_red(name):
+    old, new = MUTATIONS[name]
+    src = open(ORACLE_SRC).read()
+    assert src.count(old) == 1, f"the text to plant '{name}' in is not in the oracle once"
+    red = _red_pins(_load_oracle(src.replace(old, new)))
+    assert red, f"no pin fails when the oracle has: {name}"
+    print(f"{name}: caught by {', '.join(red)}")

@@ -487,3 +487,151 @@ def test_accept_sample_inverse_cdf_boundaries():
     for r, want in [(0, 0), (2 ** 30 - 1, 0), (2 ** 30, 1), (2 ** 31, 2), (2 ** 32 - 1, 3)]:
         _, nxt = O.accept_sample(p, q, draft, u, np.array([r], dtype=np.uint64))
         assert nxt[0] == want, (r, nxt[0])
+
+
+# --------------------------------------------------------------------------
+# drafter wiring pins: each fixes one place where the drafter reading could
+# be slipped (MLP wiring, where RoPE goes, block and context positions, the
+# context norm, the gate under the per-path norm, the log-softmax temperature)
+# with a closed form of a special case
+# --------------------------------------------------------------------------
+
+def _const_block_weights(d, F, gamma_mlp, seed=3):
+    """Drafter weights whose block input rows are all 0.5 (so RMSNorm(h) is
+    the norm weight itself at eps 0) and whose attention adds nothing (W_o = 0)."""
+    W = _tiny_weights(d=d, F=F, seed=seed)
+    W["embed"] = np.full_like(W["embed"], 0.5)
+    W["mask_vec"] = np.full_like(W["mask_vec"], 0.5)
+    lw = W["layers"][0]
+    lw["wo"][:] = 0.0
+    lw["mlp_norm"] = gamma_mlp
+    return W
+
+
+def test_swiglu_gate_closes_the_mlp_when_the_gate_logit_is_very_negative():
+    # x2 = mlp_norm = gamma for every block row (h0 = 0.5 * ones, eps 0).  Gate
+    # rows with gamma . W_g[f] = -60 give silu(-60) ~ -5e-25: the MLP adds
+    # nothing and the output is RMSNorm_final(0.5 * ones) = final_norm exactly.
+    # With the gate and up projections swapped the MLP adds silu(u) * (-60).
+    d, F = 16, 8
+    r = np.random.default_rng(71)
+    gamma = 1.0 + 0.2 * r.random(d)
+    W = _const_block_weights(d, F, gamma)
+    lw = W["layers"][0]
+    lw["wg"] = np.tile(-60.0 * gamma / np.dot(gamma, gamma), (F, 1))
+    lw["wu"] = r.standard_normal((F, d))
+    lw["wd"] = r.standard_normal((d, F))
+    out = O.draft_block(W, r.standard_normal((5, d)), [0, 5], [3], block=4, n_heads=2, head_dim=8,
+                        rope_theta=1e4, norm_eps=0.0, act_dtype="f64")
+    np.testing.assert_allclose(out, np.broadcast_to(W["final_norm"], out.shape), rtol=0, atol=1e-12)
+
+
+def test_swiglu_is_linear_in_the_up_projection_when_the_gate_saturates_high():
+    # gamma . W_g[f] = 40: silu(40) = 40 to 1e-16, so act = 40 * (W_u gamma) and
+    # h = 0.5 * ones + 40 * W_d W_u gamma, out = h / rms(h) * final_norm.
+    d, F = 16, 8
+    r = np.random.default_rng(72)
+    gamma = 1.0 + 0.2 * r.random(d)
+    W = _const_block_weights(d, F, gamma)
+    lw = W["layers"][0]
+    lw["wg"] = np.tile(40.0 * gamma / np.dot(gamma, gamma), (F, 1))
+    lw["wu"] = r.standard_normal((F, d)) * 0.1
+    lw["wd"] = r.standard_normal((d, F)) * 0.1
+    out = O.draft_block(W, r.standard_normal((5, d)), [0, 5], [3], block=4, n_heads=2, head_dim=8,
+                        rope_theta=1e4, norm_eps=0.0, act_dtype="f64")
+    h = 0.5 + 40.0 * (lw["wd"] @ (lw["wu"] @ gamma))
+    expect = h / math.sqrt(np.mean(h * h)) * W["final_norm"]
+    # the block residual h is stored in fp32 (the precision contract), so
+    # agreement is to fp32 rounding of h
+    np.testing.assert_allclose(out, np.broadcast_to(expect, out.shape), rtol=4e-7, atol=0)
+
+
+def _rot(pairs, angle):
+    """Rotate 2-vectors (last axis) by angle, as complex multiplication."""
+    z = (pairs[..., 0] + 1j * pairs[..., 1]) * np.exp(1j * np.asarray(angle, np.float64))
+    return np.stack([z.real, z.imag], axis=-1)
+
+
+def test_context_projection_rotates_keys_and_not_values():
+    # head_dim 2 (frequency theta^0 = 1: the angle is the position), identity
+    # projections: K_c[t] is c_t turned by t radians per head, V_c[t] is c_t.
+    c = rng.standard_normal((3, 4))
+    pos = np.array([0.0, 3.0, 7.0])
+    K, V = O.context_kv(c, np.eye(4), np.eye(4), pos, n_heads=2, head_dim=2, theta=10000.0, act_dtype="f64")
+    expect_k = _rot(c.reshape(3, 2, 2), pos[:, None]).reshape(3, 4)
+    np.testing.assert_allclose(K, expect_k, rtol=1e-14, atol=1e-15)
+    np.testing.assert_array_equal(V, c)
+
+
+def test_block_attention_positions_rotary_and_context_norm_closed_form():
+    """Identity Q/K/V projections, head_dim 2: per head the score of a block
+    query (slot k, position T_i + k) and a key at position p is
+    Re(z_q e^{i(T_i+k)} conj(z_k e^{ip})) / sqrt(2) for the complex pairs z of
+    the normed rows, and the values are the unrotated pairs.  The normed
+    context rows are y / rms(y) * ctx_norm, the normed block rows
+    h0 / rms(h0) * attn_norm.  Checks block slot k at exactly T_i + k, context
+    row t at t, RoPE on Q and both kinds of keys, none on either kind of
+    values, the context norm weight and the 1/sqrt(hd) scale."""
+    d, B, hd = 4, 3, 2
+    W = _tiny_weights(d=d, F=8, V=6, seed=9)
+    lw = W["layers"][0]
+    for k in ("wq", "wk", "wv"):
+        lw[k] = np.eye(d)
+    lw["wo"][:] = 0.0
+    ctx = rng.standard_normal((5, d))
+    cu, anchor = [0, 3, 5], [4, 1]
+    inter = {}
+    O.draft_block(W, ctx, cu, anchor, block=B, n_heads=2, head_dim=hd, rope_theta=1e4, norm_eps=0.0,
+                  act_dtype="f64", intermediates=inter)
+    got = inter["layers"][0]["O"]
+
+    def normed(rows, w):
+        return rows / np.sqrt(np.mean(rows * rows, axis=1, keepdims=True)) * w
+    c = normed(ctx, W["ctx_norm"])
+    for i in range(2):
+        T = cu[i + 1] - cu[i]
+        # the block residual starts as the fp32 copy of its input rows
+        h0 = np.stack([W["embed"][anchor[i]]] + [W["mask_vec"]] * (B - 1)).astype(np.float32).astype(np.float64)
+        x = normed(h0, W["layers"][0]["attn_norm"])
+        keys = np.concatenate([c[cu[i]:cu[i + 1]], x])            # [T + B, d], unrotated
+        kpos = np.concatenate([np.arange(T), T + np.arange(B)])
+        for hh in range(2):
+            kz = keys[:, 2 * hh] + 1j * keys[:, 2 * hh + 1]
+            for k in range(B):
+                qz = (x[k, 2 * hh] + 1j * x[k, 2 * hh + 1]) * np.exp(1j * (T + k))
+                s = np.real(qz * np.conj(kz * np.exp(1j * kpos))) / math.sqrt(hd)
+                p = np.exp(s - s.max())
+                p /= p.sum()
+                np.testing.assert_allclose(got[i * B + k, 2 * hh:2 * hh + 2], p @ keys[:, 2 * hh:2 * hh + 2],
+                                           rtol=1e-12, atol=1e-14)
+
+
+def test_per_path_norm_leaves_the_gate_on_the_raw_residual():
+    # m = 2, d = 4, path 0 = 1 and path 1 = 3 everywhere: mean(H^2) = 5, so
+    # r = 1/sqrt(5) (eps 0).  W_f row 0 reads H[1][0] (+1), row 1 reads
+    # H[0][2] (-2): gates sigmoid(3/sqrt5 + b0), sigmoid(-2/sqrt5 + b1) whether
+    # or not the drafter-side per-path norm is on; with it on each normed path
+    # is its weight gamma_j, so y = alpha_0 gamma_0 + alpha_1 gamma_1.
+    m, d = 2, 4
+    H = np.concatenate([np.ones((1, 1, d)), 3.0 * np.ones((1, 1, d))], axis=1)
+    Wf = np.zeros((m, m * d))
+    Wf[0, 1 * d + 0] = 1.0
+    Wf[1, 0 * d + 2] = -2.0
+    b = np.array([0.1, -0.2])
+    gamma = np.array([[0.5, 1.5, -1.0, 2.0], [1.0, -0.5, 0.25, 3.0]])
+    y, a = O.gated_reduce(H, Wf, b, rms_eps=0.0, path_norm_w=gamma, path_norm_eps=0.0, out_dtype="f64")
+    s5 = math.sqrt(5.0)
+    expect_a = 1.0 / (1.0 + np.exp(-np.array([3.0 / s5 + 0.1, -2.0 / s5 - 0.2])))
+    np.testing.assert_allclose(a[0], expect_a, rtol=1e-14)
+    np.testing.assert_allclose(y[0], expect_a[0] * gamma[0] + expect_a[1] * gamma[1], rtol=1e-14)
+
+
+def test_logsoftmax_two_class_closed_form_at_temperature():
+    # z = (2, 0.5): at inv_temp t the two classes differ by 1.5 t
+    h = np.array([[1.0]])
+    W = np.array([[2.0], [0.5]])
+    for t in (0.5, 3.0):
+        res = O.lm_head(h, W, inv_temp=t, logsoftmax=True)
+        np.testing.assert_allclose(res["logsoftmax"][0], [-math.log1p(math.exp(-1.5 * t)),
+                                                          -math.log1p(math.exp(1.5 * t))], rtol=1e-13)
+        assert res["tok"][0] == 0 and res["zmax"][0] == 2.0
