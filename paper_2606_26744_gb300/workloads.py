@@ -98,12 +98,17 @@ def _gen(seed: int, device) -> torch.Generator:
     return g
 
 
-def _randn(shape, std, dtype, g, device, chunk_rows: int = 1 << 14):
+def _randn(shape, std, dtype, g, device, chunk_elems: Optional[int] = None):
     """N(0, std^2) drawn in fp32 then cast; large tensors are drawn in row
-    chunks so the fp32 staging buffer stays small (same values on one device
-    for a given seed)."""
+    chunks of about chunk_elems values so the fp32 staging buffer stays small
+    (same values on one device for a given seed).  Host chunks are kept small
+    enough to be reused by the allocator; device chunks are large, so few
+    kernels draw them."""
+    if chunk_elems is None:
+        chunk_elems = 1 << 22 if torch.device(device).type == "cpu" else 1 << 27
     out = torch.empty(shape, dtype=dtype, device=device)
     flat = out.view(shape[0], -1)
+    chunk_rows = max(1, chunk_elems // max(1, flat.shape[1]))
     for r0 in range(0, shape[0], chunk_rows):
         r1 = min(shape[0], r0 + chunk_rows)
         t = torch.randn((r1 - r0, flat.shape[1]), generator=g, device=device,
