@@ -113,22 +113,33 @@ HDF_API int hdf_gated_reduce(const void* H, int dtype, int64_t n_tokens, int m, 
                      const float* alpha_override,
                      void* y, float* alpha_out, hdf_stream_t stream);
 
-/* Kernel choice of hdf_gated_reduce; all compute Eq. 1 and agree within
- * fp32 summation order.  HDF_REDUCE_GENERAL: one CTA streams whole tokens and
- * re-reads them from L2 for the weighted sum (every dtype and option).
- * HDF_REDUCE_CLUSTER: 8-CTA clusters split d, keep W_f slices in shared
- * memory and exchange the gate partials of small token batches over
- * distributed shared memory.  HDF_REDUCE_TILE: 8-CTA clusters split d over
- * tiles of 32 tokens, gate dots on the tensor cores, one exchange per tile.
+/* hdf_gated_reduce with an explicit kernel choice for this call only (no
+ * state is kept between calls, so no call can change which kernel, and so
+ * which fp32 summation order, another call uses).  The paper has no
+ * counterpart: it is a tuning and test hook.  All kernels compute Eq. 1 and
+ * agree within fp32 summation order.
+ *   HDF_REDUCE_AUTO     what hdf_gated_reduce runs: the tile kernel for m = 4,
+ *                       the general kernel otherwise, whatever n_tokens is,
+ *                       so that a token's y does not depend on how many
+ *                       tokens share the call
+ *   HDF_REDUCE_GENERAL  one CTA streams whole tokens and re-reads them from L2
+ *                       for the weighted sum (every dtype and option)
+ *   HDF_REDUCE_CLUSTER  8-CTA clusters split d, keep W_f slices in shared
+ *                       memory and exchange the gate partials of small token
+ *                       batches over distributed shared memory
+ *   HDF_REDUCE_TILE     clusters split d over tiles of 32 tokens, gate dots on
+ *                       the tensor cores, one exchange per tile
  * CLUSTER and TILE need bf16, m in {1,2,4}, d % 512 == 0 and neither
  * alpha_override nor path_norm_w (TILE also a whole number of its 4 box
  * phases per tile, always so for m = 4); the general kernel runs otherwise.
- * HDF_REDUCE_AUTO (the default) takes the tile kernel for m = 4 and the
- * general kernel otherwise, whatever n_tokens is, so that a token's y does not
- * depend on how many tokens share the call.  Process-wide; returns HDF_ERR_INVALID_ARG for another value.  The
- * paper has no counterpart: it is a tuning and test hook. */
+ * Another kernel value returns HDF_ERR_INVALID_ARG. */
 enum { HDF_REDUCE_AUTO = 0, HDF_REDUCE_GENERAL = 1, HDF_REDUCE_CLUSTER = 2, HDF_REDUCE_TILE = 3 };
-HDF_API int hdf_set_reduce_path(int path);
+HDF_API int hdf_gated_reduce_kernel(int kernel, const void* H, int dtype, int64_t n_tokens, int m, int d,
+                     const void* Wf, const float* b,
+                     float rms_eps, float gate_scale, float gate_offset,
+                     const void* path_norm_w, float path_norm_eps,
+                     const float* alpha_override,
+                     void* y, float* alpha_out, hdf_stream_t stream);
 
 /* Gradient of the reducer (Eq. 1) with respect to its trainable gate
  * parameters W_f and b (Table 1's 65K parameters), for the loss

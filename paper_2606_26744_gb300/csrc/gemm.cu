@@ -426,6 +426,7 @@ __global__ void __launch_bounds__(128, 1) gemm_kernel(const __grid_constant__ Ge
   __shared__ __align__(8) uint64_t acc_bar;
   __shared__ uint32_t tmem_slot;
   __shared__ volatile int abort_flag;
+  __shared__ int cluster_abort;  // split-K, rank 0: some rank of the cluster gave up a wait
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   pdl_launch_dependents();
@@ -579,7 +580,14 @@ __global__ void __launch_bounds__(128, 1) gemm_kernel(const __grid_constant__ Ge
     } else {
       for (int c = 0; c < BN; ++c) part[tid * BN + c] = 0.f;
     }
-    cluster_sync_all();  // every rank's partial tile is visible to the cluster
+    cluster_sync_all();  // every rank's partial tile and abort flag are visible to the cluster
+    // a rank that gave up a wait left zeros as its partial: rank 0 then skips
+    // the store (the device status word already records the failure)
+    if (cluster_rank() == 0 && tid == 0) {
+      int any = 0;
+      for (int u = 0; u < g.k_splits; ++u) any |= ld_dsmem_s32(map_rank(smem_u32((const void*)&abort_flag), (uint32_t)u));
+      cluster_abort = any;
+    }
     // Every rank sums a slice of the tile's rows over all ranks (one float4
     // column per thread and round, every source in flight at once, summed in
     // rank order) and writes the result over rank 0's partial of that slice:
@@ -614,7 +622,7 @@ __global__ void __launch_bounds__(128, 1) gemm_kernel(const __grid_constant__ Ge
       }
     }
     cluster_sync_all();  // rank 0's tile holds the sums; no rank reads another's memory any more
-    if (cluster_rank() == 0 && !aborted) {
+    if (cluster_rank() == 0 && !cluster_abort) {
       const float* red = part;
 #pragma unroll 1
       for (int c0 = 0; c0 < BN; c0 += 16) {
@@ -637,6 +645,200 @@ __global__ void __launch_bounds__(128, 1) gemm_kernel(const __grid_constant__ Ge
     tc_fence_after();
     tmem_dealloc(tmem, TMEM_COLS);
   }
+}
+
+// ---------------------------------------------------------------------------
+// 2-SM tile (cta_group::2) for the row-major store GEMMs (kEpiStore, bf16):
+// a cluster of two CTAs computes a 256 x 256 tile.  Rank r loads rows
+// [256 i + 128 r, +128) of A and rows [256 j + 128 r, +128) of B into its own
+// shared memory, 32 KB per 64-deep stage; rank 0 issues
+// tcgen05.mma.cta_group::2 with M = 256, N = 256, whose operands are read from
+// both CTAs and whose accumulator rows land in the tensor memory of the CTA
+// that holds them.  Per SM that is 32 KB of operands per 128 x 256 x 64 of
+// MMA work instead of 48 KB, so the same bytes in flight feed 1.5x the
+// tensor-core work.  Both CTAs' loads are counted on rank 0's full barrier
+// (armed by rank 0 for the pair's 64 KB); rank 0's commits arrive on the
+// empty and accumulator barriers of both CTAs.  Three stages per CTA and two
+// CTAs per SM.  Each output element is one K-ordered chain of MMAs, as in
+// gemm_kernel.
+constexpr int kPairStages = 3;
+constexpr int kPairStageBytes = 2 * BM * ROW_BYTES;  // A half + B half
+constexpr int kPairSmem = kPairStages * kPairStageBytes + 1024;
+static_assert(BM * (2 * 64 + 4) * 4 <= kPairStages * kPairStageBytes, "RoPE rows fit the drained stages");
+
+__global__ void __launch_bounds__(128, 1) gemm_pair_kernel(const __grid_constant__ GemmArgs g) {
+  constexpr int BN = 256;
+  constexpr int STAGES = kPairStages;
+  constexpr int BK = 64;
+  constexpr int A_BYTES = BM * ROW_BYTES;
+  constexpr int STAGE_BYTES = kPairStageBytes;
+  constexpr uint32_t TMEM_COLS = 256;
+  constexpr uint32_t IDESC = umma_idesc(2 * BM, BN, 1);
+
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                             ~static_cast<uintptr_t>(1023));
+  __shared__ __align__(8) uint64_t full_bar[STAGES];
+  __shared__ __align__(8) uint64_t empty_bar[STAGES];
+  __shared__ __align__(8) uint64_t acc_bar;
+  __shared__ uint32_t tmem_slot;
+  __shared__ volatile int abort_flag;
+  __shared__ int pair_abort;
+
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  pdl_launch_dependents();
+  const uint32_t rank = cluster_rank();
+  const bool leader = rank == 0;
+  const int tiles_m = (g.M + 2 * BM - 1) / (2 * BM);
+  const int tiles_n = (g.N + BN - 1) / BN;
+  const int bid = blockIdx.x >> 1;
+  const int GN = g.group_n < 1 ? 1 : g.group_n;
+  const int per_group = tiles_m * GN;
+  const int grp = bid / per_group;
+  const int rem = bid - grp * per_group;
+  const int n0 = grp * GN;
+  const int gw = min(GN, tiles_n - n0);
+  const int tile_m = rem / gw;          // 256-row tile of the pair
+  const int tile_n = n0 + rem % gw;     // 256-column tile
+  const int my_m = tile_m * 2 + (int)rank;  // this CTA's 128-row tile
+  const int num_kb = (g.K + BK - 1) / BK;
+
+  if (tid == 0) {
+    for (int s = 0; s < STAGES; ++s) {
+      mbar_init(smem_u32(&full_bar[s]), 1);
+      mbar_init(smem_u32(&empty_bar[s]), 1);
+    }
+    mbar_init(smem_u32(&acc_bar), 1);
+    abort_flag = 0;
+    fence_mbar_init();
+  }
+  if (warp == 2) tmem_alloc_pair(smem_u32(&tmem_slot), TMEM_COLS);
+  if (warp == 3 && lane == 0) {
+    prefetch_tmap(&g.A.map[0]);
+    prefetch_tmap(&g.B.map[0]);
+  }
+  tc_fence_before();
+  cluster_sync_all();  // both CTAs' barriers and tensor memory exist before either touches the other's
+  tc_fence_after();
+  const uint32_t tmem = tmem_slot;
+
+  if (!(warp == 0 && lane == 0)) pdl_wait();  // the producer waits after its weight prefetch
+  if (warp == 0 && lane == 0) {
+    // ------------------------------------------------ TMA producer (both CTAs)
+    auto full_of = [&](int st) { return map_rank(smem_u32(&full_bar[st]), 0u); };
+    auto load_a = [&](int st, int kb) {
+      const uint32_t sa = smem_u32(smem + st * STAGE_BYTES);
+      const CUtensorMap* map;
+      int row;
+#pragma unroll
+      for (int h = 0; h < 2; ++h) {
+        operand_rows(g.A, my_m * BM, h, my_m, &map, &row);
+        tma_load_2d_pair(sa + h * (64 * ROW_BYTES), map, kb * BK, row, full_of(st));
+      }
+    };
+    auto load_b = [&](int st, int kb) {
+      const CUtensorMap* map;
+      int row;
+      operand_rows(g.B, tile_n * BN + (int)rank * BM, 0, tile_n, &map, &row);
+      tma_load_2d_pair(smem_u32(smem + st * STAGE_BYTES) + A_BYTES, map, kb * BK, row, full_of(st));
+    };
+    // rank 0 arms each stage for the bytes of both CTAs; the peer's copies
+    // may land before that (the transaction count then dips below zero, but
+    // the phase cannot complete before rank 0's arrival)
+    const int npre = g.pre_operand ? min(STAGES, num_kb) : 0;
+    for (int i = 0; i < npre; ++i) {
+      if (leader) mbar_arrive_expect_tx(smem_u32(&full_bar[i]), 2 * STAGE_BYTES);
+      if (g.pre_operand == 1) load_a(i, i); else load_b(i, i);
+    }
+    pdl_wait();
+    for (int i = 0; i < npre; ++i) {
+      if (g.pre_operand == 1) load_b(i, i); else load_a(i, i);
+    }
+    int s = npre % STAGES;
+    uint32_t ph = npre == STAGES ? 1u : 0u;
+    int issued = npre;
+    for (int kb = npre; kb < num_kb; ++kb) {
+      if (!mbar_wait(smem_u32(&empty_bar[s]), ph ^ 1, g.status)) { abort_flag = 1; break; }
+      if (abort_flag) break;
+      if (leader) mbar_arrive_expect_tx(smem_u32(&full_bar[s]), 2 * STAGE_BYTES);
+      load_a(s, kb);
+      load_b(s, kb);
+      ++issued;
+      if (++s == STAGES) { s = 0; ph ^= 1; }
+    }
+    if (abort_flag && leader) {
+      // copies already in flight (both CTAs' copies of every armed stage)
+      // land before shared memory is released
+      int ss = s;
+      uint32_t pp = ph;
+      for (int i = 0; i < min(issued, STAGES); ++i) {
+        if (--ss < 0) { ss = STAGES - 1; pp ^= 1; }
+        mbar_wait(smem_u32(&full_bar[ss]), pp, nullptr);
+      }
+    }
+  } else if (warp == 1 && lane == 0 && leader) {
+    // ------------------------------------------------ MMA issuer (rank 0)
+    int s = 0;
+    uint32_t ph = 0;
+    for (int kb = 0; kb < num_kb; ++kb) {
+      if (!mbar_wait(smem_u32(&full_bar[s]), ph, g.status)) { abort_flag = 1; break; }
+      if (abort_flag) break;
+      tc_fence_after();
+      const uint32_t sa = smem_u32(smem + s * STAGE_BYTES);
+      const uint64_t ad = umma_desc_sw128(sa);
+      const uint64_t bd = umma_desc_sw128(sa + A_BYTES);
+#pragma unroll
+      for (int k = 0; k < 4; ++k)  // 4 x 32 bytes of K per 128-byte row
+        mma_bf16_pair(tmem, ad + 2 * k, bd + 2 * k, IDESC, (kb > 0 || k > 0) ? 1u : 0u);
+      mma_commit_pair(smem_u32(&empty_bar[s]), (uint16_t)0x3);
+      if (++s == STAGES) { s = 0; ph ^= 1; }
+    }
+    mma_commit_pair(smem_u32(&acc_bar), (uint16_t)0x3);  // also drains every MMA issued above
+  }
+  __syncwarp();
+
+  // ------------------------------------------------------ epilogue
+  if (!mbar_wait(smem_u32(&acc_bar), 0, g.status)) abort_flag = 1;
+  tc_fence_after();
+  __syncthreads();
+  cluster_sync_all();  // both CTAs' abort flags are final and visible
+  if (tid == 0)
+    pair_abort = abort_flag | ld_dsmem_s32(map_rank(smem_u32((const void*)&abort_flag), rank ^ 1u));
+  __syncthreads();
+  const uint32_t taddr = tmem + ((uint32_t)(warp * 32) << 16);
+  int spos = 0;
+  const long long t = (long long)my_m * BM + tid;
+  const long long srow = t < g.M ? ctx_store_row(g.epi, t, &spos, g.status) : -1;
+  if (!pair_abort && num_kb > 0) {
+    const float* rope_row = stage_rope_row<BN>(g, my_m, tile_n, smem, spos);
+#pragma unroll 1
+    for (int c0 = 0; c0 < BN; c0 += 16) {
+      float v[16];
+      tmem_ld16(taddr + c0, v);
+      epilogue_chunk<__nv_bfloat16, BN>(g, my_m, tile_n, c0, v, smem, rope_row, srow, spos);
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  cluster_sync_all();  // neither CTA frees the pair's tensor memory while the other still reads it
+  if (warp == 2) {
+    tc_fence_after();
+    tmem_dealloc_pair(tmem, TMEM_COLS);
+  }
+}
+
+cudaError_t prepare_pair() {
+  static cudaError_t state =
+      cudaFuncSetAttribute(gemm_pair_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, kPairSmem);
+  return state;
+}
+
+cudaError_t launch_pair(const GemmArgs& g, cudaStream_t s) {
+  cudaError_t e;
+  if ((e = prepare_pair()) != cudaSuccess) return e;
+  if (g.dtype != HDF_BF16 || g.k_splits != 1 || g.bn != 256 || g.epi.kind != kEpiStore) return cudaErrorInvalidValue;
+  const long long tiles = (long long)((g.M + 2 * BM - 1) / (2 * BM)) * ((g.N + 255) / 256);
+  return launch_kernel(gemm_pair_kernel, dim3((unsigned)(2 * tiles)), dim3(128), (size_t)kPairSmem, s, 2u, g);
 }
 
 // Function attributes of one instantiation, set once per process: the
@@ -732,6 +934,7 @@ size_t gemm_smem_bytes(int, int bn) { return (size_t)smem_for(bn); }
 
 cudaError_t launch_gemm(const GemmArgs& g, cudaStream_t s) {
   if (g.M <= 0 || g.N <= 0) return cudaSuccess;
+  if (g.pair) return launch_pair(g, s);
   return g.dtype == HDF_BF16 ? launch_t<__nv_bfloat16>(g, s) : launch_t<float>(g, s);
 }
 

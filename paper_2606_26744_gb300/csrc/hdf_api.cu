@@ -48,28 +48,34 @@ bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) ==
 size_t esize(int dtype) { return dtype == HDF_BF16 ? 2 : 4; }
 size_t up256(size_t x) { return (x + 255) & ~size_t(255); }
 
+// Per-device caches filled on first use.  Host threads may race to fill a
+// slot; they store the same value, and the slots are atomics, so the race is
+// benign and defined.
 int* device_status_ptr() {
-  static int* ptr[64] = {nullptr};
+  static std::atomic<int*> ptr[64];
   int dev = 0;
   if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return nullptr;
-  if (!ptr[dev]) {
-    void* p = nullptr;
-    if (cudaGetSymbolAddress(&p, g_device_status) != cudaSuccess) return nullptr;
-    ptr[dev] = static_cast<int*>(p);
+  int* p = ptr[dev].load(std::memory_order_acquire);
+  if (!p) {
+    void* q = nullptr;
+    if (cudaGetSymbolAddress(&q, g_device_status) != cudaSuccess) return nullptr;
+    p = static_cast<int*>(q);
+    ptr[dev].store(p, std::memory_order_release);
   }
-  return ptr[dev];
+  return p;
 }
 
 int num_sms() {
-  static int cache[64] = {0};
+  static std::atomic<int> cache[64];
   int dev = 0;
   if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return 148;
-  if (!cache[dev]) {
-    int n = 0;
+  int n = cache[dev].load(std::memory_order_relaxed);
+  if (n <= 0) {
     cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev);
-    cache[dev] = n > 0 ? n : 148;
+    if (n <= 0) n = 148;
+    cache[dev].store(n, std::memory_order_relaxed);
   }
-  return cache[dev];
+  return n;
 }
 
 PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
@@ -186,6 +192,10 @@ void init_gemm(GemmArgs& g, int dtype, long long M, long long N, long long K, co
   g.A.rows_per_map = 1 << 30;
   g.B.rows_per_map = 1 << 30;
 }
+
+// Row-major bf16 GEMMs with 256-wide column tiles and at least 256 rows run
+// on CTA pairs (gemm_pair_kernel).
+bool use_pair_tiles(int dtype, int bn, long long rows) { return dtype == HDF_BF16 && bn == 256 && rows >= 256; }
 
 // ---------------------------------------------------- draft-block layout
 struct DraftLayout {
@@ -388,21 +398,21 @@ int hdf_gated_reduce_backward(const void* H, int dtype, int64_t n_tokens, int m,
 }
 
 // ------------------------------------------------------------- reducer
-static std::atomic<int> g_reduce_path{HDF_REDUCE_AUTO};
-
-int hdf_set_reduce_path(int path) {
-  g_err.clear();
-  if (path != HDF_REDUCE_AUTO && path != HDF_REDUCE_GENERAL && path != HDF_REDUCE_CLUSTER && path != HDF_REDUCE_TILE)
-    return fail(HDF_ERR_INVALID_ARG, "reduce path %d", path);
-  g_reduce_path.store(path);
-  return HDF_OK;
-}
-
 int hdf_gated_reduce(const void* H, int dtype, int64_t n_tokens, int m, int d, const void* Wf, const float* b,
                      float rms_eps, float gate_scale, float gate_offset, const void* path_norm_w,
                      float path_norm_eps, const float* alpha_override, void* y, float* alpha_out,
                      hdf_stream_t stream) {
+  return hdf_gated_reduce_kernel(HDF_REDUCE_AUTO, H, dtype, n_tokens, m, d, Wf, b, rms_eps, gate_scale, gate_offset,
+                                 path_norm_w, path_norm_eps, alpha_override, y, alpha_out, stream);
+}
+
+int hdf_gated_reduce_kernel(int path, const void* H, int dtype, int64_t n_tokens, int m, int d, const void* Wf,
+                            const float* b, float rms_eps, float gate_scale, float gate_offset,
+                            const void* path_norm_w, float path_norm_eps, const float* alpha_override, void* y,
+                            float* alpha_out, hdf_stream_t stream) {
   g_err.clear();
+  if (path != HDF_REDUCE_AUTO && path != HDF_REDUCE_GENERAL && path != HDF_REDUCE_CLUSTER && path != HDF_REDUCE_TILE)
+    return fail(HDF_ERR_INVALID_ARG, "reduce kernel %d", path);
   if (dtype != HDF_BF16 && dtype != HDF_F32) return fail(HDF_ERR_DTYPE, "dtype %d", dtype);
   if (n_tokens < 0) return fail(HDF_ERR_SHAPE, "n_tokens < 0");
   if (!(m == 1 || m == 2 || m == 3 || m == 4 || m == 8)) return fail(HDF_ERR_UNSUPPORTED, "m=%d", m);
@@ -434,7 +444,6 @@ int hdf_gated_reduce(const void* H, int dtype, int64_t n_tokens, int m, int d, c
   a.path_norm_eps = path_norm_eps;
   a.status = device_status_ptr();
   unsigned box[3];
-  const int path = g_reduce_path.load();
   unsigned tail_box[3];
   // auto: the tile kernel for m = 4 (1.2-1.6x the general kernel from 4096
   // tokens, a tie below), the general kernel for other m.  The choice does not
@@ -477,9 +486,10 @@ int hdf_fc_reduce(const void* H, int dtype, int64_t n_tokens, int m, int d, cons
   GemmArgs g;
   init_gemm(g, dtype, n_tokens, d, K, p);
   g.group_n = 8;
+  g.pair = use_pair_tiles(dtype, p.bn, n_tokens);
   int rc;
   if ((rc = make_map(&g.A.map[0], H, dtype, n_tokens, K, K, 64))) return rc;
-  if ((rc = make_map(&g.B.map[0], W_fc, dtype, d, K, K, p.bn))) return rc;
+  if ((rc = make_map(&g.B.map[0], W_fc, dtype, d, K, K, g.pair ? 128 : p.bn))) return rc;
   g.pre_operand = 2;  // the weight
   g.epi.kind = kEpiStore;
   g.epi.out[0] = y;
@@ -583,9 +593,13 @@ int launch_ctx_kv(const hdf_drafter_weights* w, const hdf_layer_weights& Lw, con
     const SplitPlan p{ctx_kv_bn(sh, rows), 1, 0};
     init_gemm(g, dt, rows, 2 * d, d, p);
     g.group_n = 8;
+    // 256-wide tiles run as 256 x 256 tiles on CTA pairs: each CTA loads
+    // 128 rows of the weights
+    g.pair = use_pair_tiles(dt, p.bn, rows);
+    const int b_box = g.pair ? 128 : p.bn;
     if ((rc = make_map(&g.A.map[0], c, dt, rows, d, d, 64))) return rc;
-    if ((rc = make_map(&g.B.map[0], Lw.wk, dt, d, d, d, p.bn))) return rc;
-    if ((rc = make_map(&g.B.map[1], Lw.wv, dt, d, d, d, p.bn))) return rc;
+    if ((rc = make_map(&g.B.map[0], Lw.wk, dt, d, d, d, b_box))) return rc;
+    if ((rc = make_map(&g.B.map[1], Lw.wv, dt, d, d, d, b_box))) return rc;
     g.pre_operand = 2;
     g.B.rows_per_map = (int)d;
     g.epi.kind = kEpiStore;
@@ -1112,8 +1126,9 @@ int hdf_lm_head_argmax_static(const void* h, int dtype, int64_t M, int d, const 
   void* ws = nullptr;
   int rc = lm_static_scratch(&ws);
   if (rc) return rc;
-  // the tile tickets are cleared inside hdf_lm_head_argmax; every other
-  // scratch entry is written before it is read
+  // nothing in the shared array needs clearing between calls: the GEMM
+  // epilogue writes every [tile, row] partial (max, argmax, sum-exp) of this
+  // call before lm_reduce_kernel, the next kernel in the stream, reads it
   return hdf_lm_head_argmax(h, dtype, M, d, W_lm, V, inv_temp, tok, zmax, logsoftmax, ws,
                             (size_t)HDF_LM_HEAD_STATIC_SCRATCH_BYTES, stream);
 }

@@ -143,6 +143,8 @@ struct GemmArgs {
   int pre_operand;      // 1: A, 2: B does not depend on earlier kernels (weights) and is loaded
                         // before pdl_wait(); 0: neither
   int group_n;          // raster: n-tiles swept together
+  int pair;             // 1: 256 x 256 tiles on CTA pairs (cta_group::2); bf16, bn 256, kEpiStore, no K split
+                        // (B maps with 128-row boxes)
   Epilogue epi;
   int* status;
 };

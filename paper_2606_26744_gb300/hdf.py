@@ -88,7 +88,8 @@ _SIGS = {
     "hdf_accept_len": (c_int, [c_vp, c_i64, c_vp, c_i64, c_int, c_int, c_vp, c_vp]),
     "hdf_lm_head_argmax_static": (c_int, [c_vp, c_int, c_i64, c_int, c_vp, c_i64, c_float, c_vp, c_vp, c_vp,
                                           c_vp]),
-    "hdf_set_reduce_path": (c_int, [c_int]),
+    "hdf_gated_reduce_kernel": (c_int, [c_int, c_vp, c_int, c_i64, c_int, c_int, c_vp, c_vp, c_float, c_float,
+                                        c_float, c_vp, c_float, c_vp, c_vp, c_vp, c_vp]),
     "hdf_accept_sample": (c_int, [c_vp, c_vp, c_vp, c_i64, c_vp, c_vp, c_int, c_int, c_i64, c_vp, c_vp, c_vp]),
     "hdf_kl_distill_workspace_size": (c_size, [c_i64, c_i64]),
     "hdf_kl_distill": (c_int, [c_vp, c_vp, c_i64, c_i64, c_float, c_vp, c_vp, c_vp, c_size, c_vp]),
@@ -145,12 +146,7 @@ def device_status(reset: bool = True) -> int:
 
 
 # ----------------------------------------------------------------- reducer
-REDUCE_PATHS = {"auto": 0, "general": 1, "cluster": 2, "tile": 3}
-
-
-def hdf_set_reduce_path(path: str) -> None:
-    """Kernel choice of hdf_gated_reduce: "auto", "general" or "cluster"."""
-    _check(load().hdf_set_reduce_path(REDUCE_PATHS[path]))
+REDUCE_KERNELS = {"auto": 0, "general": 1, "cluster": 2, "tile": 3}
 
 
 def hdf_gated_reduce_backward(H: torch.Tensor, Wf: torch.Tensor, b: torch.Tensor, dy: torch.Tensor, *,
@@ -177,14 +173,20 @@ def hdf_gated_reduce(H: torch.Tensor, Wf: Optional[torch.Tensor], b: Optional[to
                      rms_eps: float = 1e-6, gate_scale: float = 1.0, gate_offset: float = 0.0,
                      path_norm_w: Optional[torch.Tensor] = None, path_norm_eps: float = 1e-6,
                      alpha_override: Optional[torch.Tensor] = None, y: Optional[torch.Tensor] = None,
-                     alpha_out: Optional[torch.Tensor] = None, stream=None) -> torch.Tensor:
-    """Eq. 1 reducer: H [N, m, d] -> y [N, d]."""
+                     alpha_out: Optional[torch.Tensor] = None, kernel: Optional[str] = None,
+                     stream=None) -> torch.Tensor:
+    """Eq. 1 reducer: H [N, m, d] -> y [N, d].  ``kernel`` ("general",
+    "cluster", "tile", "auto") picks the kernel for this call through
+    hdf_gated_reduce_kernel; None calls hdf_gated_reduce."""
     N, m, d = H.shape
     if y is None:
         y = torch.empty((N, d), dtype=H.dtype, device=H.device)
-    _check(load().hdf_gated_reduce(_p(H), _dtype(H), N, m, d, _p(Wf), _p(b), rms_eps, gate_scale,
-                                   gate_offset, _p(path_norm_w), path_norm_eps, _p(alpha_override),
-                                   _p(y), _p(alpha_out), _stream(stream)))
+    args = (_p(H), _dtype(H), N, m, d, _p(Wf), _p(b), rms_eps, gate_scale, gate_offset, _p(path_norm_w),
+            path_norm_eps, _p(alpha_override), _p(y), _p(alpha_out), _stream(stream))
+    if kernel is None:
+        _check(load().hdf_gated_reduce(*args))
+    else:
+        _check(load().hdf_gated_reduce_kernel(REDUCE_KERNELS[kernel], *args))
     return y
 
 

@@ -77,11 +77,13 @@ def test_reduce_backward_host_validation(lib):
     assert lib.hdf_gated_reduce_backward_workspace_size(4, 5, 64, 1) == 0   # unsupported m
 
 
-def test_reduce_path_switch(lib):
-    assert lib.hdf_set_reduce_path(3) == 0            # HDF_REDUCE_TILE
-    assert lib.hdf_set_reduce_path(4) == 1            # HDF_ERR_INVALID_ARG
-    for path in (1, 2, 0):                            # general, cluster, auto (left at the default)
-        assert lib.hdf_set_reduce_path(path) == 0
+def test_reduce_kernel_choice_is_validated_per_call(lib):
+    v = ctypes.c_void_p
+    args = (v(256), 1, 0, 4, 64, v(256), v(256), 1e-6, 1.0, 0.0, None, 1e-6, None, v(256), None, None)
+    for kernel in (0, 1, 2, 3):                       # auto, general, cluster, tile: n_tokens = 0 is a no-op
+        assert lib.hdf_gated_reduce_kernel(kernel, *args) == 0
+    assert lib.hdf_gated_reduce_kernel(4, *args) == 1   # HDF_ERR_INVALID_ARG
+    assert lib.hdf_gated_reduce_kernel(-1, *args) == 1
 
 
 def test_accept_sample_host_validation(lib):

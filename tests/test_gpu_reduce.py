@@ -13,12 +13,10 @@ pytestmark = pytest.mark.gpu
 
 @pytest.fixture(params=["general", "cluster", "tile"])
 def reduce_path(request):
-    """Runs a test on each kernel of the reducer (the cluster and tile kernels
-    take the bf16 shapes they support; the others fall back to the general
-    kernel)."""
-    hdf.hdf_set_reduce_path(request.param)
-    yield request.param
-    hdf.hdf_set_reduce_path("auto")
+    """Runs a test on each kernel of the reducer, chosen per call (the
+    cluster and tile kernels take the bf16 shapes they support; the others
+    fall back to the general kernel)."""
+    return request.param
 
 
 def _run(inp, **kw):
@@ -51,7 +49,7 @@ def _run(inp, **kw):
 ])
 def test_reduce_parity(N, m, d, dtype, std, reduce_path):
     inp = W.make_reduce_inputs(N, m, d, dtype, std, seed=N * 131 + d)
-    y, a = _run(inp)
+    y, a = _run(inp, kernel=reduce_path)
     y_ref, a_ref = O.gated_reduce(to64(inp["H"]), to64(inp["Wf"]), to64(inp["b"]), out_dtype=dtype)
     tol = TOL_F32_REDUCE if dtype == "f32" else TOL_BF16
     assert rowwise_rel(to64(y), y_ref) <= tol
@@ -87,7 +85,7 @@ def test_reduce_one_hot_selects_path_bit_exact(reduce_path):
     for j in range(4):
         a = torch.zeros(21, 4, device="cuda")
         a[:, j] = 1
-        y = hdf.hdf_gated_reduce(H, inp["Wf"].cuda(), inp["b"].cuda(), alpha_override=a)
+        y = hdf.hdf_gated_reduce(H, inp["Wf"].cuda(), inp["b"].cuda(), alpha_override=a, kernel=reduce_path)
         assert torch.equal(y, H[:, j, :])
 
 
@@ -108,7 +106,7 @@ def test_reduce_sweep_width_sampled_rows(reduce_path):
     # reducer-only workload width (m=4, d=7168) at 65536 tokens, checked on sampled tokens
     N, m, d = 65536, 4, 7168
     inp = W.make_reduce_inputs(N, m, d, "bf16", 0.1, seed=11, device="cuda")
-    y = hdf.hdf_gated_reduce(inp["H"], inp["Wf"], inp["b"])
+    y = hdf.hdf_gated_reduce(inp["H"], inp["Wf"], inp["b"], kernel=reduce_path)
     torch.cuda.synchronize()
     rows = torch.cat([torch.tensor([0, 1, 2, N - 2, N - 1]), torch.randperm(N, generator=torch.Generator().manual_seed(0))[:59]])
     Hs = to64(inp["H"][rows.cuda()])
@@ -129,6 +127,10 @@ def test_reduce_rows_do_not_depend_on_the_call():
     for lo, hi in [(0, 1), (4095, 4101), (17, 60), (4990, 5000)]:
         y_part = hdf.hdf_gated_reduce(H[lo:hi].contiguous(), Wf, b)
         assert torch.equal(y_part.view(torch.int16), y_all[lo:hi].view(torch.int16))
+    # an explicit kernel choice in one call does not change what the next
+    # default call runs (no state is kept between calls)
+    hdf.hdf_gated_reduce(H[:64].contiguous(), Wf, b, kernel="general")
+    assert torch.equal(hdf.hdf_gated_reduce(H, Wf, b).view(torch.int16), y_all.view(torch.int16))
 
 
 # ------------------------------------------------ gradient w.r.t. W_f and b
