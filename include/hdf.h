@@ -248,6 +248,29 @@ typedef struct {
 } hdf_trace;
 
 HDF_API size_t hdf_draft_block_workspace_size(const hdf_draft_shape* shape);
+
+/* Where hdf_draft_block leaves its intermediates in the caller's workspace:
+ * byte offsets from the workspace start (256-byte aligned), for inspecting a
+ * call stage by stage.  Once the call has completed on its stream, and until
+ * the workspace is reused, the regions hold (M = batch * block, last = the
+ * last layer):
+ *   c          [n_ctx, d] dtype  RMSNorm_{ctx_norm}(ctx)
+ *   k_ctx      [n_ctx, d] dtype  K_c of the last layer (RoPE applied)
+ *   v_ctx      [n_ctx, d] dtype  V_c of the last layer
+ *   h          [M, d]     fp32   the residual after the last layer, before the final norm
+ *   x          [M, d]     dtype  RMSNorm_{mlp_norm}(h) of the last layer (the MLP input)
+ *   q, k_blk, v_blk [M, d] dtype Q, K_b (RoPE applied) and V_b of the last layer
+ *   o          [M, d]     dtype  the attention output of the last layer
+ *   act        [M, F]     dtype  silu(x W_g^T) * (x W_u^T) of the last layer
+ *   total      bytes of the workspace (hdf_draft_block_workspace_size)
+ * With shape->n_ctx = 0 the same holds for hdf_draft_block_cached (c, k_ctx
+ * and v_ctx are then empty).  The paper has no counterpart: this exists so
+ * that each stage can be checked against a reference fed the previous
+ * stage's output.  Returns a status like hdf_draft_block's shape check. */
+typedef struct {
+  size_t c, k_ctx, v_ctx, h, x, q, k_blk, v_blk, o, act, total;
+} hdf_draft_workspace_layout;
+HDF_API int hdf_draft_block_workspace_layout(const hdf_draft_shape* shape, hdf_draft_workspace_layout* out);
 HDF_API int hdf_draft_block(const hdf_drafter_weights* w, const hdf_draft_shape* shape,
                     const void* ctx,        /* [n_ctx, d] dtype (y of Eq. 1) */
                     const int32_t* cu_ctx,  /* [batch + 1] prefix sums of T_i */

@@ -872,6 +872,26 @@ size_t hdf_draft_block_workspace_size(const hdf_draft_shape* shape) {
   return draft_layout(shape).total;
 }
 
+int hdf_draft_block_workspace_layout(const hdf_draft_shape* shape, hdf_draft_workspace_layout* out) {
+  g_err.clear();
+  int rc = check_draft_shape(shape);
+  if (rc) return rc;
+  if (!out) return fail(HDF_ERR_INVALID_ARG, "out is NULL");
+  const DraftLayout L = draft_layout(shape);
+  out->c = L.c;
+  out->k_ctx = L.kc;
+  out->v_ctx = L.vc;
+  out->h = L.h;
+  out->x = L.x;
+  out->q = L.q;
+  out->k_blk = L.kb;
+  out->v_blk = L.vb;
+  out->o = L.o;
+  out->act = L.act;
+  out->total = L.total;
+  return HDF_OK;
+}
+
 int hdf_draft_block(const hdf_drafter_weights* w, const hdf_draft_shape* sh, const void* ctx,
                     const int32_t* cu_ctx, const int32_t* anchor, void* h_out, void* ws, size_t ws_bytes,
                     const hdf_trace* trace, hdf_stream_t stream) {

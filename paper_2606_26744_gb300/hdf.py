@@ -55,6 +55,10 @@ class Trace(ctypes.Structure):
     _fields_ = [("events", ctypes.POINTER(c_vp)), ("n_events", c_int)]
 
 
+class DraftWorkspaceLayout(ctypes.Structure):
+    _fields_ = [(n, c_size) for n in ("c", "k_ctx", "v_ctx", "h", "x", "q", "k_blk", "v_blk", "o", "act", "total")]
+
+
 class CtxCache(ctypes.Structure):
     _fields_ = [("k", c_vp), ("v", c_vp), ("len", c_vp), ("capacity", c_int)]
 
@@ -74,6 +78,7 @@ _SIGS = {
     "hdf_draft_block_workspace_size": (c_size, [ctypes.POINTER(DraftShape)]),
     "hdf_draft_block": (c_int, [ctypes.POINTER(DrafterWeights), ctypes.POINTER(DraftShape), c_vp, c_vp,
                                 c_vp, c_vp, c_vp, c_size, ctypes.POINTER(Trace), c_vp]),
+    "hdf_draft_block_workspace_layout": (c_int, [ctypes.POINTER(DraftShape), ctypes.POINTER(DraftWorkspaceLayout)]),
     "hdf_ctx_append_workspace_size": (c_size, [ctypes.POINTER(DraftShape)]),
     "hdf_ctx_append": (c_int, [ctypes.POINTER(DrafterWeights), ctypes.POINTER(DraftShape), c_vp, c_vp,
                                ctypes.POINTER(CtxCache), c_vp, c_size, c_vp]),
@@ -242,6 +247,26 @@ class Drafter:
     def workspace_size(self, batch: int, block: int, n_ctx: int, max_ctx: int) -> int:
         sh = self.shape(batch, block, n_ctx, max_ctx)
         return load().hdf_draft_block_workspace_size(ctypes.byref(sh))
+
+    def workspace_views(self, ws: torch.Tensor, batch: int, block: int, n_ctx: int, max_ctx: int) -> Dict:
+        """Views of the intermediates hdf_draft_block leaves in ``ws``
+        (hdf_draft_block_workspace_layout): c, k_ctx, v_ctx [n_ctx, d];
+        h [M, d] fp32; x, q, k_blk, v_blk, o [M, d]; act [M, F]."""
+        sh = self.shape(batch, block, n_ctx, max_ctx)
+        lay = DraftWorkspaceLayout()
+        _check(load().hdf_draft_block_workspace_layout(ctypes.byref(sh), ctypes.byref(lay)))
+        dt = self.w["embed"].dtype
+        es = torch.empty((), dtype=dt).element_size()
+        M = batch * block
+
+        def view(off, rows, cols, dtype, esz):
+            return ws[off:off + rows * cols * esz].view(dtype).view(rows, cols)
+        out = {k: view(getattr(lay, k), n_ctx, self.d, dt, es) for k in ("c", "k_ctx", "v_ctx")}
+        out["h"] = view(lay.h, M, self.d, torch.float32, 4)
+        for k in ("x", "q", "k_blk", "v_blk", "o"):
+            out[k] = view(getattr(lay, k), M, self.d, dt, es)
+        out["act"] = view(lay.act, M, self.ffn, dt, es)
+        return out
 
     def n_trace_events(self) -> int:
         return 3 + STAGES_PER_LAYER * self.n_layers
