@@ -614,7 +614,11 @@ NCU_DRAM_BYTES = {
         "gated_reduce": 33675264,
     },
 }
-NCU_DRAM_BYTES_PER_CTX_ROW = {}
+NCU_DRAM_BYTES_PER_CTX_ROW = {
+    # gemm_pair_kernel, one layer's context projection, captured on 16,384
+    # rows at the large widths (profiles/ctx_kv_gemm_pair_large.md)
+    "large": {f"L{l}.ctx_kv_gemm": (16384, 2497119000 + 456967936) for l in range(2)},
+}
 
 
 # DRAM bytes (read + write) per token of the tile reducer at m = 4, d = 7168,
