@@ -150,6 +150,17 @@ def fc_param_count(m: int, d: int) -> int:
     return (m * d) * d
 
 
+def fc_reduce(H, W_fc, out_dtype: str = "f64") -> np.ndarray:
+    """Generic fc collapse of vanilla DFlash (Sec. 2.2, Table 1): the learned
+    linear map of the flattened residual, y_t = W_fc vec(H_t), vec() path-major
+    as in Eq. 1.  W_fc is [d_out, m * d_in]; with d_out != d_in it is the
+    fallback the paper names for a drafter narrower or wider than the target."""
+    H = _f64(H)
+    N, m, d_in = H.shape
+    x = H.reshape(N, m * d_in)                       # vec(H_t), path-major
+    return store(x @ _f64(W_fc).T, out_dtype)
+
+
 # ----------------------------------------------------------------------------
 # (2) drafter block forward
 # ----------------------------------------------------------------------------
@@ -411,3 +422,62 @@ def kl_distill(teacher_logits, student_logits, t_kd: float = 1.0) -> float:
     p = np.exp(lp)
     P = t.shape[0]
     return float(t_kd * t_kd / P * np.sum(p * (lp - lq)))
+
+
+# ----------------------------------------------------------------------------
+# Training objective of the drafter, Eq. 3 (Sec. 2.3)
+# ----------------------------------------------------------------------------
+
+
+def _log_softmax(z) -> np.ndarray:
+    z = _f64(z)
+    zmax = z.max(axis=-1, keepdims=True)
+    return z - (zmax + np.log(np.exp(z - zmax).sum(axis=-1, keepdims=True)))
+
+
+def cross_entropy(logits, labels) -> np.ndarray:
+    """One-hot supervision of Sec. 2.3 per row: -log softmax(z_r)[label_r].
+    A negative label marks a row without supervision; it gets NaN here and
+    takes no part in any mean."""
+    ls = _log_softmax(logits)
+    labels = np.asarray(labels, np.int64)
+    out = np.full(ls.shape[0], np.nan)
+    on = labels >= 0
+    out[on] = -ls[np.nonzero(on)[0], labels[on]]
+    return out
+
+
+def draft_loss(teacher_logits, student_logits, labels, *, block: int, P: int = 2, t_kd: float = 1.0,
+               alpha: float = 0.1) -> Dict[str, float]:
+    """L = L_CE + alpha * L_KL (Eq. 3) for a batch of drafted blocks.
+
+    student_logits [batch * block, V]: row i * block + k holds z_k of block i
+        (k = 0 is the anchor slot, k >= 1 draft position k, which predicts the
+        token at a + k);
+    labels [batch, block - 1]: the true token at a + k for draft position k
+        (negative = unsupervised);
+    teacher_logits [batch, P, V]: LMHead(h_{a+k-1}) for k = 1..P.
+    L_CE is the mean of the per-position cross-entropy over every supervised
+    draft position of the batch (one-hot supervision of the draft logits, at
+    temperature 1); L_KL is Eq. 2, T_KD^2 / P * sum_{k=1..P} KL(p_k^T || q_k^T),
+    with the expectation taken as the mean over the blocks of the batch.
+    Any logits may be passed, log-softmax rows included: both softmaxes are
+    unchanged by a constant shift of a row."""
+    S = _f64(student_logits)
+    Tt = _f64(teacher_logits)
+    batch, Pt, V = Tt.shape
+    assert Pt == P and S.shape == (batch * block, V)
+    labels = np.asarray(labels, np.int64).reshape(batch, block - 1)
+    draft_rows = np.array([i * block + k for i in range(batch) for k in range(1, block)], np.int64)
+    ce = cross_entropy(S[draft_rows], labels.reshape(-1))
+    n_sup = int(np.sum(labels >= 0))
+    l_ce = float(np.nansum(ce) / n_sup) if n_sup else 0.0
+    kl_rows = np.empty((batch, P))
+    for i in range(batch):
+        for k in range(1, P + 1):
+            lp = _log_softmax(Tt[i, k - 1] / t_kd)
+            lq = _log_softmax(S[i * block + k] / t_kd)
+            p = np.exp(lp)
+            kl_rows[i, k - 1] = np.sum(np.where(p > 0, p * (lp - lq), 0.0))
+    l_kl = float(t_kd * t_kd / P * np.sum(kl_rows) / batch)
+    return {"loss": l_ce + alpha * l_kl, "ce": l_ce, "kl": l_kl, "ce_rows": ce, "kl_rows": kl_rows.reshape(-1)}

@@ -91,6 +91,32 @@ MUTATIONS = {
     "argmax takes the last index on ties": (
         "tok = np.argmax(z, axis=1)          # numpy returns the first maximiser",
         "tok = z.shape[1] - 1 - np.argmax(z[:, ::-1], axis=1)"),
+    # --------------------------------------------------------- fc reducer
+    "fc vec() taken element-major": (
+        "x = H.reshape(N, m * d_in)                       # vec(H_t), path-major",
+        "x = H.transpose(0, 2, 1).reshape(N, m * d_in)"),
+    # ------------------------------------------------------ Eq. 3 training loss
+    "CE reads the label's neighbour": (
+        "out[on] = -ls[np.nonzero(on)[0], labels[on]]",
+        "out[on] = -ls[np.nonzero(on)[0], (labels[on] + 1) % ls.shape[1]]"),
+    "CE mean over every draft row, supervised or not": (
+        "l_ce = float(np.nansum(ce) / n_sup) if n_sup else 0.0",
+        "l_ce = float(np.nansum(ce) / len(ce))"),
+    "draft positions start at the anchor slot": (
+        "draft_rows = np.array([i * block + k for i in range(batch) for k in range(1, block)], np.int64)",
+        "draft_rows = np.array([i * block + k - 1 for i in range(batch) for k in range(1, block)], np.int64)"),
+    "KL student row off by one": (
+        "lq = _log_softmax(S[i * block + k] / t_kd)",
+        "lq = _log_softmax(S[i * block + k - 1] / t_kd)"),
+    "loss KL without the temperature-squared factor": (
+        "l_kl = float(t_kd * t_kd / P * np.sum(kl_rows) / batch)",
+        "l_kl = float(1.0 / P * np.sum(kl_rows) / batch)"),
+    "loss KL summed over the batch instead of averaged": (
+        "l_kl = float(t_kd * t_kd / P * np.sum(kl_rows) / batch)",
+        "l_kl = float(t_kd * t_kd / P * np.sum(kl_rows))"),
+    "loss KL weight applied to CE": (
+        'return {"loss": l_ce + alpha * l_kl,',
+        'return {"loss": alpha * l_ce + l_kl,'),
     # --------------------------------------------------------------------- KL
     "KL direction reversed": (
         "return float(t_kd * t_kd / P * np.sum(p * (lp - lq)))",

@@ -362,8 +362,10 @@ def test_draft_block_sequences_are_independent():
 # --------------------------------------------------------------------------
 
 def test_lm_head_argmax_first_index_on_ties_brute_force():
-    h = rng.standard_normal((6, 8))
-    W = rng.standard_normal((40, 8))
+    # small integers: every dot product is exact whatever order the matmul
+    # sums in, so duplicate weight rows give an exact tie
+    h = rng.integers(-8, 9, (6, 8)).astype(np.float64)
+    W = rng.integers(-8, 9, (40, 8)).astype(np.float64)
     W[17] = W[5]                       # exact duplicate rows -> exact tie in z
     h[2] = W[5] * 10                   # row 2's max is the (5, 17) tie
     res = O.lm_head(h, W)
@@ -635,3 +637,129 @@ def test_logsoftmax_two_class_closed_form_at_temperature():
         np.testing.assert_allclose(res["logsoftmax"][0], [-math.log1p(math.exp(-1.5 * t)),
                                                           -math.log1p(math.exp(1.5 * t))], rtol=1e-13)
         assert res["tok"][0] == 0 and res["zmax"][0] == 2.0
+
+
+# --------------------------------------------------------------------------
+# generic fc reducer (Sec. 2.2, Table 1): the fallback for unequal widths
+# --------------------------------------------------------------------------
+
+def test_fc_reduce_identity_blocks_sum_the_paths():
+    """W_fc = [I I ... I] maps vec(H_t) to the plain path sum; a block of
+    the identity's first d_out rows truncates each path to d_out features
+    (a narrower drafter), and the position of a block picks its path."""
+    N, m, d_in = 5, 3, 8
+    H = rng.standard_normal((N, m, d_in))
+    I = np.eye(d_in)
+    np.testing.assert_array_equal(O.fc_reduce(H, np.concatenate([I] * m, axis=1)), H.sum(axis=1))
+    d_out = 4
+    W = np.zeros((d_out, m * d_in))
+    W[:, 2 * d_in:2 * d_in + d_out] = np.eye(d_out)        # path 2, first d_out features
+    np.testing.assert_array_equal(O.fc_reduce(H, W), H[:, 2, :d_out])
+    # a wider drafter: path 0 placed twice, the second copy negated
+    W = np.zeros((2 * d_in, m * d_in))
+    W[:d_in, :d_in] = I
+    W[d_in:, :d_in] = -I
+    np.testing.assert_array_equal(O.fc_reduce(H, W), np.concatenate([H[:, 0], -H[:, 0]], axis=1))
+
+
+def test_fc_reduce_brute_force_loops():
+    N, m, d_in, d_out = 3, 2, 5, 7
+    H = rng.standard_normal((N, m, d_in))
+    W = rng.standard_normal((d_out, m * d_in))
+    ref = np.zeros((N, d_out))
+    for t in range(N):
+        for o in range(d_out):
+            ref[t, o] = sum(W[o, j * d_in + e] * H[t, j, e] for j in range(m) for e in range(d_in))
+    np.testing.assert_allclose(O.fc_reduce(H, W), ref, rtol=1e-13, atol=1e-13)
+
+
+# --------------------------------------------------------------------------
+# training objective, Eq. 3: L = L_CE + alpha * L_KL
+# --------------------------------------------------------------------------
+
+def test_cross_entropy_closed_forms():
+    # two classes with logits (0, x): CE of class 1 = log(1 + e^-x), of class 0 = log(1 + e^x)
+    for x in (-3.0, 0.0, 0.7, 5.0):
+        z = np.array([[0.0, x], [0.0, x]])
+        np.testing.assert_allclose(O.cross_entropy(z, [1, 0]),
+                                   [math.log1p(math.exp(-x)), math.log1p(math.exp(x))], rtol=1e-12)
+    # uniform logits over V classes: log V whatever the label; a shift changes nothing
+    z = np.full((3, 10), 2.5)
+    np.testing.assert_allclose(O.cross_entropy(z, [0, 4, 9]), math.log(10.0), rtol=1e-14)
+    # an unsupervised row is NaN (kept out of any mean)
+    assert np.isnan(O.cross_entropy(z, [-1, 0, 0])[0])
+
+
+def _two_class_kl(a, b, T):
+    p1 = 1.0 / (1.0 + math.exp(-a / T))
+    q1 = 1.0 / (1.0 + math.exp(-b / T))
+    return p1 * math.log(p1 / q1) + (1 - p1) * math.log((1 - p1) / (1 - q1))
+
+
+def test_draft_loss_two_class_closed_form():
+    """batch 2, block 3, P = 2, two classes.  Logit rows are (0, x).  Student
+    rows: anchor slots get a logit the loss must ignore, draft k of block i
+    gets s[i][k-1]; teacher row k - 1 of block i gets t[i][k-1].  Labels make
+    each CE a log1p term.  Every term is written out by hand."""
+    s = [[0.4, -1.2], [2.0, 0.3]]
+    t = [[1.5, -0.5], [0.0, 3.0]]
+    lab = [[1, 0], [0, 1]]
+    S = np.zeros((6, 2))
+    for i in range(2):
+        S[i * 3, 1] = 40.0  # anchor rows: neither CE nor KL may read them
+        for k in (1, 2):
+            S[i * 3 + k, 1] = s[i][k - 1]
+    Tt = np.zeros((2, 2, 2))
+    for i in range(2):
+        for k in range(2):
+            Tt[i, k, 1] = t[i][k]
+
+    def ce(x, y):
+        return math.log1p(math.exp(-x)) if y == 1 else math.log1p(math.exp(x))
+    for T, a in ((1.0, 0.1), (2.0, 0.2), (0.5, 1.0)):
+        out = O.draft_loss(Tt, S, lab, block=3, P=2, t_kd=T, alpha=a)
+        l_ce = sum(ce(s[i][k], lab[i][k]) for i in range(2) for k in range(2)) / 4
+        l_kl = T * T / 2 * sum(_two_class_kl(t[i][k], s[i][k], T) for i in range(2) for k in range(2)) / 2
+        np.testing.assert_allclose(out["ce"], l_ce, rtol=1e-13)
+        np.testing.assert_allclose(out["kl"], l_kl, rtol=1e-12)
+        np.testing.assert_allclose(out["loss"], l_ce + a * l_kl, rtol=1e-12)
+
+
+def test_draft_loss_kl_covers_the_first_P_positions_only():
+    """Teacher equal to the student on positions 1..P gives L_KL = 0 whatever
+    positions past P and the anchor slot hold; changing position P + 1 or the
+    anchor leaves the loss's KL part alone, changing position P does not."""
+    batch, B, P, V = 3, 5, 2, 7
+    S = rng.standard_normal((batch * B, V))
+    Tt = np.stack([S[i * B + 1:i * B + 1 + P] for i in range(batch)])
+    lab = rng.integers(0, V, (batch, B - 1))
+    base = O.draft_loss(Tt, S, lab, block=B, P=P, t_kd=1.7, alpha=0.3)
+    assert abs(base["kl"]) < 1e-14
+    S2 = S.copy()
+    S2[0] += 5.0 * rng.standard_normal(V)            # anchor of block 0
+    S2[1 * B + P + 1] += 5.0 * rng.standard_normal(V)  # position P + 1 of block 1
+    assert abs(O.draft_loss(Tt, S2, lab, block=B, P=P, t_kd=1.7, alpha=0.3)["kl"]) < 1e-14
+    S3 = S.copy()
+    S3[2 * B + P] += 5.0 * rng.standard_normal(V)      # position P of block 2
+    assert O.draft_loss(Tt, S3, lab, block=B, P=P, t_kd=1.7, alpha=0.3)["kl"] > 1e-3
+
+
+def test_draft_loss_ce_is_at_temperature_one_and_skips_unlabelled_rows():
+    batch, B, V = 2, 4, 6
+    S = rng.standard_normal((batch * B, V))
+    Tt = rng.standard_normal((batch, 2, V))
+    lab = np.array([[3, -1, 0], [-1, -1, 5]])
+    a = O.draft_loss(Tt, S, lab, block=B, P=2, t_kd=1.0, alpha=0.0)
+    b = O.draft_loss(Tt, S, lab, block=B, P=2, t_kd=4.0, alpha=0.0)
+    assert a["ce"] == b["ce"] and a["loss"] == a["ce"]
+    # the mean runs over the three supervised positions, each a brute-force -log softmax
+    def nll(z, y):
+        return -(z[y] - math.log(sum(math.exp(v) for v in z)))
+    ref = (nll(S[1], 3) + nll(S[3], 0) + nll(S[7], 5)) / 3
+    np.testing.assert_allclose(a["ce"], ref, rtol=1e-13)
+    # a constant shift of any row changes nothing (log-softmax rows may be passed)
+    S4 = S + rng.standard_normal((batch * B, 1))
+    T4 = Tt + rng.standard_normal((batch, 2, 1))
+    c = O.draft_loss(T4, S4, lab, block=B, P=2, t_kd=2.0, alpha=0.5)
+    d = O.draft_loss(Tt, S, lab, block=B, P=2, t_kd=2.0, alpha=0.5)
+    np.testing.assert_allclose(c["loss"], d["loss"], rtol=1e-12)
