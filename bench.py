@@ -339,7 +339,27 @@ def run_ours(args, rank, world, local_rank, config=None, light=False):
     kl_us = k0.elapsed_time(k1) / 20 * 1000
     kl = {"rows": kl_rows_n, "vocab": V, "us": round(kl_us, 2),
           "gbs": round(2 * kl_rows_n * V * 4 / kl_us / 1e3, 1), "launches": 2}
-    del ls_t, ls_s
+    # the whole objective of Eq. 3 over the batch's blocks: CE of every draft
+    # position (a gather from the student's log-softmax rows) plus the KL of
+    # the first P = 2 positions renormalised at T_KD = 2 in one pass
+    ls_blk = torch.log_softmax(torch.randn(batch * B, V, device=dev, generator=gk) * 3, dim=1)
+    lab = torch.randint(0, V, (batch, B - 1), device=dev, dtype=torch.int32, generator=gk)
+    lt3 = ls_t.view(batch, 2, V)
+    lossv = torch.empty(3, device=dev)
+    lws = torch.empty(max(1, hdf.load().hdf_draft_loss_workspace_size(batch, 2, V)), dtype=torch.uint8, device=dev)
+    for _ in range(3):
+        hdf.hdf_draft_loss(lt3, ls_blk, lab, block=B, t_kd=2.0, alpha=0.1, loss=lossv, ws=lws, stream=stream)
+    stream.synchronize()
+    k0.record(stream)
+    for _ in range(20):
+        hdf.hdf_draft_loss(lt3, ls_blk, lab, block=B, t_kd=2.0, alpha=0.1, loss=lossv, ws=lws, stream=stream)
+    k1.record(stream)
+    stream.synchronize()
+    loss_us = k0.elapsed_time(k1) / 20 * 1000
+    loss_bytes = 2 * batch * 2 * V * 4 + batch * (B - 1) * 8 + 12
+    draft_loss = {"blocks": batch, "P": 2, "vocab": V, "us": round(loss_us, 2), "bytes": loss_bytes,
+                  "gbs": round(loss_bytes / loss_us / 1e3, 1), "launches": 2}
+    del ls_t, ls_s, ls_blk, lt3
 
     # -------------------- reducer gradient w.r.t. W_f and b (training-time)
     # over this workload's context residual, upstream dy ~ N(0, 1); timed
@@ -460,7 +480,8 @@ def run_ours(args, rank, world, local_rank, config=None, light=False):
         t = torch.tensor([ms, e2e_ms], device=dev)
         torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
         ms, e2e_ms = float(t[0]), float(t[1])
-    return dict(cfg=cfg, ms=ms, ms_staged=ms_staged, e2e_ms=e2e_ms, dur=dur, clk=clk, kl=kl, verify_t1=verify_t1,
+    return dict(cfg=cfg, ms=ms, ms_staged=ms_staged, e2e_ms=e2e_ms, dur=dur, clk=clk, kl=kl, draft_loss=draft_loss,
+                verify_t1=verify_t1,
                 reduce_bwd=reduce_bwd,
                 warm=warm, pct=pct, accept_sweep=accept_sweep, batch=batch, n_ctx=n_ctx, lens=lens,
                 h2d=h2d, d2h=d2h, acc_mean=acc_mean, tok=tok, y=y, inputs=inp, tgt=tgt)
@@ -788,6 +809,79 @@ def run_sweep(args):
     return 0
 
 
+def run_kernel_only(args):
+    """One kernel of the path alone, for profiling runs (not a bench line):
+    3 warm-up launches, then args.steps launches timed with CUDA events.
+      accept      hdf_accept_len over args.tokens blocks of 15 drafts
+      reduce_bwd  hdf_gated_reduce_backward over args.tokens tokens, m 4, d 7168
+      reduce      hdf_gated_reduce (tile kernel) over args.tokens tokens, m 4, d 7168
+      loss        hdf_draft_loss over the large workload's blocks (8 x 16, P 2, V 129280)"""
+    from paper_2606_26744_gb300 import build, hdf
+    build.build()
+    dev = torch.device("cuda", 0)
+    pk = peaks()
+    g = torch.Generator(device=dev).manual_seed(7)
+    n = args.tokens
+    if args.kernel_only == "accept":
+        nd = 15
+        dr = torch.randint(0, 129280, (n, nd), device=dev, dtype=torch.int32, generator=g)
+        keep = torch.randint(0, nd + 1, (n, 1), device=dev, generator=g)
+        tg = torch.where(torch.arange(nd, device=dev)[None, :] < keep, dr, (dr + 1) % 129280)
+        acc = torch.empty(n, dtype=torch.int32, device=dev)
+
+        def launch():
+            hdf.hdf_accept_len(dr, tg, n_draft=nd, draft_stride=nd, batch=n, accept=acc)
+        byt = 2 * n * nd * 4 + n * 4
+    elif args.kernel_only in ("reduce_bwd", "reduce"):
+        m, d = 4, 7168
+        inp = W.make_reduce_inputs(n, m, d, "bf16", 0.1, seed=1004, device=dev)
+        H, Wf, b = inp["H"], inp["Wf"], inp["b"]
+        if args.kernel_only == "reduce":
+            y = torch.empty((n, d), dtype=torch.bfloat16, device=dev)
+
+            def launch():
+                hdf.hdf_gated_reduce(H, Wf, b, y=y)
+            byt = n * m * d * 2 + n * d * 2 + m * m * d * 2
+        else:
+            dy = torch.randn((n, d), device=dev, generator=g).to(torch.bfloat16)
+            dwf = torch.empty((m, m * d), dtype=torch.float32, device=dev)
+            dbv = torch.empty(m, dtype=torch.float32, device=dev)
+            ws = torch.empty(max(1, hdf.load().hdf_gated_reduce_backward_workspace_size(n, m, d, hdf._dtype(H))),
+                             dtype=torch.uint8, device=dev)
+
+            def launch():
+                hdf.hdf_gated_reduce_backward(H, Wf, b, dy, dWf=dwf, db=dbv, ws=ws)
+            byt = 2 * n * m * d * 2 + n * d * 2 + m * m * d * 2 + m * m * d * 4
+    elif args.kernel_only == "loss":
+        batch, block, P, V = 8, 16, 2, 129280
+        ls_s = torch.log_softmax(torch.randn(batch * block, V, device=dev, generator=g) * 3, dim=-1)
+        ls_t = torch.log_softmax(torch.randn(batch, P, V, device=dev, generator=g) * 3, dim=-1)
+        lab = torch.randint(0, V, (batch, block - 1), device=dev, dtype=torch.int32, generator=g)
+        loss = torch.empty(3, device=dev)
+
+        def launch():
+            hdf.hdf_draft_loss(ls_t, ls_s, lab, block=block, t_kd=2.0, alpha=0.1, loss=loss)
+        byt = 2 * batch * P * V * 4 + batch * (block - 1) * 8 + 12
+    else:
+        raise SystemExit(f"unknown kernel {args.kernel_only}")
+    for _ in range(3):
+        launch()
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record()
+    for _ in range(args.steps):
+        launch()
+    e1.record()
+    torch.cuda.synchronize()
+    us = e0.elapsed_time(e1) / args.steps * 1e3
+    if hdf.device_status() != 0:
+        raise RuntimeError("a device-side check failed")
+    print(json.dumps({"kernel": args.kernel_only, "units": n, "us": round(us, 2), "algorithmic_bytes": int(byt),
+                      "gbs": round(byt / us / 1e3, 1), "frac_hbm": round(byt / us / 1e3 / pk["hbm_gbs"], 4)}),
+          flush=True)
+    return 0
+
+
 def host_cores():
     try:
         return len(os.sched_getaffinity(0))
@@ -982,6 +1076,9 @@ def main():
     ap.add_argument("--batch", type=int, default=None, help="profiling override of the workload's batch")
     ap.add_argument("--vocab", type=int, default=None, help="profiling override of the workload's vocabulary")
     ap.add_argument("--layers", type=int, default=None, help="profiling override of the workload's layers")
+    ap.add_argument("--kernel-only", default=None, choices=["accept", "reduce_bwd", "reduce", "loss"],
+                    help="time one kernel alone (profiling runs; not a bench line)")
+    ap.add_argument("--tokens", type=int, default=1 << 20, help="units of a --kernel-only run")
     args = ap.parse_args()
     args.overrides = {k: v for k, v in (("batch", args.batch), ("vocab", args.vocab), ("n_layers", args.layers))
                       if v is not None}
@@ -995,6 +1092,8 @@ def main():
         return run_reference(args)
     if args.config == "sweep":
         return run_sweep(args)
+    if args.kernel_only:
+        return run_kernel_only(args)
 
     world = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
@@ -1048,6 +1147,7 @@ def main():
             "roofline": rf,
             "reducer": {"gbs": red.get("gbs"), "frac_hbm": red.get("frac"), "us": red["us"]},
             "kl_target": dict(res["kl"], frac_hbm=round(res["kl"]["gbs"] / pk["hbm_gbs"], 3)),
+            "draft_loss": dict(res["draft_loss"], frac_hbm=round(res["draft_loss"]["gbs"] / pk["hbm_gbs"], 3)),
             "reducer_backward": dict(res["reduce_bwd"], frac_hbm=round(res["reduce_bwd"]["gbs"] / pk["hbm_gbs"], 3)),
             "verify_t1": res["verify_t1"],
             "accept_sweep": dict(res["accept_sweep"], frac_hbm=round(res["accept_sweep"]["gbs"] / pk["hbm_gbs"], 3)),

@@ -167,11 +167,16 @@ HDF_API int hdf_gated_reduce_backward(const void* H, int dtype, int64_t n_tokens
                               hdf_stream_t stream);
 
 /* Generic fc reducer of vanilla DFlash (Sec. 2.2, Table 1 "generic fc"),
- * kept as the comparison path and the fallback the paper names:
- *   y_t = W_fc vec(H_t),   W_fc [d, m*d] dtype, y [n_tokens, d] dtype.
- * Runs on the tcgen05 GEMM.  Workspace: hdf_fc_reduce_workspace_size(). */
-HDF_API size_t hdf_fc_reduce_workspace_size(int64_t n_tokens, int m, int d, int dtype);
-HDF_API int hdf_fc_reduce(const void* H, int dtype, int64_t n_tokens, int m, int d,
+ * the comparison path and the fallback the paper names for when the
+ * reducer's assumptions fail (a source other than the pre-collapse residual,
+ * or a drafter width d_out that differs from the target width d_in):
+ *   y_t = W_fc vec(H_t),   H [n_tokens, m, d_in], W_fc [d_out, m*d_in],
+ *   y [n_tokens, d_out], all dtype; vec() path-major as in Eq. 1.
+ * Needs d_out % 128 == 0 and m * d_in * sizeof(dtype) % 16 == 0.  Runs on the
+ * tcgen05 GEMM (fp32 accumulation; tf32 inputs for HDF_F32).  Workspace:
+ * hdf_fc_reduce_workspace_size() (currently 0 bytes). */
+HDF_API size_t hdf_fc_reduce_workspace_size(int64_t n_tokens, int m, int d_in, int d_out, int dtype);
+HDF_API int hdf_fc_reduce(const void* H, int dtype, int64_t n_tokens, int m, int d_in, int d_out,
                   const void* W_fc, void* y, void* ws, size_t ws_bytes,
                   hdf_stream_t stream);
 
@@ -436,8 +441,8 @@ HDF_API int hdf_accept_sample(const float* p_target, const float* q_draft, const
  * 1 / t_kd (teacher: the target LM head on the path-mean residual, which
  * hdf_gated_reduce gives with alpha_override = 1/m; student: the draft
  * logits of the first P block positions).  For a batch of blocks with P rows
- * each, kl_mean is the batch mean of L_KL.  L = L_CE + alpha * L_KL (Eq. 3)
- * is left to the caller.
+ * each, kl_mean is the batch mean of L_KL.  hdf_draft_loss below gives the
+ * whole objective of Eq. 3.
  *   ls_teacher, ls_student  [rows, V] fp32 (device), rows >= 0, V >= 1
  *   kl_rows                 [rows] fp32 or NULL
  *   kl_mean                 [1] fp32 or NULL
@@ -451,6 +456,43 @@ HDF_API size_t hdf_kl_distill_workspace_size(int64_t rows, int64_t V);
 HDF_API int hdf_kl_distill(const float* ls_teacher, const float* ls_student, int64_t rows, int64_t V,
                            float t_kd, float* kl_rows, float* kl_mean, void* ws, size_t ws_bytes,
                            hdf_stream_t stream);
+
+/* ------------------------------------------------------------------------
+ * (5') Training objective of the drafter — Eq. 3 with Eq. 2 (Sec. 2.3):
+ *   L = L_CE + alpha * L_KL
+ * over a batch of drafted blocks.  Block i's rows of the student are
+ * i*block + k (k = 0 the anchor slot, k >= 1 draft position k, which predicts
+ * the token at a + k, as hdf_lm_head_argmax lays them out).
+ *   L_CE  mean over every supervised draft position (i, k), k = 1..block-1, of
+ *         -log q_k(labels[i][k-1]) at temperature 1 (one-hot supervision)
+ *   L_KL  T_KD^2 / P * sum_{k=1..P} KL(p_k^T || q_k^T), averaged over the
+ *         blocks, p^T / q^T = softmax(ls / T_KD) of the teacher / student rows
+ *   ls_teacher [batch, P, V] fp32  log-softmax at temperature 1 of the
+ *              teacher LMHead(h_{a+k-1}), k = 1..P (the target LM head on the
+ *              path-mean residual: hdf_gated_reduce with alpha_override = 1/m,
+ *              then hdf_lm_head_argmax with inv_temp = 1); NULL when P == 0
+ *   ls_student [batch*block, V] fp32  log-softmax at temperature 1 of the
+ *              draft logits (hdf_lm_head_argmax, inv_temp = 1)
+ *   labels     [batch, block-1] int32 device: true token of each draft
+ *              position; < 0 = unsupervised.  A label >= V is a contract
+ *              violation: the position is left out and HDF_ERR_DEVICE_CHECK
+ *              is recorded in the device status word.
+ *   ce_rows    [batch, block-1] fp32 or NULL: per-position CE (NaN where
+ *              unsupervised);  kl_rows [batch, P] fp32 or NULL
+ *   loss       [3] fp32 device: {L, L_CE, L_KL}; L_CE = 0 when no position
+ *              is supervised
+ *   ws         hdf_draft_loss_workspace_size(batch, P, V) bytes, 256-byte
+ *              aligned (0 bytes when P == 0)
+ * Both log-softmax inputs must be normalised at temperature 1: the KL part
+ * renormalises them at T_KD in its single pass, the CE part reads one entry.
+ * 0 <= P <= block - 1 (the paper supervises P = 2), 2 <= block <= 64,
+ * batch * block <= 65535.  Every sum runs in a fixed order (bitwise
+ * reproducible); identical teacher and student rows give L_KL = 0 exactly.
+ * ---------------------------------------------------------------------- */
+HDF_API size_t hdf_draft_loss_workspace_size(int batch, int P, int64_t V);
+HDF_API int hdf_draft_loss(const float* ls_teacher, const float* ls_student, const int32_t* labels, int batch,
+                           int block, int P, int64_t V, float t_kd, float alpha, float* ce_rows, float* kl_rows,
+                           float* loss, void* ws, size_t ws_bytes, hdf_stream_t stream);
 
 #ifdef __cplusplus
 }

@@ -479,5 +479,5 @@ def draft_loss(teacher_logits, student_logits, labels, *, block: int, P: int = 2
             lq = _log_softmax(S[i * block + k] / t_kd)
             p = np.exp(lp)
             kl_rows[i, k - 1] = np.sum(np.where(p > 0, p * (lp - lq), 0.0))
-    l_kl = float(t_kd * t_kd / P * np.sum(kl_rows) / batch)
+    l_kl = float(t_kd * t_kd / P * np.sum(kl_rows) / batch) if P else 0.0  # no position distilled: empty sum
     return {"loss": l_ce + alpha * l_kl, "ce": l_ce, "kl": l_kl, "ce_rows": ce, "kl_rows": kl_rows.reshape(-1)}

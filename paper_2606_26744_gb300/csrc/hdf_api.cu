@@ -288,7 +288,7 @@ int check_draft_shape(const hdf_draft_shape* sh) {
 // =====================================================================
 extern "C" {
 
-int hdf_version(void) { return 100; }
+int hdf_version(void) { return 101; }
 
 const char* hdf_status_str(int s) {
   switch (s) {
@@ -469,32 +469,34 @@ int hdf_gated_reduce_kernel(int path, const void* H, int dtype, int64_t n_tokens
 }
 
 // -------------------------------------------------------- fc comparison
-size_t hdf_fc_reduce_workspace_size(int64_t, int, int, int) { return 0; }
+size_t hdf_fc_reduce_workspace_size(int64_t, int, int, int, int) { return 0; }
 
-int hdf_fc_reduce(const void* H, int dtype, int64_t n_tokens, int m, int d, const void* W_fc, void* y, void*,
-                  size_t, hdf_stream_t stream) {
+int hdf_fc_reduce(const void* H, int dtype, int64_t n_tokens, int m, int d_in, int d_out, const void* W_fc, void* y,
+                  void*, size_t, hdf_stream_t stream) {
   g_err.clear();
   if (dtype != HDF_BF16 && dtype != HDF_F32) return fail(HDF_ERR_DTYPE, "dtype %d", dtype);
-  if (n_tokens < 0 || m < 1 || d <= 0 || d % 128) return fail(HDF_ERR_SHAPE, "need d %% 128 == 0");
-  if ((long long)m * d * esize(dtype) % 16) return fail(HDF_ERR_SHAPE, "row stride");
+  if (n_tokens < 0 || m < 1 || d_in <= 0 || d_out <= 0 || d_out % 128)
+    return fail(HDF_ERR_SHAPE, "need m >= 1, d_in > 0 and d_out %% 128 == 0 (m %d, d_in %d, d_out %d)", m, d_in,
+                d_out);
+  if ((long long)m * d_in * esize(dtype) % 16) return fail(HDF_ERR_SHAPE, "row stride m * d_in not 16-byte aligned");
   if (n_tokens == 0) return HDF_OK;
   if (!H || !W_fc || !y) return fail(HDF_ERR_INVALID_ARG, "null pointer");
   if (!aligned16(H) || !aligned16(W_fc) || !aligned16(y)) return fail(HDF_ERR_ALIGNMENT, "alignment");
   if (n_tokens > 0x7fffffffLL) return fail(HDF_ERR_SHAPE, "n_tokens too large");
-  const long long K = (long long)m * d;
-  SplitPlan p{d % 256 == 0 ? 256 : 128, 1, 0};
+  const long long K = (long long)m * d_in;
+  SplitPlan p{d_out % 256 == 0 ? 256 : 128, 1, 0};
   GemmArgs g;
-  init_gemm(g, dtype, n_tokens, d, K, p);
+  init_gemm(g, dtype, n_tokens, d_out, K, p);
   g.group_n = 8;
   g.pair = use_pair_tiles(dtype, p.bn, n_tokens);
   int rc;
   if ((rc = make_map(&g.A.map[0], H, dtype, n_tokens, K, K, 64))) return rc;
-  if ((rc = make_map(&g.B.map[0], W_fc, dtype, d, K, K, g.pair ? 128 : p.bn))) return rc;
+  if ((rc = make_map(&g.B.map[0], W_fc, dtype, d_out, K, K, g.pair ? 128 : p.bn))) return rc;
   g.pre_operand = 2;  // the weight
   g.epi.kind = kEpiStore;
   g.epi.out[0] = y;
-  g.epi.seg_width = d;
-  g.epi.ld = d;
+  g.epi.seg_width = d_out;
+  g.epi.ld = d_out;
   CK(launch_gemm(g, (cudaStream_t)stream), "fc gemm launch");
   return HDF_OK;
 }
@@ -1096,6 +1098,36 @@ int hdf_kl_distill(const float* ls_teacher, const float* ls_student, int64_t row
   CK(launch_kl_distill(ls_teacher, ls_student, rows, V, t_kd, kl_rows, kl_mean, static_cast<float*>(ws),
                        (cudaStream_t)stream),
      "kl distill");
+  return HDF_OK;
+}
+
+// ------------------------------------------------ training objective, Eq. 3
+size_t hdf_draft_loss_workspace_size(int batch, int P, int64_t V) {
+  if (batch <= 0 || P <= 0 || V <= 0) return 0;
+  return up256((size_t)loss_partial_floats(batch, P, V) * 4);
+}
+
+int hdf_draft_loss(const float* ls_teacher, const float* ls_student, const int32_t* labels, int batch, int block,
+                   int P, int64_t V, float t_kd, float alpha, float* ce_rows, float* kl_rows, float* loss, void* ws,
+                   size_t ws_bytes, hdf_stream_t stream) {
+  g_err.clear();
+  if (batch < 0 || block < 2 || block > 64 || P < 0 || P > block - 1 || V <= 0 || V > ((int64_t)1 << 31))
+    return fail(HDF_ERR_SHAPE, "need batch >= 0, 2 <= block <= 64, 0 <= P <= block - 1, 0 < V <= 2^31 (batch %d, "
+                "block %d, P %d, V %lld)", batch, block, P, (long long)V);
+  if ((int64_t)batch * block > 65535) return fail(HDF_ERR_SHAPE, "batch * block above 65535");
+  if (!(t_kd > 0) || !std::isfinite(t_kd)) return fail(HDF_ERR_INVALID_ARG, "t_kd must be finite and > 0");
+  if (!std::isfinite(alpha)) return fail(HDF_ERR_INVALID_ARG, "alpha must be finite");
+  if (batch == 0) return HDF_OK;
+  if (!ls_student || !labels || !loss || (P > 0 && !ls_teacher))
+    return fail(HDF_ERR_INVALID_ARG, "ls_student, labels, loss (and ls_teacher when P > 0) are required");
+  if (!aligned16(ls_student) || (P > 0 && !aligned16(ls_teacher)))
+    return fail(HDF_ERR_ALIGNMENT, "ls_teacher and ls_student must be 16-byte aligned");
+  const size_t need = hdf_draft_loss_workspace_size(batch, P, V);
+  if (need && (!ws || ws_bytes < need || (reinterpret_cast<uintptr_t>(ws) & 255)))
+    return fail(HDF_ERR_WORKSPACE, "workspace %zu bytes (need %zu, 256-byte aligned)", ws_bytes, need);
+  CK(launch_draft_loss(ls_teacher, ls_student, labels, batch, block, P, V, t_kd, alpha, ce_rows, kl_rows, loss,
+                       static_cast<float*>(ws), device_status_ptr(), (cudaStream_t)stream),
+     "draft loss");
   return HDF_OK;
 }
 

@@ -185,6 +185,11 @@ int kl_chunks(long long V);
 // partial: [rows, kl_chunks(V)] fp32 scratch
 cudaError_t launch_kl_distill(const float* lt, const float* ls, long long rows, long long V, float t_kd,
                               float* kl_rows, float* kl_mean, float* partial, cudaStream_t s);
+// Eq. 3 over a batch of blocks; partial: loss_partial_floats() fp32 scratch
+int loss_partial_floats(int batch, int P, long long V);
+cudaError_t launch_draft_loss(const float* lt, const float* ls, const int* labels, int batch, int block, int P,
+                              long long V, float t_kd, float alpha, float* ce_rows, float* kl_rows, float* loss,
+                              float* partial, int* status, cudaStream_t s);
 
 // -------------------------------------------------------- attention ----
 struct AttnArgs {

@@ -73,8 +73,8 @@ _SIGS = {
     "hdf_gated_reduce_backward_workspace_size": (c_size, [c_i64, c_int, c_int, c_int]),
     "hdf_gated_reduce_backward": (c_int, [c_vp, c_int, c_i64, c_int, c_int, c_vp, c_vp, c_float, c_float,
                                           c_vp, c_vp, c_vp, c_vp, c_size, c_vp]),
-    "hdf_fc_reduce_workspace_size": (c_size, [c_i64, c_int, c_int, c_int]),
-    "hdf_fc_reduce": (c_int, [c_vp, c_int, c_i64, c_int, c_int, c_vp, c_vp, c_vp, c_size, c_vp]),
+    "hdf_fc_reduce_workspace_size": (c_size, [c_i64, c_int, c_int, c_int, c_int]),
+    "hdf_fc_reduce": (c_int, [c_vp, c_int, c_i64, c_int, c_int, c_int, c_vp, c_vp, c_vp, c_size, c_vp]),
     "hdf_draft_block_workspace_size": (c_size, [ctypes.POINTER(DraftShape)]),
     "hdf_draft_block": (c_int, [ctypes.POINTER(DrafterWeights), ctypes.POINTER(DraftShape), c_vp, c_vp,
                                 c_vp, c_vp, c_vp, c_size, ctypes.POINTER(Trace), c_vp]),
@@ -98,6 +98,9 @@ _SIGS = {
     "hdf_accept_sample": (c_int, [c_vp, c_vp, c_vp, c_i64, c_vp, c_vp, c_int, c_int, c_i64, c_vp, c_vp, c_vp]),
     "hdf_kl_distill_workspace_size": (c_size, [c_i64, c_i64]),
     "hdf_kl_distill": (c_int, [c_vp, c_vp, c_i64, c_i64, c_float, c_vp, c_vp, c_vp, c_size, c_vp]),
+    "hdf_draft_loss_workspace_size": (c_size, [c_int, c_int, c_i64]),
+    "hdf_draft_loss": (c_int, [c_vp, c_vp, c_vp, c_int, c_int, c_int, c_i64, c_float, c_float, c_vp, c_vp, c_vp,
+                               c_vp, c_size, c_vp]),
 }
 
 _lib = None
@@ -197,14 +200,18 @@ def hdf_gated_reduce(H: torch.Tensor, Wf: Optional[torch.Tensor], b: Optional[to
 
 def hdf_fc_reduce(H: torch.Tensor, W_fc: torch.Tensor, y: Optional[torch.Tensor] = None,
                   stream=None) -> torch.Tensor:
-    """Generic fc collapse y = vec(H) W_fc^T (comparison path)."""
-    N, m, d = H.shape
+    """Generic fc collapse y = vec(H) W_fc^T, H [N, m, d_in], W_fc [d_out, m*d_in]
+    (the comparison path, and the fallback for unequal widths)."""
+    N, m, d_in = H.shape
+    d_out = W_fc.shape[0]
+    if W_fc.shape[1] != m * d_in:
+        raise ValueError(f"W_fc is {tuple(W_fc.shape)}, expected [d_out, {m * d_in}]")
     if y is None:
-        y = torch.empty((N, d), dtype=H.dtype, device=H.device)
+        y = torch.empty((N, d_out), dtype=H.dtype, device=H.device)
     lib = load()
-    wsb = lib.hdf_fc_reduce_workspace_size(N, m, d, _dtype(H))
+    wsb = lib.hdf_fc_reduce_workspace_size(N, m, d_in, d_out, _dtype(H))
     ws = torch.empty(max(wsb, 1), dtype=torch.uint8, device=H.device)
-    _check(lib.hdf_fc_reduce(_p(H), _dtype(H), N, m, d, _p(W_fc), _p(y), _p(ws), wsb, _stream(stream)))
+    _check(lib.hdf_fc_reduce(_p(H), _dtype(H), N, m, d_in, d_out, _p(W_fc), _p(y), _p(ws), wsb, _stream(stream)))
     return y
 
 
@@ -440,6 +447,36 @@ def hdf_kl_distill(ls_teacher: torch.Tensor, ls_student: torch.Tensor, *, t_kd: 
     _check(lib.hdf_kl_distill(_p(ls_teacher), _p(ls_student), rows, V, t_kd, _p(kl_rows), _p(kl_mean), _p(ws),
                               ws.numel(), _stream(stream)))
     return kl_rows, kl_mean
+
+
+# ------------------------------------------------ training objective, Eq. 3
+def hdf_draft_loss(ls_teacher: Optional[torch.Tensor], ls_student: torch.Tensor, labels: torch.Tensor, *,
+                   block: int, t_kd: float = 1.0, alpha: float = 0.1, ce_rows: Optional[torch.Tensor] = None,
+                   kl_rows: Optional[torch.Tensor] = None, loss: Optional[torch.Tensor] = None,
+                   ws: Optional[torch.Tensor] = None, stream=None):
+    """Eq. 3, L = L_CE + alpha * L_KL: ls_teacher [batch, P, V] (or None for
+    P = 0) and ls_student [batch * block, V] fp32 log-softmax rows at
+    temperature 1, labels [batch, block - 1] int32 (< 0 = unsupervised).
+    Returns (loss [3] = {L, L_CE, L_KL}, ce_rows [batch, block-1], kl_rows
+    [batch, P])."""
+    V = ls_student.shape[1]
+    batch = ls_student.shape[0] // block
+    P = 0 if ls_teacher is None else ls_teacher.shape[1]
+    dev = ls_student.device
+    if ce_rows is None:
+        ce_rows = torch.empty((batch, block - 1), dtype=torch.float32, device=dev)
+    if kl_rows is None:
+        kl_rows = torch.empty((batch, max(P, 1)), dtype=torch.float32, device=dev)
+    if loss is None:
+        loss = torch.empty((3,), dtype=torch.float32, device=dev)
+    lib = load()
+    need = lib.hdf_draft_loss_workspace_size(batch, P, V)
+    if ws is None:
+        ws = torch.empty(max(need, 1), dtype=torch.uint8, device=dev)
+    _check(lib.hdf_draft_loss(_p(ls_teacher) if P > 0 else None, _p(ls_student), _p(labels), batch, block, P, V,
+                              t_kd, alpha, _p(ce_rows), _p(kl_rows) if P > 0 else None, _p(loss), _p(ws),
+                              ws.numel(), _stream(stream)))
+    return loss, ce_rows, kl_rows[:, :P]
 
 
 # ------------------------------------------------------ T = 1 verification

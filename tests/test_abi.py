@@ -26,7 +26,7 @@ def test_every_declared_symbol_is_exported(lib):
 
 
 def test_status_strings(lib):
-    assert lib.hdf_version() == 100
+    assert lib.hdf_version() == 101
     assert lib.hdf_status_str(0) == b"ok"
     assert b"aligned" in lib.hdf_status_str(4)
 
@@ -102,6 +102,40 @@ def test_kl_host_validation(lib):
     assert lib.hdf_kl_distill(v(16), v(24), 2, 100, 1.0, None, None, v(256), 4096, None) == 4  # alignment
     assert lib.hdf_kl_distill(v(16), v(16), 2, 100, 1.0, None, None, None, 0, None) == 5       # workspace
     assert lib.hdf_kl_distill_workspace_size(2, 8193) == 256                                   # 2 x 2 partials
+
+
+def test_draft_loss_host_validation(lib):
+    v = ctypes.c_void_p
+    ws = v(256)
+
+    def call(lt=16, ls=16, lab=16, batch=2, block=16, P=2, V=1000, t=1.0, a=0.1, loss=16, w=ws, wb=1 << 20):
+        p = lambda x: None if x is None else (x if isinstance(x, ctypes.c_void_p) else v(x))
+        return lib.hdf_draft_loss(p(lt), p(ls), p(lab), batch, block, P, V, t, a, None, None, p(loss), p(w), wb,
+                                  None)
+    assert call(block=1) == 2                    # block < 2
+    assert call(P=16) == 2                       # P > block - 1
+    assert call(V=0) == 2
+    assert call(t=0.0) == 1                      # t_kd <= 0
+    assert call(a=float("nan")) == 1
+    assert call(batch=0, lt=None, ls=None, lab=None, loss=None, w=None, wb=0) == 0   # empty batch
+    assert call(lt=None) == 1                    # teacher needed when P > 0
+    assert call(lt=None, P=0, ls=24, w=None, wb=0) == 4   # ... not when P == 0 (the next check fires)
+    assert call(lab=None) == 1
+    assert call(ls=24) == 4                      # alignment
+    assert call(w=None, wb=0) == 5               # workspace
+    assert call(w=v(300)) == 5                   # not 256-byte aligned
+    assert lib.hdf_draft_loss_workspace_size(2, 2, 8193) == 256       # 4 rows x 2 chunks x 5 floats
+    assert lib.hdf_draft_loss_workspace_size(2, 0, 8193) == 0
+
+
+def test_fc_reduce_host_validation(lib):
+    v = ctypes.c_void_p
+    assert lib.hdf_fc_reduce(v(16), 1, 4, 4, 64, 100, v(16), v(16), None, 0, None) == 2     # d_out % 128
+    assert lib.hdf_fc_reduce(v(16), 1, 4, 3, 7, 128, v(16), v(16), None, 0, None) == 2      # row stride
+    assert lib.hdf_fc_reduce(v(16), 9, 4, 4, 64, 128, v(16), v(16), None, 0, None) == 3     # dtype
+    assert lib.hdf_fc_reduce(None, 1, 0, 4, 7168, 4096, None, None, None, 0, None) == 0     # empty
+    assert lib.hdf_fc_reduce(None, 1, 4, 4, 7168, 4096, v(16), v(16), None, 0, None) == 1
+    assert lib.hdf_fc_reduce(v(24), 1, 4, 4, 7168, 4096, v(16), v(16), None, 0, None) == 4
 
 
 def test_lm_head_and_accept_host_validation(lib):

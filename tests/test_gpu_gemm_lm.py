@@ -42,6 +42,39 @@ def test_fc_reduce_large_width_sampled_rows():
     assert rowwise_rel(to64(y[rows.cuda()]), ref) <= TOL_BF16
 
 
+@pytest.mark.parametrize("N,m,d_in,d_out,dtype", [
+    (300, 4, 200, 640, torch.bfloat16),    # narrower input, 128-wide tiles, K tail of 32
+    (64, 2, 96, 256, torch.float32),       # tf32, wider output
+    (7, 4, 4096, 7168, torch.bfloat16),    # a few rows, target 4096 -> drafter 7168
+])
+def test_fc_reduce_unequal_widths(N, m, d_in, d_out, dtype):
+    """The fc fallback when the drafter width differs from the target's
+    (Sec. 2.2): W_fc [d_out, m * d_in], against the oracle's fc_reduce."""
+    H = _rand((N, m, d_in), 1.0, dtype, 5 + N)
+    Wfc = _rand((d_out, m * d_in), 0.02, dtype, 6 + d_out)
+    y = hdf.hdf_fc_reduce(H.cuda(), Wfc.cuda())
+    torch.cuda.synchronize()
+    assert hdf.device_status() == 0
+    assert y.shape == (N, d_out)
+    out = "bf16" if dtype == torch.bfloat16 else "f32"
+    ref = O.fc_reduce(to64(H), to64(Wfc), out)
+    assert rowwise_rel(to64(y), ref) <= (TOL_BF16 if out == "bf16" else TOL_F32_TF32)
+
+
+def test_fc_reduce_7168_to_4096_sampled_rows():
+    """Target width 7168 into a 4096-wide drafter on 1024 tokens (CTA-pair
+    tiles), every column of 8 sampled rows against the oracle."""
+    N, m, d_in, d_out = 1024, 4, 7168, 4096
+    H = _rand((N, m, d_in), 1.0, torch.bfloat16, 7, "cuda")
+    Wfc = _rand((d_out, m * d_in), 0.02, torch.bfloat16, 8, "cuda")
+    y = hdf.hdf_fc_reduce(H, Wfc)
+    torch.cuda.synchronize()
+    assert hdf.device_status() == 0
+    rows = torch.tensor([0, 255, 256, 511, 1023, 700, 33, 901], device="cuda")
+    ref = O.fc_reduce(to64(H[rows]), to64(Wfc), "bf16")
+    assert rowwise_rel(to64(y[rows]), ref) <= TOL_BF16
+
+
 @pytest.mark.parametrize("M,d,V,dtype,it,ls", [
     (8, 256, 1024, torch.float32, 1.0, True),     # tiny workload shape
     (16, 2048, 32768, torch.bfloat16, 1.0, False),  # decode shape

@@ -86,3 +86,101 @@ def test_kl_teacher_from_path_mean_and_lm_head():
     zs = O.lm_head(to64(h_s), to64(W_lm))["z"]
     ref = O.kl_distill(zt, zs, t_kd)
     np.testing.assert_allclose(float(m[0]), ref, rtol=2e-3, atol=1e-6)
+
+
+# -------------------------------------------------- Eq. 3: L = L_CE + alpha L_KL
+def _loss_inputs(batch, block, P, V, seed, unsup=0.2):
+    """Student and teacher log-softmax rows at temperature 1 (fp32) and labels
+    with a share of unsupervised (-1) positions."""
+    g = torch.Generator().manual_seed(seed)
+    zs = torch.randn(batch * block, V, generator=g, dtype=torch.float64) * 3
+    zt = torch.stack([zs[i * block + 1:i * block + 1 + P] for i in range(batch)]) + \
+        torch.randn(batch, P, V, generator=g, dtype=torch.float64)
+    ls_s = torch.log_softmax(zs, dim=-1).float()
+    ls_t = torch.log_softmax(zt, dim=-1).float()
+    labels = torch.randint(0, V, (batch, block - 1), generator=g, dtype=torch.int32)
+    labels[torch.rand(batch, block - 1, generator=g) < unsup] = -1
+    return ls_t, ls_s, labels
+
+
+def _check_loss(ls_t, ls_s, labels, block, t_kd, alpha, out):
+    loss, ce_rows, kl_rows = out
+    ref = O.draft_loss(to64(ls_t), to64(ls_s), labels.numpy(), block=block, P=ls_t.shape[1], t_kd=t_kd, alpha=alpha)
+    ce = to64(ce_rows).reshape(-1)
+    sup = labels.numpy().reshape(-1) >= 0
+    assert np.all(np.isnan(ce[~sup]))
+    np.testing.assert_allclose(ce[sup], ref["ce_rows"][sup], rtol=1e-5, atol=1e-5)
+    np.testing.assert_allclose(to64(kl_rows).reshape(-1), ref["kl_rows"], rtol=1e-4, atol=1e-6)
+    np.testing.assert_allclose(to64(loss), [ref["loss"], ref["ce"], ref["kl"]], rtol=1e-4, atol=1e-6)
+
+
+@pytest.mark.parametrize("batch,block,P,V,t_kd,alpha", [
+    (1, 8, 2, 1024, 1.0, 0.1),        # tiny workload's block and vocabulary
+    (1, 16, 2, 32768, 2.0, 0.2),      # decode
+    (3, 5, 4, 1001, 0.5, 1.0),        # ragged vocabulary (no 16-byte rows), P = block - 1
+    (8, 16, 2, 129280, 1.0, 0.15),    # large workload
+    (2, 16, 0, 4099, 1.0, 0.1),       # CE alone
+    (5, 3, 1, 8193, 3.0, 0.0),        # a chunk of one vector past 8192
+])
+def test_draft_loss_matches_oracle(batch, block, P, V, t_kd, alpha):
+    ls_t, ls_s, labels = _loss_inputs(batch, block, P, V, seed=batch * 1000 + V)
+    out = hdf.hdf_draft_loss(ls_t.cuda() if P else None, ls_s.cuda(), labels.cuda(), block=block, t_kd=t_kd,
+                             alpha=alpha)
+    torch.cuda.synchronize()
+    assert hdf.device_status() == 0
+    _check_loss(ls_t, ls_s, labels, block, t_kd, alpha, out)
+
+
+def test_draft_loss_exact_properties():
+    """KL exactly 0 for a teacher equal to the student's first P draft rows;
+    two calls give the same bits; a label past the vocabulary is left out and
+    recorded in the device status word; no supervised position gives L_CE 0."""
+    batch, block, P, V = 4, 16, 2, 50000
+    _, ls_s, labels = _loss_inputs(batch, block, P, V, seed=9)
+    ls_t = torch.stack([ls_s[i * block + 1:i * block + 1 + P] for i in range(batch)])
+    d_t, d_s, d_l = ls_t.cuda(), ls_s.cuda(), labels.cuda()
+    a = hdf.hdf_draft_loss(d_t, d_s, d_l, block=block, t_kd=2.0, alpha=0.5)
+    b = hdf.hdf_draft_loss(d_t, d_s, d_l, block=block, t_kd=2.0, alpha=0.5)
+    torch.cuda.synchronize()
+    assert float(a[0][2]) == 0.0 and torch.all(a[2] == 0)
+    assert torch.equal(a[0], b[0]) and torch.equal(a[1].nan_to_num(), b[1].nan_to_num())
+    assert float(a[0][0]) == float(a[0][1])                     # L = L_CE when L_KL = 0
+    assert hdf.device_status() == 0
+    bad = d_l.clone()
+    bad[1, 3] = V                                              # outside the vocabulary
+    loss, ce_rows, _ = hdf.hdf_draft_loss(d_t, d_s, bad, block=block, t_kd=2.0, alpha=0.5)
+    torch.cuda.synchronize()
+    assert hdf.load().hdf_device_status(1) != 0                 # recorded (and cleared)
+    assert torch.isnan(ce_rows[1, 3])
+    keep = labels.clone()
+    keep[1, 3] = -1
+    ref = O.draft_loss(to64(ls_t), to64(ls_s), keep.numpy(), block=block, P=P, t_kd=2.0, alpha=0.5)
+    np.testing.assert_allclose(float(loss[1]), ref["ce"], rtol=1e-5)
+    none = torch.full_like(d_l, -1)
+    loss0, _, _ = hdf.hdf_draft_loss(d_t, d_s, none, block=block, t_kd=2.0, alpha=0.5)
+    torch.cuda.synchronize()
+    assert float(loss0[1]) == 0.0
+    assert hdf.device_status() == 0
+
+
+def test_draft_loss_from_the_lm_heads():
+    """The whole objective from hidden rows: the student is the GPU LM head on
+    draft hidden rows, the teacher the LM head on the path-mean residual
+    (hdf_gated_reduce with alpha = 1/m), both log-softmax at temperature 1;
+    checked against the oracle fed the same bf16 hidden rows."""
+    batch, block, P, d, V, m = 2, 8, 2, 256, 1024, 4
+    g = torch.Generator().manual_seed(21)
+    W_lm = (torch.randn(V, d, generator=g) * 0.05).to(torch.bfloat16)
+    h_s = torch.randn(batch * block, d, generator=g).to(torch.bfloat16)
+    H = torch.randn(batch * P, m, d, generator=g).to(torch.bfloat16)
+    labels = torch.randint(0, V, (batch, block - 1), generator=g, dtype=torch.int32)
+    h_t = hdf.hdf_gated_reduce(H.cuda(), None, None, alpha_override=torch.full((batch * P, m), 1 / m, device="cuda"))
+    _, _, ls_t = hdf.hdf_lm_head_argmax(h_t, W_lm.cuda(), inv_temp=1.0, logsoftmax=True)
+    _, _, ls_s = hdf.hdf_lm_head_argmax(h_s.cuda(), W_lm.cuda(), inv_temp=1.0, logsoftmax=True)
+    loss, _, _ = hdf.hdf_draft_loss(ls_t.view(batch, P, V), ls_s, labels.cuda(), block=block, t_kd=2.0, alpha=0.2)
+    torch.cuda.synchronize()
+    assert hdf.device_status() == 0
+    zt = O.lm_head(to64(h_t), to64(W_lm))["z"].reshape(batch, P, V)
+    zs = O.lm_head(to64(h_s), to64(W_lm))["z"]
+    ref = O.draft_loss(zt, zs, labels.numpy(), block=block, P=P, t_kd=2.0, alpha=0.2)
+    np.testing.assert_allclose(to64(loss), [ref["loss"], ref["ce"], ref["kl"]], rtol=2e-3, atol=1e-5)

@@ -109,11 +109,11 @@ MUTATIONS = {
         "lq = _log_softmax(S[i * block + k] / t_kd)",
         "lq = _log_softmax(S[i * block + k - 1] / t_kd)"),
     "loss KL without the temperature-squared factor": (
-        "l_kl = float(t_kd * t_kd / P * np.sum(kl_rows) / batch)",
-        "l_kl = float(1.0 / P * np.sum(kl_rows) / batch)"),
+        "l_kl = float(t_kd * t_kd / P * np.sum(kl_rows) / batch) if P",
+        "l_kl = float(1.0 / P * np.sum(kl_rows) / batch) if P"),
     "loss KL summed over the batch instead of averaged": (
-        "l_kl = float(t_kd * t_kd / P * np.sum(kl_rows) / batch)",
-        "l_kl = float(t_kd * t_kd / P * np.sum(kl_rows))"),
+        "l_kl = float(t_kd * t_kd / P * np.sum(kl_rows) / batch) if P",
+        "l_kl = float(t_kd * t_kd / P * np.sum(kl_rows)) if P"),
     "loss KL weight applied to CE": (
         'return {"loss": l_ce + alpha * l_kl,',
         'return {"loss": alpha * l_ce + l_kl,'),
