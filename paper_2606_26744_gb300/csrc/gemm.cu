@@ -722,7 +722,34 @@ __global__ void __launch_bounds__(128, 1) gemm_pair_kernel(const __grid_constant
   tc_fence_after();
   const uint32_t tmem = tmem_slot;
 
-  if (!(warp == 0 && lane == 0)) pdl_wait();  // the producer waits after its weight prefetch
+  // This thread's output row, RoPE position and (head_dim 128, RoPE tiles)
+  // the 64 cos and 64 sin entries of that position, loaded into registers
+  // while the mainloop runs, so the epilogue waits on no global load.
+  const Epilogue& E = g.epi;
+  const long long t = (long long)my_m * BM + tid;
+  const int seg_t = (tile_n * BN) / E.seg_width;
+  const bool rope_regs = E.kind == kEpiStore && E.head_dim == 128 && ((E.rope_mask >> seg_t) & 1) &&
+                         (E.seg_width % BN) == 0;
+  int spos = 0;
+  long long srow = -1;
+  float4 rc[16], rs[16];
+  auto row_prefetch = [&]() {
+    srow = t < g.M ? ctx_store_row(E, t, &spos, g.status) : -1;
+    if (rope_regs && srow >= 0) {
+      const int pos = (int)min((long long)spos, E.rope_rows - 1);
+      const float4* cp = reinterpret_cast<const float4*>(E.rope_cos + (size_t)pos * 64);
+      const float4* sp = reinterpret_cast<const float4*>(E.rope_sin + (size_t)pos * 64);
+#pragma unroll
+      for (int i = 0; i < 16; ++i) {
+        rc[i] = __ldg(cp + i);
+        rs[i] = __ldg(sp + i);
+      }
+    }
+  };
+  if (!(warp == 0 && lane == 0)) {
+    pdl_wait();  // the producer waits after its weight prefetch
+    row_prefetch();
+  }
   if (warp == 0 && lane == 0) {
     // ------------------------------------------------ TMA producer (both CTAs)
     auto full_of = [&](int st) { return map_rank(smem_u32(&full_bar[st]), 0u); };
@@ -776,6 +803,7 @@ __global__ void __launch_bounds__(128, 1) gemm_pair_kernel(const __grid_constant
         mbar_wait(smem_u32(&full_bar[ss]), pp, nullptr);
       }
     }
+    row_prefetch();  // the last loads are issued a few stages before the mainloop ends
   } else if (warp == 1 && lane == 0 && leader) {
     // ------------------------------------------------ MMA issuer (rank 0)
     int s = 0;
@@ -806,10 +834,31 @@ __global__ void __launch_bounds__(128, 1) gemm_pair_kernel(const __grid_constant
     pair_abort = abort_flag | ld_dsmem_s32(map_rank(smem_u32((const void*)&abort_flag), rank ^ 1u));
   __syncthreads();
   const uint32_t taddr = tmem + ((uint32_t)(warp * 32) << 16);
-  int spos = 0;
-  const long long t = (long long)my_m * BM + tid;
-  const long long srow = t < g.M ? ctx_store_row(g.epi, t, &spos, g.status) : -1;
-  if (!pair_abort && num_kb > 0) {
+  if (!pair_abort && num_kb > 0 && rope_regs) {
+    // the tile is one segment and two whole heads: chunk c holds pairs
+    // 8 (c % 8) .. 8 (c % 8) + 7 of its head
+    const int col_t = tile_n * BN;
+    const int fl0 = col_t - seg_t * E.seg_width;
+    __nv_bfloat16* out = reinterpret_cast<__nv_bfloat16*>(E.out[seg_t]);
+#pragma unroll
+    for (int c = 0; c < BN / 16; ++c) {
+      float v[16];
+      tmem_ld16(taddr + 16 * c, v);
+      if (srow >= 0 && col_t + 16 * c < g.N) {
+        const float4 c0v = rc[2 * (c % 8)], c1v = rc[2 * (c % 8) + 1];
+        const float4 s0v = rs[2 * (c % 8)], s1v = rs[2 * (c % 8) + 1];
+        const float cs[8] = {c0v.x, c0v.y, c0v.z, c0v.w, c1v.x, c1v.y, c1v.z, c1v.w};
+        const float sn[8] = {s0v.x, s0v.y, s0v.z, s0v.w, s1v.x, s1v.y, s1v.z, s1v.w};
+#pragma unroll
+        for (int i = 0; i < 8; ++i) {
+          const float x0 = v[2 * i], x1 = v[2 * i + 1];
+          v[2 * i] = x0 * cs[i] - x1 * sn[i];
+          v[2 * i + 1] = x0 * sn[i] + x1 * cs[i];
+        }
+        store16<__nv_bfloat16>(out + srow * E.ld + fl0 + 16 * c, v);
+      }
+    }
+  } else if (!pair_abort && num_kb > 0) {
     const float* rope_row = stage_rope_row<BN>(g, my_m, tile_n, smem, spos);
 #pragma unroll 1
     for (int c0 = 0; c0 < BN; c0 += 16) {
