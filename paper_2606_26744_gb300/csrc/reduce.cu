@@ -812,16 +812,17 @@ cudaError_t launch_gated_reduce_cluster(const ReduceArgs& a, const CUtensorMap* 
 // ===========================================================================
 // bf16 tile path (persistent, warp-specialised).
 //
-// A cluster of S CTAs (S = 4, or 8 when d is wide) walks tiles of T = 32 (or
-// 16, for wide slices) consecutive tokens; CTA rank c owns elements [c*E, (c+1)*E) of each of the
-// m paths (E = d/S), so its W_f slice (m x m*E) stays in shared memory.
-// Roles, meeting only at mbarriers:
+// A cluster of S CTAs (S = 4, or 8 when the slices would not fit) walks
+// tiles of T = 32 (or 16, for wide slices) consecutive tokens; CTA rank c
+// owns elements [c*E, (c+1)*E) of each of the m paths (E = d/S), so its W_f
+// slice (m x m*E) stays in shared memory.  Roles, meeting only at mbarriers:
 //   producer warp   streams pass 1 of every tile from HBM into a 128 KB ring:
 //                   one TMA box per stage from the 3-D view {64 elements,
-//                   tokens, 128-byte chunks} of H, 4 chunks (512 contiguous
-//                   bytes) of 32 tokens, landing as planes [32 tokens][64
-//                   elements] with the 128-byte swizzle; it never waits on
-//                   the gates, so HBM streaming continues across tiles
+//                   tokens, 128-byte chunks} of H, C chunks (C * 128
+//                   contiguous bytes, C = 4 or 8) of T tokens, landing as
+//                   planes [T tokens][64 elements] with the 128-byte
+//                   swizzle; it never waits on the gates, so HBM streaming
+//                   continues across tiles
 //   8 gate warps    (row tile of 16 tokens) x (box phase 0..3): the m gate
 //                   dots on mma.sync m16n8k16 (tokens are the rows, the W_f
 //                   slice is B) and the sums of squares from the same A
@@ -840,7 +841,6 @@ cudaError_t launch_gated_reduce_cluster(const ReduceArgs& a, const CUtensorMap* 
 // from HBM once, W_f once per CTA.  Every wait is time-limited.
 namespace {
 
-constexpr int TP_C = 4;                    // 128-byte chunks per token in a box
 constexpr int TP_RING = 128 * 1024;        // ring bytes
 constexpr int TP_MAXST = 16;               // ring slots at most (16-token tiles)
 constexpr int TP_NGW = 8;                  // gate warps: (sub, box phase 0..3)
@@ -853,7 +853,7 @@ constexpr int TP_NPH = TP_NGW / 2;         // box phases
 // barrier (an mbarrier parity wait tells adjacent phases apart only).
 constexpr int TP_NWW = 8;                  // weighted warps
 constexpr int TP_THR = 32 * (2 + TP_NGW + TP_NWW);
-constexpr int TP_LA = 2;                   // gate warps run at most this many tiles ahead of the alpha warp
+constexpr int TP_LA = 1;                   // gate warps run at most this many tiles ahead of the alpha warp
 constexpr int TP_NX = 2 * TP_LA + 2;       // exchange buffers
 constexpr int TP_NAB = 3;                  // alpha buffers
 constexpr int TP_PS = 8;                   // floats per token in an exchange row (m + 1 <= 5 used)
@@ -864,14 +864,15 @@ struct TileGeo {
   int t;     // tokens per tile (16 or 32)
   int ec;    // elements per path in a CTA slice (multiple of 64)
   int nkb;   // 128-byte chunks per path slice
-  int ngrp;  // boxes per path slice: ngrp - 1 of TP_C chunks, then one of tail chunks
-  int tail;  // chunks in the last box of a path slice (1..TP_C)
+  int c;     // 128-byte chunks per token in a box (4 or 8)
+  int ngrp;  // boxes per path slice: ngrp - 1 of c chunks, then one of tail chunks
+  int tail;  // chunks in the last box of a path slice (1..c)
   int wrow;  // row stride (elements) of the W_f slice in shared memory
   long long ntiles;
 };
 struct TileMaps {
-  CUtensorMap main;  // box {64, 32, TP_C}
-  CUtensorMap tail;  // box {64, 32, tail}
+  CUtensorMap main;  // box {64, T, c}
+  CUtensorMap tail;  // box {64, T, tail}
 };
 
 __device__ __forceinline__ void st_async_v4(uint32_t addr, float4 v, uint32_t bar) {
@@ -890,7 +891,7 @@ constexpr size_t tp_smem(int S, int T, int m, int wrow) {
 // T tokens per tile: 32 (two 16-row tiles; the two gate warps of a phase
 // take one each) or 16 (one row tile; the two gate warps of a phase take the
 // even and the odd planes of every box).
-template <int M, int S, int T>
+template <int M, int S, int T, int TP_C>
 __global__ void __launch_bounds__(TP_THR, 1) gated_reduce_tile_kernel(const ReduceArgs a,
                                                                       const __grid_constant__ TileMaps maps,
                                                                       const TileGeo geo) {
@@ -1226,10 +1227,10 @@ __global__ void __launch_bounds__(TP_THR, 1) gated_reduce_tile_kernel(const Redu
   cluster_sync_all();  // no rank still writes into this CTA's shared memory
 }
 
-template <int M, int S, int T>
+template <int M, int S, int T, int C>
 cudaError_t launch_tile_mst(const ReduceArgs& a, const TileGeo& geo, size_t smem, const TileMaps* maps,
                             cudaStream_t s) {
-  auto k = gated_reduce_tile_kernel<M, S, T>;
+  auto k = gated_reduce_tile_kernel<M, S, T, C>;
   static size_t cached_smem = 0;
   static int cached_clusters = 0;
   cudaError_t e;
@@ -1258,37 +1259,58 @@ cudaError_t launch_tile_mst(const ReduceArgs& a, const TileGeo& geo, size_t smem
   return launch_kernel(k, dim3((unsigned)(ncl * S)), dim3(TP_THR), smem, s, (unsigned)S, a, *maps, geo);
 }
 
+// The tile geometries (CTAs per cluster, tokens per tile, chunks per box),
+// in the order tile_geometry tries them, with the largest slice (bytes of
+// H a CTA holds per tile) each may take.
+struct TileShape {
+  int s, t, c;
+  int max_slice_kb;
+};
+constexpr TileShape kTileShapes[] = {{4, 32, 8, 160}, {4, 16, 8, 240}, {8, 16, 8, 240}, {4, 32, 4, 300},
+                                     {8, 32, 4, 300}, {4, 16, 4, 300}, {8, 16, 4, 300}};
+
 template <int M>
 cudaError_t launch_tile_m(const ReduceArgs& a, const TileGeo& geo, size_t smem, const TileMaps* maps,
                           cudaStream_t s) {
-  if (geo.s == 4)
-    return geo.t == 32 ? launch_tile_mst<M, 4, 32>(a, geo, smem, maps, s) : launch_tile_mst<M, 4, 16>(a, geo, smem, maps, s);
-  return geo.t == 32 ? launch_tile_mst<M, 8, 32>(a, geo, smem, maps, s) : launch_tile_mst<M, 8, 16>(a, geo, smem, maps, s);
+  const int code = geo.s * 1000 + geo.t * 10 + geo.c;
+  switch (code) {
+    case 4328: return launch_tile_mst<M, 4, 32, 8>(a, geo, smem, maps, s);
+    case 4168: return launch_tile_mst<M, 4, 16, 8>(a, geo, smem, maps, s);
+    case 8168: return launch_tile_mst<M, 8, 16, 8>(a, geo, smem, maps, s);
+    case 4324: return launch_tile_mst<M, 4, 32, 4>(a, geo, smem, maps, s);
+    case 8324: return launch_tile_mst<M, 8, 32, 4>(a, geo, smem, maps, s);
+    case 4164: return launch_tile_mst<M, 4, 16, 4>(a, geo, smem, maps, s);
+    case 8164: return launch_tile_mst<M, 8, 16, 4>(a, geo, smem, maps, s);
+    default: return cudaErrorInvalidValue;
+  }
 }
 
 // The weighted pass re-reads a CTA's slice of a tile from L2, so the slice
-// must stay in it: with 4-CTA clusters and 32 tokens at m = 4, d = 7168 (459 KB
-// slices) the launch read 800 MB from DRAM for 470 MB of H.  The geometry is
-// the first of (4 CTAs, 32 tokens), (8, 32), (4, 16), (8, 16) whose slice is
-// at most 300 KB, whose boxes per tile are a whole number of phases and
-// whose shared memory fits: 4-CTA clusters fit more SMs (5.0 vs 3.9 TB/s at
-// d = 2048), 16-token tiles pay twice the per-box and exchange overhead (3.2
-// vs 4.1 TB/s at d = 7168).
+// must stay in it (with 4-CTA clusters and 32 tokens at m = 4, d = 7168, 459
+// KB slices, the launch read 800 MB from DRAM for 470 MB of H).  The
+// geometry is the first of kTileShapes whose slice fits its limit, whose
+// boxes per tile are a whole number of phases and whose shared memory fits.
+// It depends on m and d only, never on the token count.  Measured on GB300
+// (m = 4, TB/s): 4-CTA clusters keep 144 SMs busy where 8-CTA clusters of
+// this CTA keep 120; boxes of 8 chunks (1 KB contiguous per token) beat 4:
+//   d = 7168, 131072 tokens: (8, 32, 4) 4.10, (4, 16, 8) 4.87
+//   d = 4096, 139264 tokens: (4, 32, 4) 3.92, (4, 16, 8) 5.18
+//   d = 2048,   2048 tokens: (4, 32, 4) 2.46, (4, 32, 8) 2.71 (65536: 5.09, 4.64)
 bool tile_geometry(const ReduceArgs& a, int dtype, TileGeo* geo, size_t* smem) {
   if (dtype != HDF_BF16 || a.alpha_override || a.path_norm_w) return false;
   if (a.n_tokens <= 0 || a.n_tokens > (1ll << 31) - 64) return false;  // TMA coordinates are 32-bit
   if (!(a.m == 1 || a.m == 2 || a.m == 4)) return false;
-  const int order[4][2] = {{4, 32}, {8, 32}, {4, 16}, {8, 16}};
-  for (const auto& st : order) {
-    const int S = st[0];
+  for (const TileShape& sh : kTileShapes) {
+    const int S = sh.s;
     if (a.d % (S * 64)) continue;
     geo->s = S;
     geo->ec = a.d / S;
-    geo->t = st[1];
-    if ((size_t)geo->t * a.m * geo->ec * 2 > 300 * 1024) continue;
+    geo->t = sh.t;
+    geo->c = sh.c;
+    if ((size_t)geo->t * a.m * geo->ec * 2 > (size_t)sh.max_slice_kb * 1024) continue;
     geo->nkb = geo->ec / 64;
-    geo->ngrp = (geo->nkb + TP_C - 1) / TP_C;
-    geo->tail = geo->nkb - (geo->ngrp - 1) * TP_C;
+    geo->ngrp = (geo->nkb + geo->c - 1) / geo->c;
+    geo->tail = geo->nkb - (geo->ngrp - 1) * geo->c;
     if ((a.m * geo->ngrp) % TP_NPH) continue;  // boxes per tile: a multiple of the 4 phases
     geo->wrow = a.m * geo->ec + 8;  // + 16 bytes: the gate rows of one B fragment sit in distinct banks
     geo->ntiles = (a.n_tokens + geo->t - 1) / geo->t;
@@ -1306,7 +1328,7 @@ bool reduce_tile_boxes(const ReduceArgs& a, int dtype, unsigned box[3], unsigned
   if (!tile_geometry(a, dtype, &geo, &smem)) return false;
   box[0] = tail_box[0] = 64;
   box[1] = tail_box[1] = (unsigned)geo.t;
-  box[2] = (unsigned)std::min(TP_C, geo.nkb);
+  box[2] = (unsigned)std::min(geo.c, geo.nkb);
   tail_box[2] = (unsigned)geo.tail;
   return true;
 }
