@@ -625,27 +625,25 @@ def measure_warm(cfg, inp, drafter, y, tok_cold, tgt, stream, steps, dev, pk):
 # launch: the traffic of that kernel grows in proportion to its rows).
 NCU_DRAM_BYTES = {
     "decode": {
-        "L0.ctx_kv_gemm": 26288128 + 1536,
         "L0.qkv_gemm": 25329664,
         "L0.o_gemm": 8667136,
         "L0.gate_up_gemm": 67264768 + 301568,
         "L0.down_gemm": 34029312,
         "lm_head": 134369536 + 3009280,
         "L0.attention": 17011456,
-        "gated_reduce": 33675264,
     },
 }
 NCU_DRAM_BYTES_PER_CTX_ROW = {
     # gemm_pair_kernel, one layer's context projection, captured on 16,384
     # rows at the large widths (profiles/ctx_kv_gemm_pair_large.md)
-    "large": {f"L{l}.ctx_kv_gemm": (16384, 2497119000 + 456967936) for l in range(2)},
+    "large": {f"L{l}.ctx_kv_gemm": (16384, 2509130000 + 456764672) for l in range(2)},
 }
 
 
 # DRAM bytes (read + write) per token of the tile reducer at m = 4, d = 7168,
-# from the ncu capture summarised in profiles/gated_reduce_sweep.md (8192
+# from the ncu capture summarised in profiles/gated_reduce_sweep.md (16,384
 # tokens; traffic grows with the tokens)
-NCU_DRAM_BYTES_PER_TOKEN_SWEEP = (470209024 + 87422976) / 8192
+NCU_DRAM_BYTES_PER_TOKEN_SWEEP = (946359808 + 203782144) / 16384
 
 
 def tensor_peak(pk, step_ms):
@@ -802,8 +800,9 @@ def run_sweep(args):
                        "l2": "inputs larger than L2 for N >= 4096"},
             "roofline": {"kernel": "gated_reduce", "bound": "hbm", "achieved": big["gbs"], "peak": pk["hbm_gbs"],
                          "unit": "GB/s", "frac": big["frac_hbm"],
-                         "traffic": int(NCU_DRAM_BYTES_PER_TOKEN_SWEEP * big["n"]) if m == 4 and d == 7168 else None,
-                         "traffic_note": "ncu capture at 8192 tokens scaled to the launch by tokens"},
+                         "traffic": (int(NCU_DRAM_BYTES_PER_TOKEN_SWEEP * big["n"])
+                                     if NCU_DRAM_BYTES_PER_TOKEN_SWEEP and m == 4 and d == 7168 else None),
+                         "traffic_note": "ncu capture at 16384 tokens scaled to the launch by tokens"},
             "sweep": rows}
     print(json.dumps(line), flush=True)
     return 0
