@@ -834,37 +834,93 @@ __global__ void __launch_bounds__(128, 1) gemm_pair_kernel(const __grid_constant
     pair_abort = abort_flag | ld_dsmem_s32(map_rank(smem_u32((const void*)&abort_flag), rank ^ 1u));
   __syncthreads();
   const uint32_t taddr = tmem + ((uint32_t)(warp * 32) << 16);
-  if (!pair_abort && num_kb > 0 && rope_regs) {
+  const bool seg_rope = (E.rope_mask >> seg_t) & 1;
+  const bool tma_out = E.kind == kEpiStore && E.out_tma && (E.pos_mode == 0 || E.pos_mode == 1) &&
+                       (E.seg_width % BN) == 0 && seg_t < 2 && (rope_regs || !seg_rope);
+  if (!pair_abort && num_kb > 0 && tma_out) {
+    // The tile goes through the drained stage memory as four 128-row x 64-
+    // column boxes in the output map's 128-byte swizzle (16-byte chunk j of
+    // row r at chunk j ^ (r & 7): a warp's 32 rows hit all banks), then out
+    // by four TMA stores: whole lines instead of one 32-byte piece per row
+    // and column chunk.  Chunks c and c + 8 (the same RoPE pairs of the
+    // tile's two heads) come from tensor memory together.
+    const int fl0 = tile_n * BN - seg_t * E.seg_width;
+    uint8_t* tile_smem = smem;  // 4 x 16 KB, 1024-byte aligned
+#pragma unroll
+    for (int c = 0; c < 8; ++c) {
+      float v[2][16];
+      tmem_ld16x2(taddr + 16 * c, v[0], taddr + 16 * (c + 8), v[1]);
+      if (rope_regs) {
+        const float4 c0v = rc[2 * c], c1v = rc[2 * c + 1];
+        const float4 s0v = rs[2 * c], s1v = rs[2 * c + 1];
+        const float cs[8] = {c0v.x, c0v.y, c0v.z, c0v.w, c1v.x, c1v.y, c1v.z, c1v.w};
+        const float sn[8] = {s0v.x, s0v.y, s0v.z, s0v.w, s1v.x, s1v.y, s1v.z, s1v.w};
+#pragma unroll
+        for (int hd = 0; hd < 2; ++hd)
+#pragma unroll
+          for (int i = 0; i < 8; ++i) {
+            const float x0 = v[hd][2 * i], x1 = v[hd][2 * i + 1];
+            v[hd][2 * i] = x0 * cs[i] - x1 * sn[i];
+            v[hd][2 * i + 1] = x0 * sn[i] + x1 * cs[i];
+          }
+      }
+#pragma unroll
+      for (int hd = 0; hd < 2; ++hd) {
+        const int cc = c + 8 * hd;  // 16-column chunk of the tile
+        uint8_t* box = tile_smem + (cc >> 2) * (BM * ROW_BYTES);
+        const int j0 = (cc & 3) * 2;
+        uint8_t* rowp = box + tid * ROW_BYTES;
+        *reinterpret_cast<uint4*>(rowp + ((j0 ^ (tid & 7)) << 4)) = V16<__nv_bfloat16>::pack(v[hd]);
+        *reinterpret_cast<uint4*>(rowp + (((j0 + 1) ^ (tid & 7)) << 4)) = V16<__nv_bfloat16>::pack(v[hd] + 8);
+      }
+    }
+    fence_proxy_async();
+    __syncthreads();
+    if (tid == 0) {
+#pragma unroll
+      for (int b = 0; b < BN / 64; ++b)
+        tma_store_2d(&E.out_map[seg_t], smem_u32(tile_smem + b * (BM * ROW_BYTES)), fl0 + 64 * b, my_m * BM);
+      tma_store_commit();
+      tma_store_wait_all();
+    }
+  } else if (!pair_abort && num_kb > 0 && rope_regs) {
     // the tile is one segment and two whole heads: chunk c holds pairs
     // 8 (c % 8) .. 8 (c % 8) + 7 of its head
     const int col_t = tile_n * BN;
     const int fl0 = col_t - seg_t * E.seg_width;
     __nv_bfloat16* out = reinterpret_cast<__nv_bfloat16*>(E.out[seg_t]);
+    // chunks c and c + 8 (the same pairs of the tile's two heads) are read
+    // from tensor memory together: one wait for both
 #pragma unroll
-    for (int c = 0; c < BN / 16; ++c) {
-      float v[16];
-      tmem_ld16(taddr + 16 * c, v);
-      if (srow >= 0 && col_t + 16 * c < g.N) {
-        const float4 c0v = rc[2 * (c % 8)], c1v = rc[2 * (c % 8) + 1];
-        const float4 s0v = rs[2 * (c % 8)], s1v = rs[2 * (c % 8) + 1];
-        const float cs[8] = {c0v.x, c0v.y, c0v.z, c0v.w, c1v.x, c1v.y, c1v.z, c1v.w};
-        const float sn[8] = {s0v.x, s0v.y, s0v.z, s0v.w, s1v.x, s1v.y, s1v.z, s1v.w};
+    for (int c = 0; c < 8; ++c) {
+      float v[2][16];
+      tmem_ld16x2(taddr + 16 * c, v[0], taddr + 16 * (c + 8), v[1]);
+      const float4 c0v = rc[2 * c], c1v = rc[2 * c + 1];
+      const float4 s0v = rs[2 * c], s1v = rs[2 * c + 1];
+      const float cs[8] = {c0v.x, c0v.y, c0v.z, c0v.w, c1v.x, c1v.y, c1v.z, c1v.w};
+      const float sn[8] = {s0v.x, s0v.y, s0v.z, s0v.w, s1v.x, s1v.y, s1v.z, s1v.w};
 #pragma unroll
-        for (int i = 0; i < 8; ++i) {
-          const float x0 = v[2 * i], x1 = v[2 * i + 1];
-          v[2 * i] = x0 * cs[i] - x1 * sn[i];
-          v[2 * i + 1] = x0 * sn[i] + x1 * cs[i];
+      for (int hd = 0; hd < 2; ++hd) {
+        const int cc = c + 8 * hd;
+        if (srow >= 0 && col_t + 16 * cc < g.N) {
+#pragma unroll
+          for (int i = 0; i < 8; ++i) {
+            const float x0 = v[hd][2 * i], x1 = v[hd][2 * i + 1];
+            v[hd][2 * i] = x0 * cs[i] - x1 * sn[i];
+            v[hd][2 * i + 1] = x0 * sn[i] + x1 * cs[i];
+          }
+          store16<__nv_bfloat16>(out + srow * E.ld + fl0 + 16 * cc, v[hd]);
         }
-        store16<__nv_bfloat16>(out + srow * E.ld + fl0 + 16 * c, v);
       }
     }
   } else if (!pair_abort && num_kb > 0) {
     const float* rope_row = stage_rope_row<BN>(g, my_m, tile_n, smem, spos);
 #pragma unroll 1
-    for (int c0 = 0; c0 < BN; c0 += 16) {
-      float v[16];
-      tmem_ld16(taddr + c0, v);
-      epilogue_chunk<__nv_bfloat16, BN>(g, my_m, tile_n, c0, v, smem, rope_row, srow, spos);
+    for (int c0 = 0; c0 < BN; c0 += 32) {
+      float v[2][16];
+      tmem_ld16x2(taddr + c0, v[0], taddr + c0 + 16, v[1]);
+      epilogue_chunk<__nv_bfloat16, BN>(g, my_m, tile_n, c0, v[0], smem, rope_row, srow, spos);
+      epilogue_chunk<__nv_bfloat16, BN>(g, my_m, tile_n, c0 + 16, v[1], smem, rope_row, srow, spos);
     }
   }
   tc_fence_before();

@@ -497,6 +497,10 @@ int hdf_fc_reduce(const void* H, int dtype, int64_t n_tokens, int m, int d_in, i
   g.epi.out[0] = y;
   g.epi.seg_width = d_out;
   g.epi.ld = d_out;
+  if (g.pair) {
+    if ((rc = make_map(&g.epi.out_map[0], y, dtype, n_tokens, d_out, d_out, 128))) return rc;
+    g.epi.out_tma = 1;
+  }
   CK(launch_gemm(g, (cudaStream_t)stream), "fc gemm launch");
   return HDF_OK;
 }
@@ -621,6 +625,11 @@ int launch_ctx_kv(const hdf_drafter_weights* w, const hdf_layer_weights& Lw, con
   g.epi.pos_mode = pos_mode;
   g.epi.ctx_len = len;
   g.epi.cache_cap = cap;
+  if (g.pair && pos_mode == 1) {  // packed rows: the tile leaves by TMA stores
+    if ((rc = make_map(&g.epi.out_map[0], kout, dt, rows, d, d, 128))) return rc;
+    if ((rc = make_map(&g.epi.out_map[1], vout, dt, rows, d, d, 128))) return rc;
+    g.epi.out_tma = 1;
+  }
   CK(launch_gemm(g, s), "ctx kv gemm");
   return HDF_OK;
 }
@@ -641,7 +650,13 @@ SideStream* side_stream(size_t n_events) {
   cudaStreamCaptureMode mode = cudaStreamCaptureModeRelaxed;
   cudaThreadExchangeStreamCaptureMode(&mode);
   bool ok = true;
-  if (!ss.s) ok = cudaStreamCreateWithFlags(&ss.s, cudaStreamNonBlocking) == cudaSuccess;
+  if (!ss.s) {
+    // the context path (norm, then each layer's K/V projection) is the
+    // step's critical path: its CTAs go first when both streams have work
+    int least = 0, greatest = 0;
+    if (cudaDeviceGetStreamPriorityRange(&least, &greatest) != cudaSuccess) greatest = 0;
+    ok = cudaStreamCreateWithPriority(&ss.s, cudaStreamNonBlocking, greatest) == cudaSuccess;
+  }
   while (ok && ss.ev.size() < n_events) {
     cudaEvent_t e;
     ok = cudaEventCreateWithFlags(&e, cudaEventDisableTiming) == cudaSuccess;
@@ -702,32 +717,37 @@ int draft_forward(const hdf_drafter_weights* w, const hdf_draft_shape* sh, const
     return HDF_OK;
   };
 
-  // The context path (RMSNorm, then each layer's K/V projection: compute-
-  // bound) runs on a second stream beside the block path (weight-streaming
-  // GEMMs): layer l's projection joins before layer l's attention and starts
-  // once layer l-1's attention has read the shared K/V buffers.  Serial when
-  // stage times are traced.
-  cudaStream_t sc = s;
+  // Each layer's context K/V projection (compute-bound) and its block path
+  // (input norm and Q/K_b/V_b projection: weight streaming) run on two
+  // streams and join before the layer's attention.  Layer 0's projection
+  // is the step's critical path (behind the reduce and the context norm): it
+  // stays on the caller's stream and the block path is forked onto a second
+  // stream only after the context norm, so that the projection's CTAs take
+  // the SMs first and the few CTAs of the block path fill the rest.  Later
+  // layers' projections go on the second stream, forked once the previous
+  // layer's attention has read the shared K/V buffers, beside that layer's
+  // MLP and the next block path.  Serial when stage times are traced.
   SideStream* side = nullptr;
   if (!trace && n_ctx > 0) side = side_stream(2 * (size_t)sh->n_layers + 1);
-  if (side) {
-    sc = side->s;
-    CK(cudaEventRecord(side->ev[0], s), "fork record");
-    CK(cudaStreamWaitEvent(sc, side->ev[0], 0), "fork wait");
-  }
+  const cudaStream_t s2 = side ? side->s : s;
   // ---- context RMSNorm
   if ((rc = mark())) return rc;
-  if (n_ctx > 0) CK(launch_rmsnorm(ctx, 0, w->ctx_norm, c, dt, n_ctx, (int)d, sh->norm_eps, sc), "ctx norm");
+  if (n_ctx > 0) CK(launch_rmsnorm(ctx, 0, w->ctx_norm, c, dt, n_ctx, (int)d, sh->norm_eps, s), "ctx norm");
 
   for (int l = 0; l < sh->n_layers; ++l) {
     const hdf_layer_weights& Lw = w->layers[l];
+    // streams of this layer's projection and block path
+    const cudaStream_t s_ctx = l == 0 ? s : s2;
+    const cudaStream_t s_blk = l == 0 ? s2 : s;
     // ---- conditioning projection: [K_c | V_c] = c [W_k; W_v]^T, RoPE on K_c
     if ((rc = mark())) return rc;
-    if (side && l > 0) CK(cudaStreamWaitEvent(sc, side->ev[2 * l], 0), "attention-done wait");
+    if (side && l == 0) CK(cudaEventRecord(side->ev[0], s), "fork record");  // behind the context norm
+    if (side && l > 0) CK(cudaStreamWaitEvent(s2, side->ev[2 * l], 0), "fork wait");  // behind attention l-1
     if (n_ctx > 0 &&
-        (rc = launch_ctx_kv(w, Lw, sh, c, n_ctx, kc, vc, cu_ctx, 1, nullptr, 0, sc)))
+        (rc = launch_ctx_kv(w, Lw, sh, c, n_ctx, kc, vc, cu_ctx, 1, nullptr, 0, s_ctx)))
       return rc;
-    if (side) CK(cudaEventRecord(side->ev[2 * l + 1], sc), "join record");
+    if (side && l == 0) CK(cudaStreamWaitEvent(s2, side->ev[0], 0), "fork wait");
+    if (side && l > 0) CK(cudaEventRecord(side->ev[2 * l + 1], s2), "join record");
     // context K / V of this layer: the workspace, or the cache
     const void* kctx = kc;
     const void* vctx = vc;
@@ -741,10 +761,10 @@ int draft_forward(const hdf_drafter_weights* w, const hdf_draft_shape* sh, const
     if ((rc = mark())) return rc;
     if (l == 0)
       CK(launch_embed_norm(w->embed, w->mask_vec, anchor, Lw.attn_norm, h, x, dt, sh->batch, sh->block, (int)d,
-                           sh->vocab, sh->norm_eps, s),
+                           sh->vocab, sh->norm_eps, s_blk),
          "embed norm");
     else
-      CK(launch_rmsnorm(h, 1, Lw.attn_norm, x, dt, M, (int)d, sh->norm_eps, s), "attn norm");
+      CK(launch_rmsnorm(h, 1, Lw.attn_norm, x, dt, M, (int)d, sh->norm_eps, s_blk), "attn norm");
     // ---- Q / K_b / V_b with RoPE at block positions
     if ((rc = mark())) return rc;
     {
@@ -772,7 +792,8 @@ int draft_forward(const hdf_drafter_weights* w, const hdf_draft_shape* sh, const
       g.epi.batch = sh->batch;
       g.epi.block = sh->block;
       g.epi.pos_mode = cached ? 4 : 2;
-      CK(launch_gemm(g, s), "qkv gemm");
+      CK(launch_gemm(g, s_blk), "qkv gemm");
+      if (side && l == 0) CK(cudaEventRecord(side->ev[1], s2), "join record");
     }
     // ---- attention over [K_c; K_b]
     if ((rc = mark())) return rc;

@@ -11,15 +11,26 @@ namespace hdf {
 // (its prologue may overlap the previous kernel in the stream; the kernel
 // calls pdl_wait() before touching that kernel's results) and, when
 // cluster_x > 1, as clusters of cluster_x consecutive blocks.
+// The launch carries the stream's priority as a launch attribute, so that
+// kernels captured into a CUDA graph keep the priority of the stream they
+// were issued on.
 template <typename... KArgs, typename... Args>
 cudaError_t launch_kernel(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t s,
                           unsigned cluster_x, Args&&... args) {
   cudaLaunchConfig_t cfg = {};
-  cudaLaunchAttribute attr[2];
+  cudaLaunchAttribute attr[3];
   unsigned n = 0;
   attr[n].id = cudaLaunchAttributeProgrammaticStreamSerialization;
   attr[n].val.programmaticStreamSerializationAllowed = 1;
   ++n;
+  int prio = 0;
+  if (cudaStreamGetPriority(s, &prio) == cudaSuccess && prio != 0) {
+    attr[n].id = cudaLaunchAttributePriority;
+    attr[n].val.priority = prio;
+    ++n;
+  } else {
+    cudaGetLastError();
+  }
   if (cluster_x > 1) {
     attr[n].id = cudaLaunchAttributeClusterDimension;
     attr[n].val.clusterDim.x = cluster_x;
@@ -132,6 +143,11 @@ struct Epilogue {
   float* part_max;      // [tiles_m, N]
   int* part_arg;
   float* part_sum;
+  // kEpiStore on CTA pairs with packed output rows (pos_mode 0 or 1): the
+  // tile is written by TMA stores through these maps of out[0], out[1]
+  // ([rows, seg_width], boxes {64, 128}, 128-byte swizzle) when out_tma != 0
+  int out_tma;
+  CUtensorMap out_map[2];
 };
 
 struct GemmArgs {
