@@ -296,16 +296,28 @@ __device__ __forceinline__ void epilogue_chunk(const GemmArgs& g, int tile_m, in
               if (jb + k < V) dst[k] = v[k] * it;
           }
         }
+        // the chunk's maximum and first argmax in column order, then its
+        // sum of exponentials (independent of one another), then one merge
+        // with the running values (an earlier chunk keeps a tie)
+        float cm = -INFINITY;
+        int ca = INT_MAX;
 #pragma unroll
-        for (int k = 0; k < 16; ++k) {
-          if (jb + k >= V) break;
-          const float x = v[k];
-          if (x > m) {
-            sum = (m == -INFINITY ? 0.f : sum * expf((m - x) * it)) + 1.f;
-            m = x;
-            a = jb + k;
-          } else if (x != -INFINITY) {
-            sum += expf((x - m) * it);
+        for (int k = 0; k < 16; ++k)
+          if (jb + k < V && v[k] > cm) {
+            cm = v[k];
+            ca = jb + k;
+          }
+        if (cm != -INFINITY) {
+          float cs = 0.f;
+#pragma unroll
+          for (int k = 0; k < 16; ++k)
+            if (jb + k < V) cs += expf((v[k] - cm) * it);
+          if (cm > m) {
+            sum = (m == -INFINITY ? 0.f : sum * expf((m - cm) * it)) + cs;
+            m = cm;
+            a = ca;
+          } else {
+            sum += cs * expf((cm - m) * it);
           }
         }
       }
@@ -342,19 +354,22 @@ __device__ __forceinline__ void epilogue_chunk(const GemmArgs& g, int tile_m, in
       __syncthreads();
       const int k = row >> 3, part = row & 7;
       const float it = E.inv_temp;
+      // this thread's 16 rows (increasing): maximum and first argmax, then
+      // the sum of exponentials, independent of one another
+      float xs[16];
       float m = -INFINITY, sum = 0.f;
       int a = INT_MAX;
-#pragma unroll 4
+#pragma unroll
       for (int i = 0; i < 16; ++i) {
-        const int r = i * 8 + part;  // this thread's rows, increasing
-        const float x = tv[k * 136 + r];
-        if (x > m) {
-          sum = (m == -INFINITY ? 0.f : sum * expf((m - x) * it)) + 1.f;
-          m = x;
-          a = tile_m * BM + r;
-        } else if (x != -INFINITY) {
-          sum += expf((x - m) * it);
+        xs[i] = tv[k * 136 + i * 8 + part];
+        if (xs[i] > m) {
+          m = xs[i];
+          a = tile_m * BM + i * 8 + part;
         }
+      }
+      if (m != -INFINITY) {
+#pragma unroll
+        for (int i = 0; i < 16; ++i) sum += expf((xs[i] - m) * it);
       }
 #pragma unroll
       for (int o = 1; o < 8; o <<= 1) {
@@ -557,11 +572,19 @@ __global__ void __launch_bounds__(128, 1) gemm_kernel(const __grid_constant__ Ge
     const float* rope_row = BM * (2 * 64 + 4) * 4 <= STAGES * STAGE_BYTES
                                 ? stage_rope_row<BN>(g, tile_m, tile_n, smem, spos)
                                 : nullptr;
+    if (BN >= 32) {
+      // two chunks read from tensor memory per wait
 #pragma unroll 1
-    for (int c0 = 0; c0 < BN; c0 += 16) {
+      for (int c0 = 0; c0 < BN; c0 += 32) {
+        float v[2][16];
+        tmem_ld16x2(taddr + c0, v[0], taddr + c0 + 16, v[1]);
+        epilogue_chunk<T, BN>(g, tile_m, tile_n, c0, v[0], smem, rope_row, srow, spos);
+        epilogue_chunk<T, BN>(g, tile_m, tile_n, c0 + 16, v[1], smem, rope_row, srow, spos);
+      }
+    } else {
       float v[16];
-      tmem_ld16(taddr + c0, v);
-      epilogue_chunk<T, BN>(g, tile_m, tile_n, c0, v, smem, rope_row, srow, spos);
+      tmem_ld16(taddr, v);
+      epilogue_chunk<T, BN>(g, tile_m, tile_n, 0, v, smem, rope_row, srow, spos);
     }
   }
   if (g.k_splits > 1) {

@@ -213,8 +213,13 @@ __device__ __forceinline__ MaxArgSum combine(MaxArgSum x, MaxArgSum y, float it)
   return r;
 }
 
-// One CTA per token row: merge the per-vocab-tile partials, then subtract
-// the log-sum-exp from the scaled logits already stored in logsoftmax.
+// CTA (j, c): merge token row j's per-vocabulary-tile partials (every CTA of
+// the row in the same order, so all get the same bits), then subtract the
+// log-sum-exp from vocabulary chunk c of the scaled logits already stored in
+// logsoftmax (16-byte accesses when rows are 16-byte multiples).  Chunk 0
+// writes the row's token and maximal logit.
+constexpr long long kLsChunk = 8192;  // vocabulary entries normalised per CTA
+
 __global__ void lm_reduce_kernel(const float* __restrict__ pmax, const int* __restrict__ parg,
                                  const float* __restrict__ psum, int tiles, long long M, long long V,
                                  float it, int* tok, float* zmax, float* ls) {
@@ -223,6 +228,7 @@ __global__ void lm_reduce_kernel(const float* __restrict__ pmax, const int* __re
   pdl_launch_dependents();
   pdl_wait();
   const long long j = blockIdx.x;
+  const long long chunk = blockIdx.y;
   MaxArgSum acc{-INFINITY, INT_MAX, 0.f};
   for (int t = threadIdx.x; t < tiles; t += blockDim.x) {
     const size_t o = (size_t)t * M + j;
@@ -239,15 +245,30 @@ __global__ void lm_reduce_kernel(const float* __restrict__ pmax, const int* __re
   if (threadIdx.x == 0) {
     MaxArgSum r = sh[0];
     for (int w = 1; w < (int)(blockDim.x >> 5); ++w) r = combine(r, sh[w], it);
-    tok[j] = r.a;
-    if (zmax) zmax[j] = r.m;
+    if (chunk == 0) {
+      tok[j] = r.a;
+      if (zmax) zmax[j] = r.m;
+    }
     lse_sh = r.m * it + logf(r.s);
   }
   __syncthreads();
   if (ls) {
     const float lse = lse_sh;
     float* row = ls + j * V;
-    for (long long v = threadIdx.x; v < V; v += blockDim.x) row[v] -= lse;
+    const long long v0 = chunk * kLsChunk, v1 = min(V, v0 + kLsChunk);
+    if ((V & 3) == 0) {
+      float4* r4 = reinterpret_cast<float4*>(row);
+      for (long long q = v0 / 4 + threadIdx.x; q < v1 / 4; q += blockDim.x) {
+        float4 x = r4[q];
+        x.x -= lse;
+        x.y -= lse;
+        x.z -= lse;
+        x.w -= lse;
+        r4[q] = x;
+      }
+    } else {
+      for (long long v = v0 + threadIdx.x; v < v1; v += blockDim.x) row[v] -= lse;
+    }
   }
 }
 
@@ -301,8 +322,9 @@ cudaError_t launch_cache_advance(int* len, const int* cu, int batch, long long c
 cudaError_t launch_lm_reduce(const float* pmax, const int* parg, const float* psum, int tiles, long long M,
                              long long V, float it, int* tok, float* zmax, float* ls, cudaStream_t s) {
   if (M == 0) return cudaSuccess;
-  return launch_kernel(lm_reduce_kernel, dim3((unsigned)M), dim3(256), 0, s, 1u, pmax, parg, psum, tiles, M, V, it,
-                       tok, zmax, ls);
+  const unsigned chunks = ls ? (unsigned)((V + kLsChunk - 1) / kLsChunk) : 1u;
+  return launch_kernel(lm_reduce_kernel, dim3((unsigned)M, chunks), dim3(256), 0, s, 1u, pmax, parg, psum, tiles, M,
+                       V, it, tok, zmax, ls);
 }
 
 }  // namespace hdf
