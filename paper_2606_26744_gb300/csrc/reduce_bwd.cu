@@ -14,7 +14,9 @@
 //   2. weight gradient: CTA (slice, split) owns 256 x VEC columns of W_f and a
 //      contiguous token range; each thread keeps m x VEC fp32 sums over its
 //      tokens in token order (and the CTAs of slice 0 the db sums) and writes
-//      them to the split's partial.
+//      them to the split's partial.  The CTA streams its 4 KB slice of 16
+//      tokens at a time (and their u rows) through a 3-deep cp.async ring in
+//      shared memory, one CTA per SM: 128 KB of H in flight per SM.
 //   3. finalize: the partials are added in split order.
 // HBM-bound: H is read twice (passes 1 and 2), dy once.
 #include <algorithm>
@@ -114,11 +116,33 @@ __global__ void __launch_bounds__(RB_THREADS) reduce_bwd_gate_kernel(const Reduc
   }
 }
 
+constexpr int WG_TOK = 16;    // tokens per ring stage
+constexpr int WG_STAGES = 3;  // ring depth
+constexpr int wg_stage_bytes(int m) { return WG_TOK * RB_THREADS * 16 + WG_TOK * 8 * 4; }  // H slice + u rows
+constexpr size_t wg_smem(int m) { return (size_t)WG_STAGES * wg_stage_bytes(m); }
+
+__device__ __forceinline__ void cp_async16(void* dst, const void* src, bool pred) {
+  asm volatile(
+      "{\n .reg .pred p;\n setp.ne.u32 p, %2, 0;\n @p cp.async.cg.shared.global [%0], [%1], 16;\n}\n" ::"r"(
+          smem_u32(dst)),
+      "l"(src), "r"((uint32_t)pred)
+      : "memory");
+}
+__device__ __forceinline__ void cp_async4(void* dst, const void* src, bool pred) {
+  asm volatile(
+      "{\n .reg .pred p;\n setp.ne.u32 p, %2, 0;\n @p cp.async.ca.shared.global [%0], [%1], 4;\n}\n" ::"r"(
+          smem_u32(dst)),
+      "l"(src), "r"((uint32_t)pred)
+      : "memory");
+}
+
 template <typename T, int M>
-__global__ void __launch_bounds__(RB_THREADS) reduce_bwd_wgrad_kernel(const ReduceBwdArgs a, long long tok_per) {
+__global__ void __launch_bounds__(RB_THREADS, 1) reduce_bwd_wgrad_kernel(const ReduceBwdArgs a, long long tok_per) {
+  extern __shared__ __align__(16) uint8_t wg_smem_raw[];
   pdl_launch_dependents();
   pdl_wait();
   constexpr int VEC = V16<T>::N;
+  constexpr int SB = wg_stage_bytes(M);
   const long long md = (long long)M * a.d;
   const T* H = reinterpret_cast<const T*>(a.H);
   const int tid = threadIdx.x;
@@ -128,47 +152,64 @@ __global__ void __launch_bounds__(RB_THREADS) reduce_bwd_wgrad_kernel(const Redu
   const long long c = ((long long)blockIdx.x * RB_THREADS + tid) * VEC;  // first column of this thread
   const bool active = c < md;
   const bool db_thread = blockIdx.x == 0 && tid < M;
+  const long long ntok = t1 > t0 ? t1 - t0 : 0;
+  const long long nstage = (ntok + WG_TOK - 1) / WG_TOK;
+  // stage g: tokens t0 + g*WG_TOK .. ; this thread copies its 16 bytes of
+  // every token, threads 0 .. WG_TOK*M-1 one u entry each
+  auto issue = [&](long long g) {
+    uint8_t* st = wg_smem_raw + (g % WG_STAGES) * SB;
+    const long long tb = t0 + g * WG_TOK;
+#pragma unroll
+    for (int i = 0; i < WG_TOK; ++i) {
+      const long long t = tb + i;
+      cp_async16(st + (i * RB_THREADS + tid) * 16, H + (t < t1 ? t : t0) * md + (active ? c : 0), active && t < t1);
+    }
+    if (tid < WG_TOK * M) {
+      const int i = tid / M, j = tid - i * M;
+      const long long t = tb + i;
+      cp_async4(st + WG_TOK * RB_THREADS * 16 + (i * 8 + j) * 4, a.u + (t < t1 ? t : t0) * M + j, t < t1);
+    }
+    asm volatile("cp.async.commit_group;" ::: "memory");
+  };
   float acc[M][VEC];
 #pragma unroll
   for (int j = 0; j < M; ++j)
 #pragma unroll
     for (int e = 0; e < VEC; ++e) acc[j][e] = 0.f;
   float dbs = 0.f;
-  long long t = t0;
-  // four tokens per round: their loads are in flight together
-  for (; t + 4 <= t1; t += 4) {
-    float u[4][M], x[4][VEC], dgv[4];
-#pragma unroll
-    for (int i = 0; i < 4; ++i) {
-#pragma unroll
-      for (int j = 0; j < M; ++j) u[i][j] = __ldg(a.u + (t + i) * M + j);
-      if (active) V16<T>::unpack(ld_stream16(H + (t + i) * md + c), x[i]);
-      dgv[i] = db_thread ? __ldg(a.dg + (t + i) * M + tid) : 0.f;
-    }
-#pragma unroll
-    for (int i = 0; i < 4; ++i) {
-      if (active) {
-#pragma unroll
-        for (int j = 0; j < M; ++j)
-#pragma unroll
-          for (int e = 0; e < VEC; ++e) acc[j][e] += u[i][j] * x[i][e];
-      }
-      dbs += dgv[i];
-    }
+  for (long long g = 0; g < WG_STAGES - 1; ++g) {
+    if (g < nstage) issue(g);
+    else asm volatile("cp.async.commit_group;" ::: "memory");
   }
-  for (; t < t1; ++t) {
-    float u[M], x[VEC];
-#pragma unroll
-    for (int j = 0; j < M; ++j) u[j] = __ldg(a.u + t * M + j);
+  for (long long g = 0; g < nstage; ++g) {
+    if (g + WG_STAGES - 1 < nstage) issue(g + WG_STAGES - 1);
+    else asm volatile("cp.async.commit_group;" ::: "memory");
+    asm volatile("cp.async.wait_group %0;" ::"n"(WG_STAGES - 1) : "memory");  // stage g has landed (this thread's copies)
+    __syncthreads();                                                           // ... and every thread's
+    const uint8_t* st = wg_smem_raw + (g % WG_STAGES) * SB;
+    const float* us = reinterpret_cast<const float*>(st + WG_TOK * RB_THREADS * 16);
+    const long long tb = t0 + g * WG_TOK;
+    const int nt = (int)min((long long)WG_TOK, t1 - tb);
     if (active) {
-      V16<T>::unpack(ld_stream16(H + t * md + c), x);
+#pragma unroll 4
+      for (int i = 0; i < WG_TOK; ++i) {
+        if (i < nt) {  // tokens in order
+          float x[VEC];
+          V16<T>::unpack(*reinterpret_cast<const uint4*>(st + (i * RB_THREADS + tid) * 16), x);
 #pragma unroll
-      for (int j = 0; j < M; ++j)
+          for (int j = 0; j < M; ++j) {
+            const float u = us[i * 8 + j];
 #pragma unroll
-        for (int e = 0; e < VEC; ++e) acc[j][e] += u[j] * x[e];
+            for (int e = 0; e < VEC; ++e) acc[j][e] += u * x[e];
+          }
+        }
+      }
     }
-    if (db_thread) dbs += __ldg(a.dg + t * M + tid);
+    if (db_thread)
+      for (int i = 0; i < nt; ++i) dbs += __ldg(a.dg + (tb + i) * M + tid);
+    __syncthreads();  // the stage is read before it is refilled
   }
+  asm volatile("cp.async.wait_all;" ::: "memory");
   if (active) {
 #pragma unroll
     for (int j = 0; j < M; ++j) {
@@ -205,8 +246,11 @@ cudaError_t launch_m(const ReduceBwdArgs& a, const ReduceBwdPlan& p, cudaStream_
   cudaError_t e = launch_kernel(reduce_bwd_gate_kernel<T, M>, dim3((unsigned)p.gate_ctas), dim3(RB_THREADS), 0, s,
                                 1u, a);
   if (e != cudaSuccess) return e;
+  static cudaError_t attr = cudaFuncSetAttribute(reduce_bwd_wgrad_kernel<T, M>,
+                                                 cudaFuncAttributeMaxDynamicSharedMemorySize, (int)wg_smem(M));
+  if (attr != cudaSuccess) return attr;
   e = launch_kernel(reduce_bwd_wgrad_kernel<T, M>, dim3((unsigned)p.slices, (unsigned)p.splits), dim3(RB_THREADS),
-                    0, s, 1u, a, p.tok_per);
+                    wg_smem(M), s, 1u, a, p.tok_per);
   if (e != cudaSuccess) return e;
   const long long n = (long long)M * M * a.d + M;
   const unsigned blocks = (unsigned)std::min<long long>((n + 255) / 256, 4096);
@@ -233,7 +277,7 @@ ReduceBwdPlan reduce_bwd_plan(long long n_tokens, int m, int d, int dtype, int n
   const int vec = dtype == HDF_BF16 ? 8 : 4;
   const long long md = (long long)m * d;
   p.slices = (int)((md + (long long)RB_THREADS * vec - 1) / ((long long)RB_THREADS * vec));
-  const long long want = std::max(1LL, (2LL * n_sm + p.slices - 1) / p.slices);
+  const long long want = std::max(1LL, (long long)n_sm / p.slices);  // one CTA per SM
   p.splits = (int)std::max(1LL, std::min({want, 1024LL, n_tokens}));
   p.tok_per = (n_tokens + p.splits - 1) / p.splits;
   p.splits = (int)std::max(1LL, (n_tokens + p.tok_per - 1) / p.tok_per);  // no empty split
