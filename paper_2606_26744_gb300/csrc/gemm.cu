@@ -47,7 +47,7 @@ template <> struct GT<float> {
 // Rings of ~96 KB, so that two CTAs share an SM: two independent producers
 // keep more loads in flight than one CTA with a ring twice as deep
 // (measured on the skinny weight-streaming GEMMs of the draft step).
-constexpr int stages_for(int bn) { return bn >= 256 ? 2 : (bn >= 128 ? 3 : (bn >= 64 ? 4 : 5)); }
+constexpr int stages_for(int bn) { return bn >= 224 ? 2 : (bn >= 128 ? 3 : (bn >= 64 ? 4 : 5)); }
 constexpr int kPartialOffset = 12288;  // split-K partial tile (rank 0's is reduced in place), in the drained
                                        // stage memory above the epilogue's scratch (at most 16 x 136 floats)
 constexpr bool partial_fits(int bn) { return kPartialOffset + BM * bn * 4 <= stages_for(bn) * (BM + bn) * ROW_BYTES; }
@@ -430,7 +430,7 @@ __global__ void __launch_bounds__(128, 1) gemm_kernel(const __grid_constant__ Ge
   constexpr int A_BYTES = BM * ROW_BYTES;
   constexpr int B_BYTES = BN * ROW_BYTES;
   constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
-  constexpr uint32_t TMEM_COLS = BN < 32 ? 32 : BN;
+  constexpr uint32_t TMEM_COLS = BN <= 32 ? 32 : (BN <= 64 ? 64 : (BN <= 128 ? 128 : 256));  // a power of two
   constexpr uint32_t IDESC = umma_idesc(BM, BN, GT<T>::FMT);
 
   extern __shared__ uint8_t smem_raw[];
@@ -1024,6 +1024,7 @@ int resident_ctas_t(int bn, int cluster) {
     case 32: return resident_ctas_bn<T, 32>(cluster);
     case 64: return resident_ctas_bn<T, 64>(cluster);
     case 128: return resident_ctas_bn<T, 128>(cluster);
+    case 224: return resident_ctas_bn<T, 224>(cluster);
     case 256: return resident_ctas_bn<T, 256>(cluster);
     default: return -1;
   }
@@ -1036,6 +1037,7 @@ cudaError_t launch_t(const GemmArgs& g, cudaStream_t s) {
     case 32: return launch_bn<T, 32>(g, s);
     case 64: return launch_bn<T, 64>(g, s);
     case 128: return launch_bn<T, 128>(g, s);
+    case 224: return launch_bn<T, 224>(g, s);
     case 256: return launch_bn<T, 256>(g, s);
     default: return cudaErrorInvalidValue;
   }
@@ -1047,9 +1049,9 @@ int gemm_stages(int, int bn) { return stages_for(bn); }
 
 int gemm_resident_ctas(int dtype, int bn, int cluster) {
   if (cluster < 1 || cluster > 16) return -1;
-  const int bi = bn == 16 ? 0 : bn == 32 ? 1 : bn == 64 ? 2 : bn == 128 ? 3 : bn == 256 ? 4 : -1;
+  const int bi = bn == 16 ? 0 : bn == 32 ? 1 : bn == 64 ? 2 : bn == 128 ? 3 : bn == 256 ? 4 : bn == 224 ? 5 : -1;
   if (bi < 0) return -1;
-  static std::atomic<int> cache[2][5][17];  // 0: not asked yet
+  static std::atomic<int> cache[2][6][17];  // 0: not asked yet
   std::atomic<int>& c = cache[dtype == HDF_BF16 ? 0 : 1][bi][cluster];
   int v = c.load(std::memory_order_relaxed);
   if (v == 0) {

@@ -1000,18 +1000,38 @@ struct LmLayout {
   int tiles_m;
   size_t pmax, parg, psum, total;
 };
-// Token-major LM head (tokens on the GEMM rows, vocabulary 256 columns per
-// tile) from this many tokens: each CTA then streams 1.5 bytes per weight
-// byte instead of 2 (the swapped tile re-reads a token tile as large as its
-// weight tile)
+// Token-major LM head (tokens on the GEMM rows, 224 or 256 vocabulary columns
+// per tile) from this many tokens: each CTA then streams about 1.5 bytes per
+// weight byte instead of 2 (the swapped tile re-reads a token tile as large
+// as its weight tile)
 constexpr int64_t kLmTokenMajorFrom = 64;
+
+// Vocabulary columns per token-major tile: of 256 and 224, the one with the
+// least waves x width over two resident CTAs per SM.  At V = 129,280 and
+// 128 tokens: 505 tiles of 256 take 1.66 waves (2 x 256), 578 tiles of 224
+// take 1.90 (2 x 224).
+int lm_token_major_bn(int64_t M, int64_t V) {
+  const long long slots = 2LL * num_sms(), tm = (M + 127) / 128;
+  int best = 256;
+  long long best_cost = LLONG_MAX;
+  for (int bn : {256, 224}) {
+    const long long tiles = tm * ((V + bn - 1) / bn);
+    const long long cost = (tiles + slots - 1) / slots * bn;
+    if (cost < best_cost) {
+      best_cost = cost;
+      best = bn;
+    }
+  }
+  return best;
+}
 
 LmLayout lm_layout(int64_t M, int64_t V, int dtype, int d) {
   LmLayout L;
   L.token_major = M >= kLmTokenMajorFrom;
-  L.p = L.token_major ? SplitPlan{256, 1, (int)(((M + 127) / 128) * ((V + 255) / 256))} : plan_swap(dtype, V, M, d);
+  const int tbn = L.token_major ? lm_token_major_bn(M, V) : 0;
+  L.p = L.token_major ? SplitPlan{tbn, 1, (int)(((M + 127) / 128) * ((V + tbn - 1) / tbn))} : plan_swap(dtype, V, M, d);
   L.tiles_m = (int)((V + 127) / 128);  // partial rows reserved: enough for either orientation
-  L.tiles = L.token_major ? (int)((V + 255) / 256) : L.tiles_m;
+  L.tiles = L.token_major ? (int)((V + tbn - 1) / tbn) : L.tiles_m;
   size_t off = 0;
   auto take = [&](size_t b) {
     const size_t o = off;
