@@ -636,7 +636,7 @@ NCU_DRAM_BYTES = {
 NCU_DRAM_BYTES_PER_CTX_ROW = {
     # gemm_pair_kernel, one layer's context projection, captured on 16,384
     # rows at the large widths (profiles/ctx_kv_gemm_pair_large.md)
-    "large": {f"L{l}.ctx_kv_gemm": (16384, 2509130000 + 456764672) for l in range(2)},
+    "large": {f"L{l}.ctx_kv_gemm": (16384, 2518131000 + 457346816) for l in range(2)},
 }
 
 
@@ -814,7 +814,9 @@ def run_kernel_only(args):
       accept      hdf_accept_len over args.tokens blocks of 15 drafts
       reduce_bwd  hdf_gated_reduce_backward over args.tokens tokens, m 4, d 7168
       reduce      hdf_gated_reduce (tile kernel) over args.tokens tokens, m 4, d 7168
-      loss        hdf_draft_loss over the large workload's blocks (8 x 16, P 2, V 129280)"""
+      loss        hdf_draft_loss over the large workload's blocks (8 x 16, P 2, V 129280)
+      lmhead      hdf_lm_head_argmax at the large workload's widths: 128 tokens,
+                  d 7168, V 129280, fp32 log-softmax"""
     from paper_2606_26744_gb300 import build, hdf
     build.build()
     dev = torch.device("cuda", 0)
@@ -851,6 +853,19 @@ def run_kernel_only(args):
             def launch():
                 hdf.hdf_gated_reduce_backward(H, Wf, b, dy, dWf=dwf, db=dbv, ws=ws)
             byt = 2 * n * m * d * 2 + n * d * 2 + m * m * d * 2 + m * m * d * 4
+    elif args.kernel_only == "lmhead":
+        M, d, V = 128, 7168, 129280
+        h = (torch.randn(M, d, device=dev, generator=g)).to(torch.bfloat16)
+        Wl = (torch.randn(V, d, device=dev, generator=g) * 0.02).to(torch.bfloat16)
+        tok = torch.empty(M, dtype=torch.int32, device=dev)
+        zmax = torch.empty(M, dtype=torch.float32, device=dev)
+        ls = torch.empty((M, V), dtype=torch.float32, device=dev)
+        lws = torch.empty(hdf.lm_head_workspace_size(M, d, V, torch.bfloat16), dtype=torch.uint8, device=dev)
+
+        def launch():
+            hdf.hdf_lm_head_argmax(h, Wl, logsoftmax=True, tok=tok, zmax=zmax, ls=ls, ws=lws)
+        byt = V * d * 2 + M * d * 2 + 2 * M * V * 4
+        n = M
     elif args.kernel_only == "loss":
         batch, block, P, V = 8, 16, 2, 129280
         ls_s = torch.log_softmax(torch.randn(batch * block, V, device=dev, generator=g) * 3, dim=-1)
@@ -1075,7 +1090,7 @@ def main():
     ap.add_argument("--batch", type=int, default=None, help="profiling override of the workload's batch")
     ap.add_argument("--vocab", type=int, default=None, help="profiling override of the workload's vocabulary")
     ap.add_argument("--layers", type=int, default=None, help="profiling override of the workload's layers")
-    ap.add_argument("--kernel-only", default=None, choices=["accept", "reduce_bwd", "reduce", "loss"],
+    ap.add_argument("--kernel-only", default=None, choices=["accept", "reduce_bwd", "reduce", "loss", "lmhead"],
                     help="time one kernel alone (profiling runs; not a bench line)")
     ap.add_argument("--tokens", type=int, default=1 << 20, help="units of a --kernel-only run")
     args = ap.parse_args()
