@@ -1006,7 +1006,10 @@ __global__ void __launch_bounds__(TP_THR, 1) gated_reduce_tile_kernel(const Redu
     const int row = (T == 32 ? sub * 16 : 0) + (lane & 15), hsel = lane >> 4;
     for (long long i = 0; i < nl; ++i) {
       float acc[2][4] = {{0.f, 0.f, 0.f, 0.f}, {0.f, 0.f, 0.f, 0.f}};  // two chains: plane parity
-      unsigned long long sq0[2] = {0ull, 0ull}, sq1[2] = {0ull, 0ull};
+      // sums of squares as the diagonals of A A^T on the tensor cores: the B
+      // fragment of A^T for tokens 0-7 is this thread's A registers 0 and 2,
+      // for tokens 8-15 its registers 1 and 3
+      float dl[4] = {0.f, 0.f, 0.f, 0.f}, dh[4] = {0.f, 0.f, 0.f, 0.f};
       bool ok = true;
       for (int j = hb; j < NB; j += TP_NPH) {
         const long long gs = i * NB + j;  // stage counter
@@ -1035,10 +1038,8 @@ __global__ void __launch_bounds__(TP_THR, 1) gated_reduce_tile_kernel(const Redu
 #pragma unroll
             for (int kk = 0; kk < 4; ++kk) {
               mma16816(acc[kk & 1], af[kk], bf[kk][0], bf[kk][1]);
-              sq_acc2(sq0[kk & 1], af[kk][0]);  // row g8
-              sq_acc2(sq0[kk & 1], af[kk][2]);
-              sq_acc2(sq1[kk & 1], af[kk][1]);  // row g8 + 8
-              sq_acc2(sq1[kk & 1], af[kk][3]);
+              mma16816(dl, af[kk], af[kk][0], af[kk][2]);
+              mma16816(dh, af[kk], af[kk][1], af[kk][3]);
             }
           }
         }
@@ -1050,11 +1051,12 @@ __global__ void __launch_bounds__(TP_THR, 1) gated_reduce_tile_kernel(const Redu
       // halves) in a fixed order and send one token row per lane to every rank
       float* rw = red + ((size_t)hb * 32 + sub * 16) * TP_PS;
       {
-        float s0 = sum2(sq0[0]) + sum2(sq0[1]), s1 = sum2(sq1[0]) + sum2(sq1[1]);
-        s0 += __shfl_xor_sync(0xffffffffu, s0, 1);
-        s0 += __shfl_xor_sync(0xffffffffu, s0, 2);
-        s1 += __shfl_xor_sync(0xffffffffu, s1, 1);
-        s1 += __shfl_xor_sync(0xffffffffu, s1, 2);
+        // token g8's diagonal entry is column g8 of row g8: lane (g8, g8 / 2),
+        // element 0 or 1 by parity; token g8 + 8's is row g8 + 8 of the
+        // second product, elements 2 or 3
+        const bool diag = (g8 >> 1) == q;
+        const float s0 = (g8 & 1) ? dl[1] : dl[0];
+        const float s1 = (g8 & 1) ? dh[3] : dh[2];
         if (2 * q < M) {
           rw[g8 * TP_PS + 2 * q] = acc[0][0] + acc[1][0];
           rw[(g8 + 8) * TP_PS + 2 * q] = acc[0][2] + acc[1][2];
@@ -1063,7 +1065,7 @@ __global__ void __launch_bounds__(TP_THR, 1) gated_reduce_tile_kernel(const Redu
           rw[g8 * TP_PS + 2 * q + 1] = acc[0][1] + acc[1][1];
           rw[(g8 + 8) * TP_PS + 2 * q + 1] = acc[0][3] + acc[1][3];
         }
-        if (q == 0) {
+        if (diag) {
           rw[g8 * TP_PS + M] = s0;
           rw[(g8 + 8) * TP_PS + M] = s1;
         }
