@@ -34,6 +34,7 @@ import torch
 ROOT = os.path.dirname(os.path.abspath(__file__))
 sys.path.insert(0, ROOT)
 
+from paper_2606_26744_gb300 import dist  # noqa: E402
 from paper_2606_26744_gb300 import workloads as W  # noqa: E402
 
 METRIC = "draft blocks/sec"
@@ -145,7 +146,7 @@ def run_ours(args, rank, world, local_rank, config=None, light=False):
     if config is None and args.overrides:
         cfg = W.scaled(cfg, name=cfg.name + "-" + "-".join(f"{k}{v}" for k, v in args.overrides.items()),
                        **args.overrides)
-    seed = 1000 + 17 * rank
+    seed = dist.rank_seed(1000, rank)
     inp = W.make_draft_inputs(cfg, seed, device=dev)
     lens = inp["ctx_lens"]
     n_ctx = sum(lens)
@@ -312,6 +313,8 @@ def run_ours(args, rank, world, local_rank, config=None, light=False):
     if light:
         del graph, staged, stepped, inp, w, drafter, H, y, h, ws
         torch.cuda.empty_cache()
+        if world > 1:
+            ms, = dist.max_over_ranks([ms], device=dev)
         return dict(cfg=cfg, ms=ms, ms_staged=ms_staged, dur=dur, pct=pct, batch=batch, n_ctx=n_ctx, lens=lens,
                     acc_mean=acc_mean)
 
@@ -477,9 +480,7 @@ def run_ours(args, rank, world, local_rank, config=None, light=False):
 
     # ----------------------------------------------------- max over ranks
     if world > 1:
-        t = torch.tensor([ms, e2e_ms], device=dev)
-        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
-        ms, e2e_ms = float(t[0]), float(t[1])
+        ms, e2e_ms = dist.max_over_ranks([ms, e2e_ms], device=dev)
     return dict(cfg=cfg, ms=ms, ms_staged=ms_staged, e2e_ms=e2e_ms, dur=dur, clk=clk, kl=kl, draft_loss=draft_loss,
                 verify_t1=verify_t1,
                 reduce_bwd=reduce_bwd,
@@ -1133,8 +1134,8 @@ def main():
     if rank == 0:
         pk = peaks()
         rf, stages = roofline_of(cfg, res, pk)
-        val = res["batch"] * world / (res["ms"] / 1e3)
-        e2e_val = res["batch"] * world / (res["e2e_ms"] / 1e3)
+        val = dist.whole_job_rate(res["batch"], world, res["ms"])
+        e2e_val = dist.whole_job_rate(res["batch"], world, res["e2e_ms"])
         cb = None
         if not args.no_cpu_baseline:
             cpu_inp = {k: v for k, v in res["inputs"].items()}
@@ -1183,7 +1184,7 @@ def main():
     if rank == 0:
         if sec is not None:
             srf, sstages = roofline_of(sec["cfg"], sec, pk)
-            line["decode"] = {"workload": "decode", "value": round(sec["batch"] * world / (sec["ms"] / 1e3), 2),
+            line["decode"] = {"workload": "decode", "value": round(dist.whole_job_rate(sec["batch"], world, sec["ms"]), 2),
                               "unit": UNIT, "ms_per_step": round(sec["ms"], 5),
                               "ms_per_step_instrumented": round(sec["ms_staged"], 5),
                               "step_ms_percentiles": sec["pct"], "roofline": srf, "stages": sstages,

@@ -34,3 +34,12 @@ def max_over_ranks(values: Sequence[float], device=None) -> List[float]:
                      device=device if device is not None else "cpu")
     torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
     return [float(v) for v in t.tolist()]
+
+
+def whole_job_rate(units_per_rank: int, world: int, ms_per_step_max: float) -> float:
+    """Whole-job throughput of N replicas in units per second: every rank
+    processes units_per_rank units per step, and the job's step takes the
+    slowest rank's time (ms_per_step_max, the max over ranks)."""
+    if world <= 0 or ms_per_step_max <= 0:
+        raise ValueError("world and step time must be positive")
+    return units_per_rank * world / (ms_per_step_max / 1e3)

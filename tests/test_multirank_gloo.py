@@ -76,3 +76,44 @@ def test_shard_edges():
     with pytest.raises(ValueError):
         dist.shard(5, 3, 3)
     assert dist.max_over_ranks([3.5]) == [3.5]
+
+
+def _bench_worker(rank, world, port, q):
+    """The bench's replica bookkeeping on one rank: its own seed and
+    synthetic draft inputs, its step time reduced to the maximum over ranks,
+    and the whole-job rate computed from it (the calls bench.py makes)."""
+    os.environ["MASTER_ADDR"] = "127.0.0.1"
+    os.environ["MASTER_PORT"] = str(port)
+    torch.distributed.init_process_group("gloo", rank=rank, world_size=world)
+    try:
+        cfg = W.CONFIGS["tiny"]
+        seed = dist.rank_seed(1000, rank)
+        inp = W.make_draft_inputs(cfg, seed, device="cpu")
+        ms_here = 2.0 + rank  # this rank's step time
+        ms, e2e = dist.max_over_ranks([ms_here, 10.0 * (world - rank)])
+        rate = dist.whole_job_rate(cfg.batch, world, ms)
+        q.put((rank, float(inp["H"].double().sum()), ms, e2e, rate))
+    finally:
+        torch.distributed.destroy_process_group()
+
+
+def test_two_rank_bench_bookkeeping():
+    world = 2
+    ctx = mp.get_context("spawn")
+    q = ctx.Queue()
+    port = _free_port()
+    procs = [ctx.Process(target=_bench_worker, args=(r, world, port, q)) for r in range(world)]
+    for p in procs:
+        p.start()
+    out = sorted(q.get(timeout=120) for _ in range(world))
+    for p in procs:
+        p.join(timeout=60)
+        assert p.exitcode == 0
+    # distinct synthetic inputs per rank; every rank sees the slowest rank's times
+    assert out[0][1] != out[1][1]
+    for _, _, ms, e2e, rate in out:
+        assert ms == 3.0 and e2e == 20.0
+        # whole job: both ranks' blocks over the slowest rank's step
+        assert rate == W.CONFIGS["tiny"].batch * world / (3.0 / 1e3)
+    with pytest.raises(ValueError):
+        dist.whole_job_rate(1, 0, 1.0)
