@@ -677,7 +677,7 @@ NCU_DRAM_BYTES_PER_CTX_ROW = {
 # DRAM bytes (read + write) per token of the tile reducer at m = 4, d = 7168,
 # from the ncu capture summarised in profiles/gated_reduce_sweep.md (16,384
 # tokens; traffic grows with the tokens)
-NCU_DRAM_BYTES_PER_TOKEN_SWEEP = (946359808 + 203782144) / 16384
+NCU_DRAM_BYTES_PER_TOKEN_SWEEP = (946523392 + 203869696) / 16384
 
 
 def tensor_peak(pk, step_ms):
@@ -711,6 +711,10 @@ def roofline_of(cfg, res, pk):
         ach = flop / t / 1e12
         rf = {"kernel": dom, "bound": "tensor", "achieved": round(ach, 2), "peak": tc_peak,
               "unit": "TFLOP/s", "frac": round(ach / tc_peak, 4), "traffic": None, "peak_source": tc_src}
+        if tc_peak != pk["bf16_tflops_sustained"]:
+            # the same kernel against the power-capped figure (seconds-long loops
+            # of a dense GEMM settle there; the clocks record says whether this run did)
+            rf["frac_of_sustained"] = round(ach / pk["bf16_tflops_sustained"], 4)
     else:
         ach = byt / t / 1e9
         rf = {"kernel": dom, "bound": "hbm", "achieved": round(ach, 1), "peak": pk["hbm_gbs"], "unit": "GB/s",
