@@ -311,12 +311,15 @@ def run_ours(args, rank, world, local_rank, config=None, light=False):
                            "the step timer does not bracket the work")
 
     if light:
+        warm = None
+        if light == "warm":
+            warm = measure_warm(cfg, inp, drafter, y, tok.clone(), tgt, stream, min(K, 100), dev, peaks())
         del graph, staged, stepped, inp, w, drafter, H, y, h, ws
         torch.cuda.empty_cache()
         if world > 1:
             ms, = dist.max_over_ranks([ms], device=dev)
         return dict(cfg=cfg, ms=ms, ms_staged=ms_staged, dur=dur, pct=pct, batch=batch, n_ctx=n_ctx, lens=lens,
-                    acc_mean=acc_mean)
+                    acc_mean=acc_mean, warm=warm)
 
     # ------------------------------------------------ KL target (Eq. 2)
     # teacher / student log-softmax rows of the first P = 2 block positions
@@ -534,16 +537,18 @@ def _timing_event():
 
 
 def warm_launches(cfg):
-    # reduce; append: norm, one K/V GEMM per layer, length advance; cached
-    # block: 7 kernels per layer and the final norm; LM head (2); accept
+    # reduce; the round's append: norm, one K/V GEMM per layer, length
+    # advance; its cached block: 7 kernels per layer and the final norm;
+    # LM head (2); accept
     return 1 + (2 + cfg.n_layers) + (7 * cfg.n_layers + 1) + 2 + 1
 
 
 def measure_warm(cfg, inp, drafter, y, tok_cold, tgt, stream, steps, dev, pk):
     """One serving round of the incremental path, as one CUDA graph: rewind
     the cache lengths, reduce the residuals of the WARM_NEW_ROWS newest tokens
-    of every sequence, append them to the K/V cache, block forward over the
-    cache, LM head, accepted length.  The cache holds every other context row
+    of every sequence, append them to the K/V cache and run the block forward
+    over the cache (one hdf_draft_round call: the first block path runs
+    beside the append), LM head, accepted length.  The cache holds every other context row
     (appended once, untimed), so each round drafts over the same contexts as
     the cold step and must give its drafts exactly."""
     from paper_2606_26744_gb300 import hdf
@@ -566,8 +571,8 @@ def measure_warm(cfg, inp, drafter, y, tok_cold, tgt, stream, steps, dev, pk):
         n_new = int(sum(new))
         cu_new = torch.tensor([0] + list(np.cumsum(new)), dtype=torch.int32, device=dev)
         y_new = torch.empty((n_new, d), dtype=cfg.torch_dtype, device=dev)
-        ws_a = torch.empty(max(1, drafter.append_workspace_size(batch, B, n_new)), dtype=torch.uint8, device=dev)
-        ws_c = torch.empty(max(1, drafter.cached_workspace_size(batch, B, max_ctx)), dtype=torch.uint8, device=dev)
+        ws_r = torch.empty(max(1, drafter.round_workspace_size(batch, B, n_new, max_ctx)), dtype=torch.uint8,
+                           device=dev)
         M = batch * B
         h = torch.empty((M, d), dtype=cfg.torch_dtype, device=dev)
         tok = torch.empty(M, dtype=torch.int32, device=dev)
@@ -578,7 +583,7 @@ def measure_warm(cfg, inp, drafter, y, tok_cold, tgt, stream, steps, dev, pk):
         acc = torch.empty(batch, dtype=torch.int32, device=dev)
         anchor = inp["anchor"].to(dev)
     stream.synchronize()
-    names = ["reduce", "append", "draft_block_cached", "lm_head", "accept"]
+    names = ["reduce", "round", "lm_head", "accept"]
 
     def wstep(ev=None):
         def mark(i):
@@ -589,15 +594,14 @@ def measure_warm(cfg, inp, drafter, y, tok_cold, tgt, stream, steps, dev, pk):
         mark(0)
         hdf.hdf_gated_reduce(H_new, Wf, b, y=y_new, stream=stream)
         mark(1)
-        drafter.hdf_ctx_append(y_new, cu_new, cache, block=B, ws=ws_a, stream=stream)
+        drafter.hdf_draft_round(y_new, cu_new, cache, anchor, block=B, max_ctx=max_ctx, h_out=h, ws=ws_r,
+                                stream=stream)
         mark(2)
-        drafter.hdf_draft_block_cached(cache, anchor, block=B, max_ctx=max_ctx, h_out=h, ws=ws_c, stream=stream)
-        mark(3)
         hdf.hdf_lm_head_argmax(h, w["lm_head"], logsoftmax=cfg.logsoftmax, tok=tok, zmax=zmax, ls=ls, ws=lmws,
                                stream=stream)
-        mark(4)
+        mark(3)
         hdf.hdf_accept_len(tok[1:], tgt, n_draft=B - 1, draft_stride=B, batch=batch, accept=acc, stream=stream)
-        mark(5)
+        mark(4)
 
     for _ in range(3):
         wstep()
@@ -608,7 +612,7 @@ def measure_warm(cfg, inp, drafter, y, tok_cold, tgt, stream, steps, dev, pk):
     if not same:
         raise RuntimeError("warm step drafts differ from the cold step's")
     K = steps
-    evs = [[_timing_event() for _ in range(6)] for _ in range(K)]
+    evs = [[_timing_event() for _ in range(len(names) + 1)] for _ in range(K)]
     for e in [x for row in evs for x in row]:
         e.record(stream)
     stream.synchronize()
@@ -1125,6 +1129,8 @@ def main():
     ap.add_argument("--no-secondary", action="store_true", help="skip the decode step measured beside the large one")
     ap.add_argument("--step-only", action="store_true",
                     help="time the cold step alone and print its stages (profiling runs; not a bench line)")
+    ap.add_argument("--with-warm", action="store_true",
+                    help="with --step-only: also time the incremental serving round")
     ap.add_argument("--batch", type=int, default=None, help="profiling override of the workload's batch")
     ap.add_argument("--vocab", type=int, default=None, help="profiling override of the workload's vocabulary")
     ap.add_argument("--layers", type=int, default=None, help="profiling override of the workload's layers")
@@ -1159,12 +1165,12 @@ def main():
     if world > 1:
         torch.distributed.barrier()
     if args.step_only:
-        res = run_ours(args, rank, world, local_rank, light=True)
+        res = run_ours(args, rank, world, local_rank, light="warm" if args.with_warm else True)
         if rank == 0:
             rf, stages = roofline_of(res["cfg"], res, peaks())
             print(json.dumps({"workload": res["cfg"].name, "ms_per_step": round(res["ms"], 5),
                               "ms_per_step_instrumented": round(res["ms_staged"], 5), "roofline": rf,
-                              "stages": stages}), flush=True)
+                              "stages": stages, "warm_step": res["warm"]}), flush=True)
         return 0
     res = run_ours(args, rank, world, local_rank)
     cfg = res["cfg"]

@@ -345,6 +345,24 @@ HDF_API int hdf_draft_block_cached(const hdf_drafter_weights* w, const hdf_draft
                                    void* ws, size_t ws_bytes, const hdf_trace* trace,
                                    hdf_stream_t stream);
 
+/* One serving round: hdf_ctx_append of the new rows followed by
+ * hdf_draft_block_cached, with the same results bit for bit (h_out, the
+ * cache rows and len).  The block's input norm and Q / K_b / V_b projection
+ * of the first layer do not depend on the new rows, so they run on a second
+ * stream beside the append (their RoPE positions are len[i] + n_i, the
+ * lengths the append leaves); the lengths are advanced once both are done,
+ * before the first attention.  Run serially when stage times are traced.
+ * shape.n_ctx is the host's row count of ctx_new (as for hdf_ctx_append);
+ * shape.max_ctx bounds every len[i] after the append (as for
+ * hdf_draft_block_cached).  Requires rope_max_pos >= capacity and
+ * >= max_ctx + block.  Errors as the two calls.
+ * Workspace: hdf_draft_round_workspace_size(shape), 256-byte aligned. */
+HDF_API size_t hdf_draft_round_workspace_size(const hdf_draft_shape* shape);
+HDF_API int hdf_draft_round(const hdf_drafter_weights* w, const hdf_draft_shape* shape,
+                            const void* ctx_new, const int32_t* cu_new, const hdf_ctx_cache* cache,
+                            const int32_t* anchor, void* h_out, void* ws, size_t ws_bytes,
+                            hdf_stream_t stream);
+
 /* cos/sin tables for the drafter's RoPE: entry [p][i] = cos/sin of
  * p * theta^(-2i/head_dim), computed in fp64 on the device and stored fp32.
  * A per-model constant: build once, pass through hdf_drafter_weights. */

@@ -78,7 +78,8 @@ __device__ __forceinline__ int ctx_position(const int* cu, int batch, long long 
 }
 __device__ __forceinline__ int block_position(const Epilogue& E, int j) {
   const int b = j / E.block;
-  const int T = E.pos_mode == 4 ? __ldg(E.ctx_len + b) : __ldg(E.cu_ctx + b + 1) - __ldg(E.cu_ctx + b);
+  const int n = E.pos_mode == 4 ? 0 : __ldg(E.cu_ctx + b + 1) - __ldg(E.cu_ctx + b);
+  const int T = E.pos_mode >= 4 ? __ldg(E.ctx_len + b) + n : n;
   return T + (j - b * E.block);
 }
 

@@ -258,7 +258,12 @@ DraftLayout draft_layout(const hdf_draft_shape* sh) {
   L.o = take(M * d * es);
   L.act = take(M * F * es);
   L.chunk = attn_chunk(sh, &L.n_chunks);
+  // The block path's Q / K_b / V_b projection runs beside the context
+  // projection (cold step) or the append (serving round), on the SM slots
+  // those leave: it takes no K split, which would multiply its CTAs past those
+  // slots and queue them behind the projection.
   L.qkv = plan_swap(sh->dtype, 3 * d, M, d);
+  L.qkv.k_splits = 1;
   L.oproj = plan_swap(sh->dtype, d, M, d);
   L.gu = plan_swap(sh->dtype, 2 * F, M, d);
   L.down = plan_swap(sh->dtype, d, M, F);
@@ -288,7 +293,7 @@ int check_draft_shape(const hdf_draft_shape* sh) {
 // =====================================================================
 extern "C" {
 
-int hdf_version(void) { return 101; }
+int hdf_version(void) { return 102; }
 
 const char* hdf_status_str(int s) {
   switch (s) {
@@ -671,11 +676,37 @@ SideStream* side_stream(size_t n_events) {
   return &ss;
 }
 
+// New context rows of a serving round (hdf_draft_round): their reduced
+// states, row offsets, count and the workspace their normed copy goes to.
+struct AppendIn {
+  const void* ctx_new;
+  const int32_t* cu_new;
+  long long n_new;
+  void* c;
+};
+
+// c = RMSNorm(ctx_new), then every layer's K_c / V_c rows written at
+// positions len[i].. of the cache (mode 3); the lengths are left alone.
+int append_rows(const hdf_drafter_weights* w, const hdf_draft_shape* sh, const AppendIn& ap,
+                const hdf_ctx_cache* cache, cudaStream_t s) {
+  int rc;
+  CK(launch_rmsnorm(ap.ctx_new, 0, w->ctx_norm, ap.c, sh->dtype, ap.n_new, sh->d, sh->norm_eps, s), "ctx norm");
+  for (int l = 0; l < sh->n_layers; ++l) {
+    char* kl = static_cast<char*>(cache->k) + cache_layer_offset(sh, cache, l);
+    char* vl = static_cast<char*>(cache->v) + cache_layer_offset(sh, cache, l);
+    if ((rc = launch_ctx_kv(w, w->layers[l], sh, ap.c, ap.n_new, kl, vl, ap.cu_new, 3, cache->len,
+                            cache->capacity, s)))
+      return rc;
+  }
+  return HDF_OK;
+}
+
 // The block forward of hdf_draft_block.  Context from packed rows (ctx,
 // cu_ctx: normed and projected here) or from a K/V cache (cache != null).
+// With ap (cached only): the serving round, new rows appended first.
 int draft_forward(const hdf_drafter_weights* w, const hdf_draft_shape* sh, const void* ctx, const int32_t* cu_ctx,
                   const hdf_ctx_cache* cache, const int32_t* anchor, void* h_out, void* ws, size_t ws_bytes,
-                  const hdf_trace* trace, cudaStream_t s) {
+                  const hdf_trace* trace, cudaStream_t s, const AppendIn* ap = nullptr) {
   int rc;
   const int dt = sh->dtype;
   const long long M = (long long)sh->batch * sh->block;
@@ -727,9 +758,22 @@ int draft_forward(const hdf_drafter_weights* w, const hdf_draft_shape* sh, const
   // layers' projections go on the second stream, forked once the previous
   // layer's attention has read the shared K/V buffers, beside that layer's
   // MLP and the next block path.  Serial when stage times are traced.
+  //
+  // In a serving round the new rows' append (norm and every layer's K/V
+  // rows) stays on the caller's stream and the first block path is forked
+  // before it; the lengths advance after both, before the first attention.
+  const bool round = cached && ap && ap->n_new > 0;
   SideStream* side = nullptr;
-  if (!trace && n_ctx > 0) side = side_stream(2 * (size_t)sh->n_layers + 1);
+  if (!trace && (n_ctx > 0 || round)) side = side_stream(2 * (size_t)sh->n_layers + 1);
   const cudaStream_t s2 = side ? side->s : s;
+  const bool beside_append = round && side;
+  if (round) {
+    if (side) CK(cudaEventRecord(side->ev[0], s), "fork record");  // the block path needs nothing new
+    if ((rc = append_rows(w, sh, *ap, cache, s))) return rc;
+    if (!side)
+      CK(launch_cache_advance(cache->len, ap->cu_new, sh->batch, cache->capacity, device_status_ptr(), s),
+         "cache advance");
+  }
   // ---- context RMSNorm
   if ((rc = mark())) return rc;
   if (n_ctx > 0) CK(launch_rmsnorm(ctx, 0, w->ctx_norm, c, dt, n_ctx, (int)d, sh->norm_eps, s), "ctx norm");
@@ -741,7 +785,7 @@ int draft_forward(const hdf_drafter_weights* w, const hdf_draft_shape* sh, const
     const cudaStream_t s_blk = l == 0 ? s2 : s;
     // ---- conditioning projection: [K_c | V_c] = c [W_k; W_v]^T, RoPE on K_c
     if ((rc = mark())) return rc;
-    if (side && l == 0) CK(cudaEventRecord(side->ev[0], s), "fork record");  // behind the context norm
+    if (side && l == 0 && !round) CK(cudaEventRecord(side->ev[0], s), "fork record");  // behind the context norm
     if (side && l > 0) CK(cudaStreamWaitEvent(s2, side->ev[2 * l], 0), "fork wait");  // behind attention l-1
     if (n_ctx > 0 &&
         (rc = launch_ctx_kv(w, Lw, sh, c, n_ctx, kc, vc, cu_ctx, 1, nullptr, 0, s_ctx)))
@@ -787,11 +831,12 @@ int draft_forward(const hdf_drafter_weights* w, const hdf_draft_shape* sh, const
       g.epi.rope_sin = w->rope_sin;
       g.epi.rope_rows = w->rope_max_pos;
       g.epi.head_dim = sh->head_dim;
-      g.epi.cu_ctx = cu_ctx;
+      const bool pending = beside_append && l == 0;  // the lengths do not count the new rows yet
+      g.epi.cu_ctx = pending ? ap->cu_new : cu_ctx;
       g.epi.ctx_len = cached ? cache->len : nullptr;
       g.epi.batch = sh->batch;
       g.epi.block = sh->block;
-      g.epi.pos_mode = cached ? 4 : 2;
+      g.epi.pos_mode = cached ? (pending ? 5 : 4) : 2;
       CK(launch_gemm(g, s_blk), "qkv gemm");
       if (side && l == 0) CK(cudaEventRecord(side->ev[1], s2), "join record");
     }
@@ -830,6 +875,9 @@ int draft_forward(const hdf_drafter_weights* w, const hdf_draft_shape* sh, const
         if ((rc = make_map(&tm.vb, vbk, dt, M, d, d, 64))) return rc;
       }
       if (side) CK(cudaStreamWaitEvent(s, side->ev[2 * l + 1], 0), "join wait");
+      if (beside_append && l == 0)
+        CK(launch_cache_advance(cache->len, ap->cu_new, sh->batch, cache->capacity, device_status_ptr(), s),
+           "cache advance");
       CK(launch_attention(a, &tm, dt, s), "attention");
       if (side && l + 1 < sh->n_layers) CK(cudaEventRecord(side->ev[2 * l + 2], s), "attention-done record");
     }
@@ -977,18 +1025,56 @@ int hdf_ctx_append(const hdf_drafter_weights* w, const hdf_draft_shape* sh, cons
   if (!ws || ws_bytes < need || (reinterpret_cast<uintptr_t>(ws) & 255))
     return fail(HDF_ERR_WORKSPACE, "workspace %zu bytes (need %zu, 256-byte aligned)", ws_bytes, need);
   cudaStream_t s = (cudaStream_t)stream;
-  const long long d = sh->d;
-  void* c = ws;
-  CK(launch_rmsnorm(ctx_new, 0, w->ctx_norm, c, sh->dtype, sh->n_ctx, (int)d, sh->norm_eps, s), "ctx norm");
-  for (int l = 0; l < sh->n_layers; ++l) {
-    char* kl = static_cast<char*>(cache->k) + cache_layer_offset(sh, cache, l);
-    char* vl = static_cast<char*>(cache->v) + cache_layer_offset(sh, cache, l);
-    if ((rc = launch_ctx_kv(w, w->layers[l], sh, c, sh->n_ctx, kl, vl, cu_new, 3, cache->len,
-                            cache->capacity, s)))
-      return rc;
-  }
+  const AppendIn ap{ctx_new, cu_new, sh->n_ctx, ws};
+  if ((rc = append_rows(w, sh, ap, cache, s))) return rc;
   CK(launch_cache_advance(cache->len, cu_new, sh->batch, cache->capacity, device_status_ptr(), s), "cache advance");
   return HDF_OK;
+}
+
+size_t hdf_draft_round_workspace_size(const hdf_draft_shape* shape) {
+  if (check_draft_shape(shape) != HDF_OK) return 0;
+  return hdf_ctx_append_workspace_size(shape) + hdf_draft_block_cached_workspace_size(shape);
+}
+
+int hdf_draft_round(const hdf_drafter_weights* w, const hdf_draft_shape* sh, const void* ctx_new,
+                    const int32_t* cu_new, const hdf_ctx_cache* cache, const int32_t* anchor, void* h_out, void* ws,
+                    size_t ws_bytes, hdf_stream_t stream) {
+  g_err.clear();
+  int rc = check_draft_shape(sh);
+  if (rc) return rc;
+  if ((rc = check_drafter_weights(w, sh))) return rc;
+  if ((rc = check_cache(cache, sh))) return rc;
+  const long long n_new = sh->batch > 0 ? sh->n_ctx : 0;
+  const bool has_block = (long long)sh->batch * sh->block > 0;
+  if (n_new == 0 && !has_block) return HDF_OK;
+  if (n_new > 0) {
+    if (!ctx_new || !cu_new) return fail(HDF_ERR_INVALID_ARG, "ctx_new / cu_new NULL");
+    if (!aligned16(ctx_new)) return fail(HDF_ERR_ALIGNMENT, "ctx_new not 16-byte aligned");
+    if (w->rope_max_pos < cache->capacity)
+      return fail(HDF_ERR_SHAPE, "rope_max_pos %lld < cache capacity %d", (long long)w->rope_max_pos,
+                  cache->capacity);
+  }
+  if (has_block) {
+    if (sh->max_ctx > cache->capacity)
+      return fail(HDF_ERR_SHAPE, "max_ctx %d > cache capacity %d", sh->max_ctx, cache->capacity);
+    if (!anchor || !h_out) return fail(HDF_ERR_INVALID_ARG, "null input");
+    if (!aligned16(h_out)) return fail(HDF_ERR_ALIGNMENT, "h_out not 16-byte aligned");
+    if (w->rope_max_pos < (long long)sh->max_ctx + sh->block)
+      return fail(HDF_ERR_SHAPE, "rope_max_pos %lld < max_ctx + block", (long long)w->rope_max_pos);
+  }
+  const size_t need_a = hdf_ctx_append_workspace_size(sh);
+  const size_t need = hdf_draft_round_workspace_size(sh);
+  if (!ws || ws_bytes < need || (reinterpret_cast<uintptr_t>(ws) & 255))
+    return fail(HDF_ERR_WORKSPACE, "workspace %zu bytes (need %zu, 256-byte aligned)", ws_bytes, need);
+  cudaStream_t s = (cudaStream_t)stream;
+  const AppendIn ap{ctx_new, cu_new, n_new, ws};
+  if (!has_block) {  // nothing to draft: the append alone
+    if ((rc = append_rows(w, sh, ap, cache, s))) return rc;
+    CK(launch_cache_advance(cache->len, cu_new, sh->batch, cache->capacity, device_status_ptr(), s), "cache advance");
+    return HDF_OK;
+  }
+  return draft_forward(w, sh, nullptr, nullptr, cache, anchor, h_out, static_cast<char*>(ws) + need_a,
+                       ws_bytes - need_a, nullptr, s, &ap);
 }
 
 // -------------------------------------------------------------- LM head

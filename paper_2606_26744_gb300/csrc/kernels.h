@@ -133,8 +133,9 @@ struct Epilogue {
   int batch;
   int block;            // block rows: pos = T_b + (j % block)
   int pos_mode;         // 0 none, 1 context rows, 2 block rows (T_b from cu_ctx),
-                        // 3 context rows appended to a cache, 4 block rows (T_b = ctx_len[b])
-  const int* ctx_len;   // modes 3, 4: rows already in the cache per sequence
+                        // 3 context rows appended to a cache, 4 block rows (T_b = ctx_len[b]),
+                        // 5 block rows beside an append (T_b = ctx_len[b] + cu[b+1] - cu[b])
+  const int* ctx_len;   // modes 3, 4, 5: rows already in the cache per sequence
   long long cache_cap;  // mode 3: row t of sequence b goes to row b * cache_cap + ctx_len[b] + t - cu[b]
   float* resid;         // kEpiResidT
   // kEpiLmHeadT

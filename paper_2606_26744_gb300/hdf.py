@@ -86,6 +86,9 @@ _SIGS = {
     "hdf_draft_block_cached": (c_int, [ctypes.POINTER(DrafterWeights), ctypes.POINTER(DraftShape),
                                        ctypes.POINTER(CtxCache), c_vp, c_vp, c_vp, c_size, ctypes.POINTER(Trace),
                                        c_vp]),
+    "hdf_draft_round_workspace_size": (c_size, [ctypes.POINTER(DraftShape)]),
+    "hdf_draft_round": (c_int, [ctypes.POINTER(DrafterWeights), ctypes.POINTER(DraftShape), c_vp, c_vp,
+                                ctypes.POINTER(CtxCache), c_vp, c_vp, c_vp, c_size, c_vp]),
     "hdf_rope_table": (c_int, [ctypes.c_double, c_int, c_i64, c_vp, c_vp, c_vp]),
     "hdf_lm_head_workspace_size": (c_size, [c_i64, c_int, c_i64, c_int]),
     "hdf_lm_head_argmax": (c_int, [c_vp, c_int, c_i64, c_int, c_vp, c_i64, c_float, c_vp, c_vp, c_vp,
@@ -345,6 +348,30 @@ class Drafter:
         _check(lib.hdf_draft_block_cached(ctypes.byref(self._w), ctypes.byref(sh), ctypes.byref(cache.c),
                                           _p(anchor), _p(h_out), _p(ws), ws.numel(),
                                           ctypes.byref(tr) if tr is not None else None, _stream(stream)))
+        return h_out
+
+
+    def round_workspace_size(self, batch: int, block: int, n_new: int, max_ctx: int) -> int:
+        sh = self.shape(batch, block, n_new, max_ctx)
+        return load().hdf_draft_round_workspace_size(ctypes.byref(sh))
+
+    def hdf_draft_round(self, ctx_new: torch.Tensor, cu_new: torch.Tensor, cache: "ContextCache",
+                        anchor: torch.Tensor, *, block: int, max_ctx: int, h_out: Optional[torch.Tensor] = None,
+                        ws: Optional[torch.Tensor] = None, stream=None) -> torch.Tensor:
+        """hdf_ctx_append(ctx_new, cu_new) then hdf_draft_block_cached, in one
+        call whose first block path runs beside the append."""
+        batch = anchor.shape[0]
+        sh = self.shape(batch, block, ctx_new.shape[0], max_ctx)
+        lib = load()
+        dev = anchor.device
+        if ws is None:
+            ws = torch.empty(max(lib.hdf_draft_round_workspace_size(ctypes.byref(sh)), 1), dtype=torch.uint8,
+                             device=dev)
+        if h_out is None:
+            h_out = torch.empty((batch * block, self.d), dtype=self.w["embed"].dtype, device=dev)
+        _check(lib.hdf_draft_round(ctypes.byref(self._w), ctypes.byref(sh), _p(ctx_new), _p(cu_new),
+                                   ctypes.byref(cache.c), _p(anchor), _p(h_out), _p(ws), ws.numel(),
+                                   _stream(stream)))
         return h_out
 
 

@@ -26,7 +26,7 @@ def test_every_declared_symbol_is_exported(lib):
 
 
 def test_status_strings(lib):
-    assert lib.hdf_version() == 101
+    assert lib.hdf_version() == 102
     assert lib.hdf_status_str(0) == b"ok"
     assert b"aligned" in lib.hdf_status_str(4)
 
@@ -217,3 +217,33 @@ def test_ctx_cache_host_validation(lib):
     cold = hdf.DraftShape(1, 4, 16, 2048, 16, 128, 8192, 32768, 2, 4096, 4 * 4096, 1e-6)
     assert (lib.hdf_draft_block_cached_workspace_size(ctypes.byref(cold)) + 3 * 4 * 4096 * 2048 * 2
             <= lib.hdf_draft_block_workspace_size(ctypes.byref(cold)))
+
+
+def test_draft_round_host_validation(lib):
+    v = ctypes.c_void_p
+    w, _keep = _fake_weights(2, 4096 + 16)
+    sh = hdf.DraftShape(1, 4, 16, 2048, 16, 128, 8192, 32768, 2, 4096, 20, 1e-6)   # 20 new rows
+    good = hdf.CtxCache(4096, 8192, 256, 4096)
+    ws = v(1 << 24)
+    need = lib.hdf_draft_round_workspace_size(ctypes.byref(sh))
+    # the append's normed rows, then the cached block's workspace
+    assert need == lib.hdf_ctx_append_workspace_size(ctypes.byref(sh)) + \
+        lib.hdf_draft_block_cached_workspace_size(ctypes.byref(sh))
+    args = lambda **k: [k.get("w", ctypes.byref(w)), k.get("sh", ctypes.byref(sh)), k.get("ctx", v(4096)),
+                        k.get("cu", v(256)), k.get("cache", ctypes.byref(good)), k.get("anchor", v(256)),
+                        k.get("h", v(4096)), k.get("ws", ws), k.get("nb", need), None]
+    assert lib.hdf_draft_round(*args(cache=None)) == 1
+    assert lib.hdf_draft_round(*args(ctx=None)) == 1
+    assert lib.hdf_draft_round(*args(anchor=None)) == 1
+    assert lib.hdf_draft_round(*args(ctx=v(4100))) == 4
+    assert lib.hdf_draft_round(*args(h=v(4100))) == 4
+    assert lib.hdf_draft_round(*args(nb=need - 1)) == 5
+    assert lib.hdf_draft_round(*args(ws=v(1 << 24 | 128))) == 5
+    small = hdf.CtxCache(4096, 8192, 256, 1024)   # max_ctx 4096 above the capacity
+    assert lib.hdf_draft_round(*args(cache=ctypes.byref(small))) == 2
+    w_short, _k2 = _fake_weights(2, 1000)
+    assert lib.hdf_draft_round(*args(w=ctypes.byref(w_short))) == 2
+    # nothing to append and no block: returns before any launch
+    none = hdf.DraftShape(1, 0, 16, 2048, 16, 128, 8192, 32768, 2, 4096, 0, 1e-6)
+    assert lib.hdf_draft_round(*args(sh=ctypes.byref(none), ctx=None, cu=None, anchor=None, h=None, ws=None,
+                                     nb=0)) == 0

@@ -265,3 +265,104 @@ def test_large_workload_full_size_warm_equals_cold():
     assert hdf.device_status() == 0
     assert cache.len.cpu().tolist() == list(lens)
     assert torch.equal(h_warm.view(torch.int16), h_cold.view(torch.int16))
+
+
+def _check_round_equals_two_calls(cfg_base, seed, lens, n_rounds, pad_rows=0):
+    """hdf_draft_round (the first block path beside the append) against
+    hdf_ctx_append + hdf_draft_block_cached, round after round: the same
+    h_out, cache rows and lengths, bit for bit; after the last round both
+    equal the cold step."""
+    rng = np.random.default_rng(seed)
+    cfg, inp, drafter, wc, cu, max_ctx = _setup(cfg_base, seed, lens)
+    y, h_cold = _cold(drafter, cfg, inp, max_ctx)
+    cap = max_ctx + 7
+    c_round = _nan_cache(drafter, cfg.batch, cap)
+    c_two = _nan_cache(drafter, cfg.batch, cap)
+    c_round.len.zero_()
+    c_two.len.zero_()
+    pieces = _rounds(lens, n_rounds, rng)
+    anchor = inp["anchor"].cuda()
+    bits = torch.int16 if h_cold.dtype == torch.bfloat16 else torch.int32
+    done = np.zeros(cfg.batch, dtype=np.int64)
+    for r in range(pieces.shape[0]):
+        idx = [cu[i] + done[i] + j for i in range(cfg.batch) for j in range(pieces[r, i])]
+        done += pieces[r]
+        n = len(idx)
+        y_new = torch.zeros((n + pad_rows, cfg.d), dtype=y.dtype, device="cuda")
+        if n:
+            y_new[:n] = y[torch.tensor(idx, device="cuda")]
+        if pad_rows:
+            y_new[n:] = torch.randn_like(y_new[n:], dtype=torch.float32).to(y.dtype)  # never appended
+        cu_new = torch.tensor(np.concatenate([[0], np.cumsum(pieces[r])]).astype(np.int32), device="cuda")
+        h_round = drafter.hdf_draft_round(y_new, cu_new, c_round, anchor, block=cfg.block, max_ctx=max_ctx)
+        drafter.hdf_ctx_append(y_new, cu_new, c_two, block=cfg.block)
+        h_two = drafter.hdf_draft_block_cached(c_two, anchor, block=cfg.block, max_ctx=max_ctx)
+        torch.cuda.synchronize()
+        assert hdf.device_status() == 0
+        assert torch.equal(c_round.len, c_two.len)
+        assert torch.equal(h_round.view(bits), h_two.view(bits)), f"round {r}: round / two calls differ"
+        for i, T in enumerate(done):
+            assert torch.equal(c_round.k[:, i, :T].view(bits), c_two.k[:, i, :T].view(bits))
+            assert torch.equal(c_round.v[:, i, :T].view(bits), c_two.v[:, i, :T].view(bits))
+    assert c_round.len.cpu().tolist() == list(lens)
+    assert torch.equal(h_round.view(bits), h_cold.view(bits))
+
+
+def test_round_equals_two_calls_decode_widths():
+    _check_round_equals_two_calls(W.CONFIGS["decode"], 2010, [2048], n_rounds=5)
+
+
+def test_round_equals_two_calls_ragged_two_layers():
+    cfg = W.DraftConfig("ragged", m=4, d=512, block=16, n_layers=2, n_heads=4, head_dim=128, ffn=1024,
+                        vocab=4096, batch=5, ctx_len=300)
+    _check_round_equals_two_calls(cfg, 2011, [0, 1, 63, 65, 300], n_rounds=4, pad_rows=9)
+
+
+def test_round_equals_two_calls_tiny_fp32():
+    _check_round_equals_two_calls(W.CONFIGS["tiny"], 2012, [64], n_rounds=4)
+
+
+def test_round_in_cuda_graph():
+    """One captured round (fixed row bound, device-side counts: the fork and
+    join of the block path are captured too) replayed round after round
+    gives the cold result."""
+    cfg_base = W.DraftConfig("graph", m=4, d=512, block=16, n_layers=2, n_heads=4, head_dim=128, ffn=1024,
+                             vocab=4096, batch=4, ctx_len=160)
+    lens = [160, 99, 3, 128]
+    cfg, inp, drafter, wc, cu, max_ctx = _setup(cfg_base, 2013, lens)
+    y, h_cold = _cold(drafter, cfg, inp, max_ctx)
+    cache = _nan_cache(drafter, cfg.batch, max_ctx + 7)
+    pieces = _rounds(lens, 5, np.random.default_rng(2013))
+    bound = int(pieces.sum(axis=1).max()) + 3
+    y_new = torch.zeros((bound, cfg.d), dtype=y.dtype, device="cuda")
+    cu_new = torch.zeros(cfg.batch + 1, dtype=torch.int32, device="cuda")
+    anchor = inp["anchor"].cuda()
+    h = torch.empty((cfg.batch * cfg.block, cfg.d), dtype=y.dtype, device="cuda")
+    ws = torch.empty(drafter.round_workspace_size(cfg.batch, cfg.block, bound, max_ctx), dtype=torch.uint8,
+                     device="cuda")
+    s = torch.cuda.Stream()
+    # one eager round (every row skipped) on a scratch cache first, so that
+    # no first-use setup happens under capture
+    scratch = drafter.new_cache(cfg.batch, max_ctx + 7, "cuda", zero=True)
+    drafter.hdf_draft_round(y_new, cu_new, scratch, anchor, block=cfg.block, max_ctx=max_ctx, h_out=h, ws=ws)
+    torch.cuda.synchronize()
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g, stream=s):
+        drafter.hdf_draft_round(y_new, cu_new, cache, anchor, block=cfg.block, max_ctx=max_ctx, h_out=h, ws=ws,
+                                stream=s)
+    cache.len.zero_()  # capture does not run the work
+    done = np.zeros(cfg.batch, dtype=np.int64)
+    for r in range(pieces.shape[0]):
+        idx = [cu[i] + done[i] + j for i in range(cfg.batch) for j in range(pieces[r, i])]
+        done += pieces[r]
+        y_new.zero_()
+        if idx:
+            y_new[:len(idx)] = y[torch.tensor(idx, device="cuda")]
+        cu_new.copy_(torch.tensor(np.concatenate([[0], np.cumsum(pieces[r])]).astype(np.int32)))
+        torch.cuda.synchronize()
+        with torch.cuda.stream(s):
+            g.replay()
+        s.synchronize()
+    assert hdf.device_status() == 0
+    assert cache.len.cpu().tolist() == lens
+    assert torch.equal(h.view(torch.int16), h_cold.view(torch.int16))
