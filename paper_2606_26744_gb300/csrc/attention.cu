@@ -435,14 +435,8 @@ constexpr size_t attn_smem() { return (size_t)NSTAGE * 2 * (HD / 64) * KT * 128 
 template <int HD>
 cudaError_t launch_hd(const AttnArgs& a, const AttnTmaps* tm, cudaStream_t s) {
   auto k = attn_bf16_kernel<HD>;
-  static bool attr_set = false;
   cudaError_t e;
-  if (!attr_set) {
-    if ((e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)attn_smem<HD>())) !=
-        cudaSuccess)
-      return e;
-    attr_set = true;
-  }
+  if ((e = ensure_smem_limit((const void*)k, attn_smem<HD>())) != cudaSuccess) return e;
   if (a.n_chunks < 1 || a.n_chunks > 8) return cudaErrorInvalidValue;
   // the chunks of one (sequence, head) are one cluster
   return launch_kernel(k, dim3(a.n_chunks, a.n_heads, a.batch), dim3(160), attn_smem<HD>(), s,
@@ -453,36 +447,19 @@ cudaError_t launch_hd(const AttnArgs& a, const AttnTmaps* tm, cudaStream_t s) {
 
 size_t attention_smem_bytes(int head_dim) { return head_dim == 64 ? attn_smem<64>() : attn_smem<128>(); }
 
-// Clusters of `cluster` attention CTAs resident at once (occupancy API), or
-// -1 if it cannot be asked (or answers none).  Cached per head_dim and
-// cluster size (0: not asked yet).
+// Clusters of `cluster` attention CTAs resident at once on the current device
+// (occupancy API), or -1 if it cannot be asked (or answers none).
 int attention_max_clusters(int head_dim, int cluster) {
   if ((head_dim != 64 && head_dim != 128) || cluster < 1 || cluster > 8) return -1;
-  static std::atomic<int> cache[2][9];
-  const int hi = head_dim == 128;
-  const int v = cache[hi][cluster].load();
-  if (v != 0) return v;
-  auto k = hi ? attn_bf16_kernel<128> : attn_bf16_kernel<64>;
+  const bool hi = head_dim == 128;
+  const void* k = hi ? (const void*)attn_bf16_kernel<128> : (const void*)attn_bf16_kernel<64>;
   const size_t smem = hi ? attn_smem<128>() : attn_smem<64>();
-  int n = -1;
-  if (cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) == cudaSuccess) {
-    cudaLaunchConfig_t cfg = {};
-    cudaLaunchAttribute attr;
-    attr.id = cudaLaunchAttributeClusterDimension;
-    attr.val.clusterDim.x = (unsigned)cluster;
-    attr.val.clusterDim.y = 1;
-    attr.val.clusterDim.z = 1;
-    cfg.gridDim = dim3((unsigned)cluster * 64);
-    cfg.blockDim = dim3(160);
-    cfg.dynamicSmemBytes = smem;
-    cfg.attrs = &attr;
-    cfg.numAttrs = 1;
-    if (cudaOccupancyMaxActiveClusters(&n, k, &cfg) != cudaSuccess) n = -1;
+  int n = 0;
+  if (ensure_smem_limit(k, smem) != cudaSuccess || max_active_clusters(k, 160, smem, cluster, &n) != cudaSuccess) {
+    cudaGetLastError();
+    return -1;
   }
-  cudaGetLastError();
-  if (n <= 0) n = -1;  // unknown or none: the caller falls back to SMs / cluster size
-  cache[hi][cluster].store(n);
-  return n;
+  return n > 0 ? n : -1;  // none: the caller falls back to SMs / cluster size
 }
 
 cudaError_t launch_attention(const AttnArgs& a, const AttnTmaps* tm, int dtype, cudaStream_t s) {

@@ -956,11 +956,7 @@ __global__ void __launch_bounds__(128, 1) gemm_pair_kernel(const __grid_constant
   }
 }
 
-cudaError_t prepare_pair() {
-  static cudaError_t state =
-      cudaFuncSetAttribute(gemm_pair_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, kPairSmem);
-  return state;
-}
+cudaError_t prepare_pair() { return ensure_smem_limit((const void*)gemm_pair_kernel, kPairSmem); }
 
 cudaError_t launch_pair(const GemmArgs& g, cudaStream_t s) {
   cudaError_t e;
@@ -970,17 +966,11 @@ cudaError_t launch_pair(const GemmArgs& g, cudaStream_t s) {
   return launch_kernel(gemm_pair_kernel, dim3((unsigned)(2 * tiles)), dim3(128), (size_t)kPairSmem, s, 2u, g);
 }
 
-// Function attributes of one instantiation, set once per process: the
+// Function attributes of one instantiation on the current device: the
 // dynamic shared memory and clusters of up to 16 CTAs.
 template <typename T, int BN>
 cudaError_t prepare_bn() {
-  static cudaError_t state = [] {
-    auto k = gemm_kernel<T, BN>;
-    cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, smem_for(BN));
-    if (e == cudaSuccess) e = cudaFuncSetAttribute(k, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
-    return e;
-  }();
-  return state;
+  return ensure_smem_limit((const void*)gemm_kernel<T, BN>, (size_t)smem_for(BN), true);
 }
 
 template <typename T, int BN>
@@ -998,20 +988,10 @@ cudaError_t launch_bn(const GemmArgs& g, cudaStream_t s) {
 // (the occupancy API packs clusters into GPCs); -1 if it cannot be asked.
 template <typename T, int BN>
 int resident_ctas_bn(int cluster) {
-  if (prepare_bn<T, BN>() != cudaSuccess) return -1;
-  cudaLaunchConfig_t cfg = {};
-  cudaLaunchAttribute attr;
-  attr.id = cudaLaunchAttributeClusterDimension;
-  attr.val.clusterDim.x = (unsigned)cluster;
-  attr.val.clusterDim.y = 1;
-  attr.val.clusterDim.z = 1;
-  cfg.gridDim = dim3((unsigned)cluster * 64u);
-  cfg.blockDim = dim3(128);
-  cfg.dynamicSmemBytes = (size_t)smem_for(BN);
-  cfg.attrs = &attr;
-  cfg.numAttrs = 1;
   int n = 0;
-  if (cudaOccupancyMaxActiveClusters(&n, gemm_kernel<T, BN>, &cfg) != cudaSuccess || n <= 0) {
+  if (prepare_bn<T, BN>() != cudaSuccess ||
+      max_active_clusters((const void*)gemm_kernel<T, BN>, 128, (size_t)smem_for(BN), cluster, &n) != cudaSuccess ||
+      n <= 0) {
     cudaGetLastError();
     return -1;
   }
@@ -1052,14 +1032,8 @@ int gemm_resident_ctas(int dtype, int bn, int cluster) {
   if (cluster < 1 || cluster > 16) return -1;
   const int bi = bn == 16 ? 0 : bn == 32 ? 1 : bn == 64 ? 2 : bn == 128 ? 3 : bn == 256 ? 4 : bn == 224 ? 5 : -1;
   if (bi < 0) return -1;
-  static std::atomic<int> cache[2][6][17];  // 0: not asked yet
-  std::atomic<int>& c = cache[dtype == HDF_BF16 ? 0 : 1][bi][cluster];
-  int v = c.load(std::memory_order_relaxed);
-  if (v == 0) {
-    v = dtype == HDF_BF16 ? resident_ctas_t<__nv_bfloat16>(bn, cluster) : resident_ctas_t<float>(bn, cluster);
-    c.store(v, std::memory_order_relaxed);
-  }
-  return v;
+  // the occupancy answer is cached per device by max_active_clusters
+  return dtype == HDF_BF16 ? resident_ctas_t<__nv_bfloat16>(bn, cluster) : resident_ctas_t<float>(bn, cluster);
 }
 size_t gemm_smem_bytes(int, int bn) { return (size_t)smem_for(bn); }
 

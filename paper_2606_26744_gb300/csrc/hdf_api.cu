@@ -11,14 +11,86 @@
 #include <cstdio>
 #include <cstring>
 #include <atomic>
+#include <map>
 #include <mutex>
 #include <string>
+#include <tuple>
+#include <utility>
 #include <vector>
 
 #include "common.cuh"
 #include "kernels.h"
 
 using namespace hdf;
+
+// --------------------------------------------- per-device kernel set-up
+namespace hdf {
+namespace {
+std::mutex g_setup_mu;  // guards the two tables below
+// (device, kernel) -> dynamic shared-memory limit set on that device
+std::map<std::pair<int, const void*>, size_t>& smem_limits() {
+  static std::map<std::pair<int, const void*>, size_t> m;
+  return m;
+}
+// (device, kernel, block, shared memory, cluster size) -> resident clusters
+std::map<std::tuple<int, const void*, int, size_t, int>, int>& cluster_answers() {
+  static std::map<std::tuple<int, const void*, int, size_t, int>, int> m;
+  return m;
+}
+}  // namespace
+
+cudaError_t ensure_smem_limit(const void* kernel, size_t smem, bool nonportable_clusters) {
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  std::lock_guard<std::mutex> lock(g_setup_mu);
+  auto& m = smem_limits();
+  const auto key = std::make_pair(dev, kernel);
+  const auto it = m.find(key);
+  if (it != m.end() && it->second >= smem) return cudaSuccess;
+  const size_t want = it == m.end() ? smem : std::max(smem, it->second);
+  if ((e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)want)) != cudaSuccess)
+    return e;
+  if (it == m.end() && nonportable_clusters &&
+      (e = cudaFuncSetAttribute(kernel, cudaFuncAttributeNonPortableClusterSizeAllowed, 1)) != cudaSuccess)
+    return e;
+  m[key] = want;
+  return cudaSuccess;
+}
+
+cudaError_t max_active_clusters(const void* kernel, int block, size_t smem, int cluster, int* n) {
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  std::lock_guard<std::mutex> lock(g_setup_mu);
+  auto& m = cluster_answers();
+  const auto key = std::make_tuple(dev, kernel, block, smem, cluster);
+  const auto it = m.find(key);
+  if (it != m.end()) {
+    *n = it->second;
+    return cudaSuccess;
+  }
+  cudaLaunchConfig_t cfg = {};
+  cudaLaunchAttribute attr;
+  attr.id = cudaLaunchAttributeClusterDimension;
+  attr.val.clusterDim.x = (unsigned)cluster;
+  attr.val.clusterDim.y = 1;
+  attr.val.clusterDim.z = 1;
+  cfg.gridDim = dim3((unsigned)cluster);
+  cfg.blockDim = dim3((unsigned)block);
+  cfg.dynamicSmemBytes = smem;
+  cfg.attrs = &attr;
+  cfg.numAttrs = 1;
+  int v = 0;
+  if ((e = cudaOccupancyMaxActiveClusters(&v, kernel, &cfg)) != cudaSuccess) {
+    cudaGetLastError();
+    return e;
+  }
+  m[key] = v;
+  *n = v;
+  return cudaSuccess;
+}
+}  // namespace hdf
 
 namespace {
 
@@ -79,15 +151,17 @@ int num_sms() {
 }
 
 PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
-  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
-  if (!fn) {
+  // looked up once per process (the driver entry point is the same for every
+  // device); the initialisation of a function-local static is thread-safe
+  static const PFN_cuTensorMapEncodeTiled_v12000 fn = [] {
     void* p = nullptr;
     cudaDriverEntryPointQueryResult q;
     if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) ==
             cudaSuccess &&
         q == cudaDriverEntryPointSuccess)
-      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
-  }
+      return reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
+    return static_cast<PFN_cuTensorMapEncodeTiled_v12000>(nullptr);
+  }();
   return fn;
 }
 

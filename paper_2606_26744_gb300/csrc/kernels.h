@@ -47,6 +47,17 @@ cudaError_t launch_kernel(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_
   return cudaLaunchKernelEx(&cfg, kernel, static_cast<KArgs>(args)...);
 }
 
+// Per-device kernel set-up, safe from concurrent host threads.  A process may
+// drive several GPUs and call the library from several threads: a kernel's
+// dynamic shared-memory limit is set on each device before its first launch
+// there (raised if a later launch needs more), and occupancy answers are kept
+// per device.  Both live in hdf_api.cu behind one lock.
+cudaError_t ensure_smem_limit(const void* kernel, size_t smem, bool nonportable_clusters = false);
+// Clusters of `cluster` CTAs (`block` threads, `smem` dynamic bytes each) that
+// can be resident at once on the current device; 0 when none fit.  The
+// caller sets the kernel's shared-memory limit first.
+cudaError_t max_active_clusters(const void* kernel, int block, size_t smem, int cluster, int* n);
+
 // ------------------------------------------------------------ reducer ----
 struct ReduceArgs {
   const void* H;

@@ -208,9 +208,7 @@ cudaError_t launch_m(const ReduceArgs& a, cudaStream_t s) {
   const long long ngroups = (a.n_tokens + G - 1) / G;
   auto go = [&](auto k, size_t smem) -> cudaError_t {
     cudaError_t e2;
-    if (smem > 48 * 1024 &&
-        (e2 = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem)) != cudaSuccess)
-      return e2;
+    if (smem > 48 * 1024 && (e2 = ensure_smem_limit((const void*)k, smem)) != cudaSuccess) return e2;
     if ((e2 = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, k, nt, smem)) != cudaSuccess) return e2;
     if (per_sm < 1) per_sm = 1;
     const long long grid = std::min<long long>(ngroups, (long long)per_sm * sms);
@@ -751,30 +749,10 @@ cudaError_t launch_cluster_mr(const ReduceArgs& a, const RedGeo& geo, size_t sme
                               cudaStream_t s) {
   auto k = gated_reduce_cluster_kernel<M, RB>;
   cudaError_t e;
-  // attribute and cluster occupancy depend only on the shared-memory size
-  static size_t cached_smem = 0;
-  static int cached_clusters = 0;
-  cudaLaunchConfig_t cfg = {};
-  cudaLaunchAttribute attr[1];
-  attr[0].id = cudaLaunchAttributeClusterDimension;
-  attr[0].val.clusterDim.x = RC;
-  attr[0].val.clusterDim.y = 1;
-  attr[0].val.clusterDim.z = 1;
-  cfg.blockDim = dim3(NTHR);
-  cfg.dynamicSmemBytes = smem;
-  cfg.stream = s;
-  cfg.attrs = attr;
-  cfg.numAttrs = 1;
-  cfg.gridDim = dim3(RC);
-  int max_clusters = cached_smem == smem ? cached_clusters : 0;
-  if (!max_clusters) {
-    if ((e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem)) != cudaSuccess)
-      return e;
-    if ((e = cudaOccupancyMaxActiveClusters(&max_clusters, k, &cfg)) != cudaSuccess) return e;
-    if (max_clusters < 1) return cudaErrorInvalidConfiguration;
-    cached_smem = smem;
-    cached_clusters = max_clusters;
-  }
+  int max_clusters = 0;
+  if ((e = ensure_smem_limit((const void*)k, smem)) != cudaSuccess) return e;
+  if ((e = max_active_clusters((const void*)k, NTHR, smem, RC, &max_clusters)) != cudaSuccess) return e;
+  if (max_clusters < 1) return cudaErrorInvalidConfiguration;
   const long long ncl = std::min<long long>(max_clusters, geo.nbatch);
   return launch_kernel(k, dim3((unsigned)(ncl * RC)), dim3(NTHR), smem, s, (unsigned)RC, a, geo, *hmap);
 }
@@ -1233,30 +1211,11 @@ template <int M, int S, int T, int C>
 cudaError_t launch_tile_mst(const ReduceArgs& a, const TileGeo& geo, size_t smem, const TileMaps* maps,
                             cudaStream_t s) {
   auto k = gated_reduce_tile_kernel<M, S, T, C>;
-  static size_t cached_smem = 0;
-  static int cached_clusters = 0;
   cudaError_t e;
-  int max_clusters = cached_smem == smem ? cached_clusters : 0;
-  if (!max_clusters) {
-    if ((e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem)) != cudaSuccess)
-      return e;
-    cudaLaunchConfig_t cfg = {};
-    cudaLaunchAttribute attr[1];
-    attr[0].id = cudaLaunchAttributeClusterDimension;
-    attr[0].val.clusterDim.x = S;
-    attr[0].val.clusterDim.y = 1;
-    attr[0].val.clusterDim.z = 1;
-    cfg.gridDim = dim3(S);
-    cfg.blockDim = dim3(TP_THR);
-    cfg.dynamicSmemBytes = smem;
-    cfg.stream = s;
-    cfg.attrs = attr;
-    cfg.numAttrs = 1;
-    if ((e = cudaOccupancyMaxActiveClusters(&max_clusters, k, &cfg)) != cudaSuccess) return e;
-    if (max_clusters < 1) return cudaErrorInvalidConfiguration;
-    cached_smem = smem;
-    cached_clusters = max_clusters;
-  }
+  int max_clusters = 0;
+  if ((e = ensure_smem_limit((const void*)k, smem)) != cudaSuccess) return e;
+  if ((e = max_active_clusters((const void*)k, TP_THR, smem, S, &max_clusters)) != cudaSuccess) return e;
+  if (max_clusters < 1) return cudaErrorInvalidConfiguration;
   const long long ncl = std::min<long long>(max_clusters, geo.ntiles);
   return launch_kernel(k, dim3((unsigned)(ncl * S)), dim3(TP_THR), smem, s, (unsigned)S, a, *maps, geo);
 }

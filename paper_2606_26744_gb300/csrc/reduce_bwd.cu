@@ -246,9 +246,7 @@ cudaError_t launch_m(const ReduceBwdArgs& a, const ReduceBwdPlan& p, cudaStream_
   cudaError_t e = launch_kernel(reduce_bwd_gate_kernel<T, M>, dim3((unsigned)p.gate_ctas), dim3(RB_THREADS), 0, s,
                                 1u, a);
   if (e != cudaSuccess) return e;
-  static cudaError_t attr = cudaFuncSetAttribute(reduce_bwd_wgrad_kernel<T, M>,
-                                                 cudaFuncAttributeMaxDynamicSharedMemorySize, (int)wg_smem(M));
-  if (attr != cudaSuccess) return attr;
+  if ((e = ensure_smem_limit((const void*)reduce_bwd_wgrad_kernel<T, M>, wg_smem(M))) != cudaSuccess) return e;
   e = launch_kernel(reduce_bwd_wgrad_kernel<T, M>, dim3((unsigned)p.slices, (unsigned)p.splits), dim3(RB_THREADS),
                     wg_smem(M), s, 1u, a, p.tok_per);
   if (e != cudaSuccess) return e;
