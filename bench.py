@@ -680,8 +680,9 @@ NCU_DRAM_BYTES_PER_CTX_ROW = {
 
 # DRAM bytes (read + write) per token of the tile reducer at m = 4, d = 7168,
 # from the ncu capture summarised in profiles/gated_reduce_sweep.md (16,384
-# tokens; traffic grows with the tokens)
-NCU_DRAM_BYTES_PER_TOKEN_SWEEP = (946523392 + 203869696) / 16384
+# tokens; traffic grows with the tokens); None while the kernel has changed
+# since the capture
+NCU_DRAM_BYTES_PER_TOKEN_SWEEP = None
 
 
 def tensor_peak(pk, step_ms):

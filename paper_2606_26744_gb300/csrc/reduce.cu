@@ -859,6 +859,14 @@ __device__ __forceinline__ void st_async_v4(uint32_t addr, float4 v, uint32_t ba
                : "memory");
 }
 
+// contiguous global -> shared copy completing on an mbarrier (16-byte aligned
+// addresses, size a multiple of 16)
+__device__ __forceinline__ void bulk_load(uint32_t dst, const void* src, uint32_t bytes, uint32_t bar) {
+  asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(dst),
+               "l"(src), "r"(bytes), "r"(bar)
+               : "memory");
+}
+
 // one tile's partials from all senders
 constexpr int tp_xbytes(int S, int T) { return S * T * TP_PS * 4; }
 constexpr size_t tp_smem(int S, int T, int m, int wrow) {
@@ -892,6 +900,7 @@ __global__ void __launch_bounds__(TP_THR, 1) gated_reduce_tile_kernel(const Redu
   __shared__ __align__(8) uint64_t xdone[TP_NX];
   __shared__ __align__(8) uint64_t alpha_ready[TP_NAB];
   __shared__ __align__(8) uint64_t alpha_free[TP_NAB];
+  __shared__ __align__(8) uint64_t wf_bar;
   __shared__ float bias_s[4];
   __shared__ volatile int abort_flag;
 
@@ -902,18 +911,19 @@ __global__ void __launch_bounds__(TP_THR, 1) gated_reduce_tile_kernel(const Redu
   const int d = a.d, ec = geo.ec, ngrp = geo.ngrp, NB = M * ngrp;  // boxes per tile
   const long long nl = geo.ntiles > (long long)cid ? (geo.ntiles - cid + ncl - 1) / ncl : 0;
 
-  {  // W_f slice: wsl[j][p*ec + e] = W_f[j][p*d + rank*ec + e]
-    const __nv_bfloat16* Wf = reinterpret_cast<const __nv_bfloat16*>(a.Wf);
-    const int v8 = ec / 8, per_row = M * v8;
-    for (int i = tid; i < M * per_row; i += TP_THR) {
-      const int j = i / per_row, r = i - j * per_row, pth = r / v8, e8 = r - pth * v8;
-      const uint4 v = __ldg(reinterpret_cast<const uint4*>(Wf + (size_t)j * M * d + (size_t)pth * d +
-                                                           (size_t)rank * ec + e8 * 8));
-      *reinterpret_cast<uint4*>(wsl + (size_t)j * geo.wrow + pth * ec + e8 * 8) = v;
-    }
-  }
   if (tid < M) bias_s[tid] = a.b[tid];
   if (tid == 0) {
+    // W_f slice, wsl[j][p*ec + e] = W_f[j][p*d + rank*ec + e]: one bulk copy
+    // per (gate, path) run of ec elements, in flight beside the first boxes
+    // of H (the gate warps wait for it once); W_f belongs to no earlier kernel
+    mbar_init(smem_u32(&wf_bar), 1);
+    fence_mbar_init();
+    mbar_arrive_expect_tx(smem_u32(&wf_bar), (uint32_t)(M * M * ec * 2));
+    const __nv_bfloat16* Wf = reinterpret_cast<const __nv_bfloat16*>(a.Wf);
+    for (int j = 0; j < M; ++j)
+      for (int pth = 0; pth < M; ++pth)
+        bulk_load(smem_u32(wsl + (size_t)j * geo.wrow + pth * ec),
+                  Wf + (size_t)j * M * d + (size_t)pth * d + (size_t)rank * ec, (uint32_t)(ec * 2), smem_u32(&wf_bar));
     for (int i = 0; i < NST; ++i) {
       mbar_init(smem_u32(&full_bar[i]), 1);
       mbar_init(smem_u32(&empty_bar[i]), 2);  // the two gate warps of the box's phase
@@ -982,14 +992,17 @@ __global__ void __launch_bounds__(TP_THR, 1) gated_reduce_tile_kernel(const Redu
     const int g8 = lane >> 2, q = lane & 3;
     const __nv_bfloat16* wrowp = wsl + (size_t)(g8 < M ? g8 : 0) * geo.wrow + 2 * q;
     const int row = (T == 32 ? sub * 16 : 0) + (lane & 15), hsel = lane >> 4;
+    // a failed W_f wait joins the first tile's decision below, so every gate
+    // warp still meets the others at the named barrier
+    const bool wf_ok = warp_wait(smem_u32(&wf_bar), 0u, false);
     for (long long i = 0; i < nl; ++i) {
       float acc[2][4] = {{0.f, 0.f, 0.f, 0.f}, {0.f, 0.f, 0.f, 0.f}};  // two chains: plane parity
       // sums of squares as the diagonals of A A^T on the tensor cores: the B
       // fragment of A^T for tokens 0-7 is this thread's A registers 0 and 2,
       // for tokens 8-15 its registers 1 and 3
       float dl[4] = {0.f, 0.f, 0.f, 0.f}, dh[4] = {0.f, 0.f, 0.f, 0.f};
-      bool ok = true;
-      for (int j = hb; j < NB; j += TP_NPH) {
+      bool ok = wf_ok;
+      for (int j = hb; j < NB && ok; j += TP_NPH) {
         const long long gs = i * NB + j;  // stage counter
         const int s = (int)(gs % NST);
         if (!warp_wait(smem_u32(&full_bar[s]), (uint32_t)((gs / NST) & 1), false)) {
@@ -1203,6 +1216,9 @@ __global__ void __launch_bounds__(TP_THR, 1) gated_reduce_tile_kernel(const Redu
       arrive(&alpha_free[ab]);
     }
   }
+  // the W_f copies have landed before the CTA exits, also when the gate
+  // warps gave up first
+  if (tid == 0) mbar_wait(smem_u32(&wf_bar), 0u, nullptr);
   __syncthreads();
   cluster_sync_all();  // no rank still writes into this CTA's shared memory
 }
