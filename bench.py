@@ -682,7 +682,7 @@ NCU_DRAM_BYTES_PER_CTX_ROW = {
 # from the ncu capture summarised in profiles/gated_reduce_sweep.md (16,384
 # tokens; traffic grows with the tokens); None while the kernel has changed
 # since the capture
-NCU_DRAM_BYTES_PER_TOKEN_SWEEP = None
+NCU_DRAM_BYTES_PER_TOKEN_SWEEP = (950845440 + 204011520) / 16384
 
 
 def tensor_peak(pk, step_ms):
