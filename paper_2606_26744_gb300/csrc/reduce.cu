@@ -915,7 +915,10 @@ __global__ void __launch_bounds__(TP_THR, 1) gated_reduce_tile_kernel(const Redu
   if (tid == 0) {
     // W_f slice, wsl[j][p*ec + e] = W_f[j][p*d + rank*ec + e]: one bulk copy
     // per (gate, path) run of ec elements, in flight beside the first boxes
-    // of H (the gate warps wait for it once); W_f belongs to no earlier kernel
+    // of H (the gate warps wait for it once).  It is read before the wait on
+    // the previous kernel: no kernel of this library writes W_f, and a kernel
+    // from elsewhere (a caller's optimizer step) lets this one start only
+    // when it completes, since it never triggers its dependents early.
     mbar_init(smem_u32(&wf_bar), 1);
     fence_mbar_init();
     mbar_arrive_expect_tx(smem_u32(&wf_bar), (uint32_t)(M * M * ec * 2));
