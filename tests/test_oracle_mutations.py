@@ -19,6 +19,87 @@ PINS = os.path.join(ROOT, "tests", "test_oracle_pins.py")
 
 # name -> (text in the oracle source, replacement)
 MUTATIONS = {
+    # ------------------------------------- reducer, its gradient, verification
+    "inverse RMS over the sum of squares, not the mean": (
+        "r = 1.0 / np.sqrt(np.mean(x * x, axis=1) + rms_eps)  # inverse RMS",
+        "r = 1.0 / np.sqrt(np.sum(x * x, axis=1) + rms_eps)  # inverse RMS"),
+    "inverse RMS dropped from the gate": (
+        "x_tilde = x * r[:, None]",
+        "x_tilde = x"),
+    "RMS eps outside the square root": (
+        "r = 1.0 / np.sqrt(np.mean(x * x, axis=1) + rms_eps)  # inverse RMS",
+        "r = 1.0 / (np.sqrt(np.mean(x * x, axis=1)) + rms_eps)  # inverse RMS"),
+    "gate scale applied to the bias too": (
+        "return gate_scale * (x_tilde @ np.asarray(Wf, np.float64).T) + np.asarray(b, np.float64)[None, :]",
+        "return gate_scale * (x_tilde @ np.asarray(Wf, np.float64).T + np.asarray(b, np.float64)[None, :])"),
+    "gate offset inside the sigmoid": (
+        "alpha = sigmoid(gate_logits(H, Wf, b, rms_eps, gate_scale)) + gate_offset",
+        "alpha = sigmoid(gate_logits(H, Wf, b, rms_eps, gate_scale) + gate_offset)"),
+    "gate offset dropped": (
+        "alpha = sigmoid(gate_logits(H, Wf, b, rms_eps, gate_scale)) + gate_offset",
+        "alpha = sigmoid(gate_logits(H, Wf, b, rms_eps, gate_scale))"),
+    "sigmoid of negative logits inverted": (
+        "out[~pos] = e / (1.0 + e)",
+        "out[~pos] = 1.0 / (1.0 + e)"),
+    "per-path norm RMS over the whole token": (
+        "rp = 1.0 / np.sqrt(np.mean(H * H, axis=2) + path_norm_eps)   # [N, m]",
+        "rp = (1.0 / np.sqrt(np.mean(H * H, axis=(1, 2)) + path_norm_eps))[:, None] * np.ones((1, H.shape[1]))"),
+    "per-path norm weight dropped": (
+        "Hh = H * rp[:, :, None] * np.asarray(path_norm_w, np.float64)[None, :, :]",
+        "Hh = H * rp[:, :, None]"),
+    "weighted sum normalised by the gate sum": (
+        "y = np.einsum(\"nj,njd->nd\", alpha, Hh)",
+        "y = np.einsum(\"nj,njd->nd\", alpha, Hh) / alpha.sum(axis=1, keepdims=True)"),
+    "backward: sigmoid derivative dropped": (
+        "dg = a * sg * (1.0 - sg)",
+        "dg = a"),
+    "backward: sign flipped": (
+        "dg = a * sg * (1.0 - sg)",
+        "dg = -a * sg * (1.0 - sg)"),
+    "backward: inverse RMS dropped from dW_f": (
+        "dWf = (gate_scale * r[:, None] * dg).T @ x",
+        "dWf = (gate_scale * dg).T @ x"),
+    "backward: gate scale dropped from dW_f": (
+        "dWf = (gate_scale * r[:, None] * dg).T @ x",
+        "dWf = (r[:, None] * dg).T @ x"),
+    "backward: dy paired with the paths reversed": (
+        "a = np.einsum(\"nd,njd->nj\", dy, H)",
+        "a = np.einsum(\"nd,njd->nj\", dy, H[:, ::-1])"),
+    "rope frequency exponent without the factor 2": (
+        "inv_freq = theta ** (-2.0 * i / hd)",
+        "inv_freq = theta ** (-1.0 * i / hd)"),
+    "rope rotation direction reversed": (
+        "out[..., 0::2] = x0 * c - x1 * s\n    out[..., 1::2] = x0 * s + x1 * c",
+        "out[..., 0::2] = x0 * c + x1 * s\n    out[..., 1::2] = -x0 * s + x1 * c"),
+    "rope pairs rotate-half instead of interleaved": (
+        "    x0 = x[..., 0::2]\n    x1 = x[..., 1::2]\n    out = np.empty_like(x)\n"
+        "    out[..., 0::2] = x0 * c - x1 * s\n    out[..., 1::2] = x0 * s + x1 * c",
+        "    x0 = x[..., : hd // 2]\n    x1 = x[..., hd // 2:]\n    out = np.empty_like(x)\n"
+        "    out[..., : hd // 2] = x0 * c - x1 * s\n    out[..., hd // 2:] = x0 * s + x1 * c"),
+    "attention softmax normalised over the queries": (
+        "p = p / p.sum(axis=1, keepdims=True)",
+        "p = p / p.sum(axis=0, keepdims=True)"),
+    "log-softmax without the log-sum-exp": (
+        "ls = s - lse",
+        "ls = s - smax"),
+    "accept length counts the first mismatch": (
+        "        out[i] = n\n    return out",
+        "        out[i] = min(n + 1, draft.shape[1])\n    return out"),
+    "accept length compares with the next target slot": (
+        "while n < draft.shape[1] and draft[i, n] == target[i, n]:",
+        "while n < draft.shape[1] and draft[i, n] == target[i, min(n + 1, draft.shape[1] - 1)]:"),
+    "T=1 acceptance test inverted": (
+        "if float(u[i, n]) / 2.0 ** 32 < float(ratio):",
+        "if float(u[i, n]) / 2.0 ** 32 > float(ratio):"),
+    "T=1 rejection resamples from p, not max(0, p - q)": (
+        "res = np.maximum(p_target[i, n] - q_draft[i, n], np.float32(0))      # fp32 subtraction",
+        "res = p_target[i, n]      # fp32 subtraction"),
+    "T=1 bonus token drawn at the last draft slot": (
+        "v = draw(p_target[i, nd], r[i])",
+        "v = draw(p_target[i, nd - 1], r[i])"),
+    "tau without the bonus token": (
+        "return float(np.mean(np.asarray(accept, np.float64) + 1.0))",
+        "return float(np.mean(np.asarray(accept, np.float64)))"),
     # ---------------------------------------------------------- drafter block
     "swiglu gate and up projections swapped": (
         'act = store(silu(x2 @ _f64(lw["wg"]).T) * (x2 @ _f64(lw["wu"]).T), A)',

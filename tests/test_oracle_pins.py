@@ -479,6 +479,24 @@ def test_accept_sample_special_cases():
     assert acc[0] == 2                                           # an id outside the vocabulary is rejected
 
 
+def test_accept_sample_bonus_token_comes_from_the_slot_after_the_drafts():
+    # Every draft accepted (q == p, so the ratio is 1 and any u < 2^32 passes):
+    # the emitted token is drawn from p at slot n_draft, the position after the
+    # block.  The draft slots put all their mass on token 1, so a draw from any
+    # of them would show.  With r = 2^32 - 1 the inverse CDF picks the last
+    # token with weight.
+    V, nd = 6, 3
+    p = np.zeros((2, nd + 1, V), np.float32)
+    p[:, :nd, 1] = 1.0
+    p[0, nd, 4] = 1.0
+    p[1, nd, 2] = 0.5
+    p[1, nd, 5] = 0.5
+    u = np.zeros((2, nd), np.uint64)
+    acc, nxt = O.accept_sample(p, p[:, :nd], np.full((2, nd), 1), u, np.array([0, 2 ** 32 - 1], np.uint64))
+    assert list(acc) == [nd, nd]
+    assert nxt[0] == 4 and nxt[1] == 5
+
+
 def test_accept_sample_inverse_cdf_boundaries():
     # uniform residual over 4 tokens: weights 2^38 each, R = 2^40, threshold = r * 2^8
     p = np.zeros((1, 2, 4), np.float32); p[0, 0] = 0.25
