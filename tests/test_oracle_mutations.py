@@ -100,6 +100,52 @@ MUTATIONS = {
     "tau without the bonus token": (
         "return float(np.mean(np.asarray(accept, np.float64) + 1.0))",
         "return float(np.mean(np.asarray(accept, np.float64)))"),
+    # ----------------------------------------- storage rounding and helpers
+    "bf16 rounding half away from zero": (
+        "q = np.rint(mant * 256.0) / 256.0        # np.rint: round half to even",
+        "q = np.sign(mant) * np.floor(np.abs(mant) * 256.0 + 0.5) / 256.0        # np.rint: round half to even"),
+    "bf16 rounding by truncation": (
+        "q = np.rint(mant * 256.0) / 256.0        # np.rint: round half to even",
+        "q = np.trunc(mant * 256.0) / 256.0        # np.rint: round half to even"),
+    "bf16 keeps 9 significant bits": (
+        "q = np.rint(mant * 256.0) / 256.0        # np.rint: round half to even",
+        "q = np.rint(mant * 512.0) / 512.0        # np.rint: round half to even"),
+    "drafter RMSNorm eps outside the square root": (
+        "r = 1.0 / np.sqrt(np.mean(x * x, axis=-1, keepdims=True) + eps)",
+        "r = 1.0 / (np.sqrt(np.mean(x * x, axis=-1, keepdims=True)) + eps)"),
+    "drafter RMSNorm over the sum of squares": (
+        "r = 1.0 / np.sqrt(np.mean(x * x, axis=-1, keepdims=True) + eps)",
+        "r = 1.0 / np.sqrt(np.sum(x * x, axis=-1, keepdims=True) + eps)"),
+    "silu is the sigmoid alone": (
+        "return x * sigmoid(x)",
+        "return sigmoid(x)"),
+    "KL divided by the vocabulary size": (
+        "return float(t_kd * t_kd / P * np.sum(p * (lp - lq)))",
+        "return float(t_kd * t_kd / t.shape[1] * np.sum(p * (lp - lq)))"),
+    "reducer output not rounded at its storage point": (
+        "    y = np.einsum(\"nj,njd->nd\", alpha, Hh)\n    return store(y, out_dtype), alpha",
+        "    y = np.einsum(\"nj,njd->nd\", alpha, Hh)\n    return y, alpha"),
+    "attention scale applied twice": (
+        "s = (q @ k.T) / math.sqrt(q.shape[-1])",
+        "s = (q @ k.T) / q.shape[-1]"),
+    "zmax taken from the tempered logits": (
+        "zmax = z[np.arange(z.shape[0]), tok]",
+        "zmax = z[np.arange(z.shape[0]), tok] * inv_temp"),
+    "cross-entropy sign flipped": (
+        "out[on] = -ls[np.nonzero(on)[0], labels[on]]",
+        "out[on] = ls[np.nonzero(on)[0], labels[on]]"),
+    "T=1 residual of q - p instead of p - q": (
+        "res = np.maximum(p_target[i, n] - q_draft[i, n], np.float32(0))      # fp32 subtraction",
+        "res = np.maximum(q_draft[i, n] - p_target[i, n], np.float32(0))      # fp32 subtraction"),
+    "T=1 acceptance ratio q/p": (
+        "ratio = np.float32(p_target[i, n, x]) / np.float32(q_draft[i, n, x])   # IEEE fp32 division",
+        "ratio = np.float32(q_draft[i, n, x]) / np.float32(p_target[i, n, x])   # IEEE fp32 division"),
+    "fc output not rounded at its storage point": (
+        "return store(x @ _f64(W_fc).T, out_dtype)",
+        "return x @ _f64(W_fc).T"),
+    "backward: bias gradient summed over paths": (
+        "db = dg.sum(axis=0)",
+        "db = np.full(dg.shape[1], dg.sum())"),
     # ---------------------------------------------------------- drafter block
     "swiglu gate and up projections swapped": (
         'act = store(silu(x2 @ _f64(lw["wg"]).T) * (x2 @ _f64(lw["wu"]).T), A)',

@@ -33,6 +33,30 @@ def test_bf16_round_matches_torch_conversion():
     assert np.array_equal(ref, got)
 
 
+def _bf16_nearest(y, exact):
+    """y holds bfloat16 values (each survives torch's float32 -> bfloat16 cast
+    unchanged) within half a bfloat16 ulp of the exact values."""
+    y = np.asarray(y, np.float64)
+    survives = np.array_equal(torch.from_numpy(y).float().to(torch.bfloat16).double().numpy(), y)
+    half_ulp = np.ldexp(1.0, np.frexp(np.asarray(exact, np.float64))[1] - 9)
+    return survives and bool(np.all(np.abs(y - exact) <= half_ulp))
+
+
+def test_reducer_and_fc_outputs_are_rounded_where_they_are_stored():
+    # y of Eq. 1 and the fc output are stored in bf16 (the precision contract):
+    # every value is the bf16 nearest to the exact one, and random data is
+    # not bf16-exact, so the rounding shows
+    r = np.random.default_rng(81)
+    H = r.standard_normal((6, 3, 16))
+    Wf, b = 0.1 * r.standard_normal((3, 48)), r.standard_normal(3)
+    y, _ = O.gated_reduce(H, Wf, b, out_dtype="bf16")
+    y64, _ = O.gated_reduce(H, Wf, b, out_dtype="f64")
+    assert _bf16_nearest(y, y64) and not np.array_equal(y, y64)
+    W = r.standard_normal((8, 48))
+    f, f64 = O.fc_reduce(H, W, out_dtype="bf16"), O.fc_reduce(H, W, out_dtype="f64")
+    assert _bf16_nearest(f, f64) and not np.array_equal(f, f64)
+
+
 def test_store_f32_is_float32_rounding():
     x = rng.standard_normal(1000)
     assert np.array_equal(O.store(x, "f32"), x.astype(np.float32).astype(np.float64))
@@ -216,6 +240,14 @@ def test_rmsnorm_constant_vector():
     x = np.where(rng.standard_normal(10) > 0, 4.0, -4.0)
     w = rng.standard_normal(10)
     np.testing.assert_allclose(O.rmsnorm(x, w, 0.0), np.sign(x) * w, rtol=1e-15)
+
+
+def test_rmsnorm_eps_inside_the_square_root():
+    # a constant vector c normalises to c / sqrt(c^2 + eps) * w; with eps far
+    # above c^2 that is about c / sqrt(eps), ten times c / (|c| + eps) here
+    c, eps = 1e-3, 1e-2
+    w = rng.standard_normal(6)
+    np.testing.assert_allclose(O.rmsnorm(np.full(6, c), w, eps), c / math.sqrt(c * c + eps) * w, rtol=1e-14)
 
 
 def test_rope_head_dim_two_is_plain_rotation():
