@@ -100,6 +100,51 @@ MUTATIONS = {
     "tau without the bonus token": (
         "return float(np.mean(np.asarray(accept, np.float64) + 1.0))",
         "return float(np.mean(np.asarray(accept, np.float64)))"),
+    # ------------------------------------------ drafter projections and layers
+    "context keys projected with the value weights": (
+        "K = (_f64(c) @ _f64(wk).T).reshape(n, n_heads, head_dim)",
+        "K = (_f64(c) @ _f64(wv).T).reshape(n, n_heads, head_dim)"),
+    "block keys projected with the query weights": (
+        "Kb = store(rope((x @ _f64(lw[\"wk\"]).T).reshape(M, n_heads, head_dim),",
+        "Kb = store(rope((x @ _f64(lw[\"wq\"]).T).reshape(M, n_heads, head_dim),"),
+    "block values projected with the key weights": (
+        "Vb = store(x @ _f64(lw[\"wv\"]).T, A)",
+        "Vb = store(x @ _f64(lw[\"wk\"]).T, A)"),
+    "block attention skips the block's own keys": (
+        "k_all = np.concatenate([Kc[ctx_rows, cols], Kb[rows, cols]], axis=0)\n"
+        "                v_all = np.concatenate([Vc[ctx_rows, cols], Vb[rows, cols]], axis=0)",
+        "k_all = Kc[ctx_rows, cols] if cu[i + 1] > cu[i] else Kb[rows, cols]\n"
+        "                v_all = Vc[ctx_rows, cols] if cu[i + 1] > cu[i] else Vb[rows, cols]"),
+    "block attention reads every sequence's context": (
+        "ctx_rows = slice(cu[i], cu[i + 1])",
+        "ctx_rows = slice(0, cu[-1])"),
+    "context positions continue across sequences": (
+        "pos_ctx = np.concatenate([np.arange(t) for t in lens]) if cu[-1] else np.zeros(0)",
+        "pos_ctx = np.arange(cu[-1])"),
+    "a head's output written into another head's columns": (
+        "O[rows, cols] = softmax_attention(Q[rows, cols], k_all, v_all)",
+        "O[rows, slice((n_heads - 1 - hh) * head_dim, (n_heads - hh) * head_dim)] = softmax_attention(Q[rows, cols], k_all, v_all)"),
+    "output projection transposed": (
+        "h = store(h + O @ _f64(lw[\"wo\"]).T, \"f32\")",
+        "h = store(h + O @ _f64(lw[\"wo\"]), \"f32\")"),
+    "down projection applied to the MLP input": (
+        "h = store(h + act @ _f64(lw[\"wd\"]).T, \"f32\")",
+        "h = store(h + silu(x2 @ _f64(lw[\"wg\"]).T) @ _f64(lw[\"wd\"]).T, \"f32\")"),
+    "context rows normalised with the final norm weight": (
+        "c = store(rmsnorm(ctx, W[\"ctx_norm\"], norm_eps), A)",
+        "c = store(rmsnorm(ctx, W[\"final_norm\"], norm_eps), A)"),
+    "every block slot gets the anchor embedding": (
+        "h[i * B + 1:(i + 1) * B] = _f64(W[\"mask_vec\"])[None, :]",
+        "h[i * B + 1:(i + 1) * B] = _f64(W[\"embed\"])[int(anchor[i])][None, :]"),
+    "layers share the first layer's weights": (
+        "    for lw in W[\"layers\"]:\n        rec = {}",
+        "    for lw in [W[\"layers\"][0]] * len(W[\"layers\"]):\n        rec = {}"),
+    "context K/V from the raw reducer output": (
+        "        Kc, Vc = context_kv(c, lw[\"wk\"], lw[\"wv\"], pos_ctx, n_heads=n_heads,",
+        "        Kc, Vc = context_kv(ctx, lw[\"wk\"], lw[\"wv\"], pos_ctx, n_heads=n_heads,"),
+    "draft tokens taken from slots 0..B-2": (
+        "return tok[:, 1:]",
+        "return tok[:, :-1]"),
     # ----------------------------------------- storage rounding and helpers
     "bf16 rounding half away from zero": (
         "q = np.rint(mant * 256.0) / 256.0        # np.rint: round half to even",

@@ -246,7 +246,7 @@ def test_rmsnorm_eps_inside_the_square_root():
     # a constant vector c normalises to c / sqrt(c^2 + eps) * w; with eps far
     # above c^2 that is about c / sqrt(eps), ten times c / (|c| + eps) here
     c, eps = 1e-3, 1e-2
-    w = rng.standard_normal(6)
+    w = np.random.default_rng(95).standard_normal(6)
     np.testing.assert_allclose(O.rmsnorm(np.full(6, c), w, eps), c / math.sqrt(c * c + eps) * w, rtol=1e-14)
 
 
@@ -372,6 +372,63 @@ def test_draft_block_zero_query_averages_own_sequence_context_and_block():
         v_all = np.concatenate([L0["Vc"][cu[i]:cu[i + 1]], L0["Vb"][i * B:(i + 1) * B]], axis=0)
         for k in range(B):
             np.testing.assert_allclose(L0["O"][i * B + k], v_all.mean(axis=0), rtol=1e-12)
+
+
+def test_zero_keys_attend_uniformly_with_values_from_w_v_and_output_through_w_o():
+    # W_k = 0: every score is 0, so each block row's attention output is the
+    # plain mean of the values of its own sequence's T_i context rows and B
+    # block rows.  Context rows are constant vectors a_t * 1 and the block
+    # input rows are 0.5 * 1, so at eps 0 their norms are the norm weights:
+    # every context value row is ctx_norm W_v^T and every block value row
+    # attn_norm W_v^T.  In every head, per sequence,
+    #     O = (T_i ctx_norm W_v^T + B attn_norm W_v^T) / (T_i + B),
+    # and the attention residual is h = 0.5 + O W_o^T.  Keys or values taken
+    # from another projection, heads reading another head's columns, or W_o
+    # applied untransposed each move O or h.
+    d, B, nh, hd = 16, 4, 2, 8
+    W = _tiny_weights(d=d, seed=91)
+    lw = W["layers"][0]
+    lw["wk"][:] = 0
+    W["embed"] = np.full_like(W["embed"], 0.5)
+    W["mask_vec"] = np.full_like(W["mask_vec"], 0.5)
+    cu = [0, 3, 10]
+    ctx = np.repeat(np.random.default_rng(92).uniform(0.5, 2.0, 10)[:, None], d, axis=1)
+    inter = {}
+    O.draft_block(W, ctx, cu, [1, 2], block=B, n_heads=nh, head_dim=hd, rope_theta=1e4,
+                  norm_eps=0.0, act_dtype="f64", intermediates=inter)
+    L0 = inter["layers"][0]
+    vc = W["ctx_norm"] @ lw["wv"].T
+    vb = lw["attn_norm"] @ lw["wv"].T
+    for i in range(2):
+        T = cu[i + 1] - cu[i]
+        want = (T * vc + B * vb) / (T + B)
+        for k in range(B):
+            np.testing.assert_allclose(L0["O"][i * B + k], want, rtol=1e-12, atol=1e-12)
+            np.testing.assert_allclose(L0["h_attn"][i * B + k], 0.5 + want @ lw["wo"].T, rtol=1e-6, atol=1e-6)
+
+
+def test_a_layer_with_zero_output_projections_adds_nothing():
+    # a second layer whose W_o and W_d are 0 leaves the residual stream as the
+    # first layer left it, so two layers equal the first alone, bit for bit;
+    # layers that read another layer's weights would not
+    d, B = 16, 4
+    W1 = _tiny_weights(d=d, L=1, seed=93)
+    extra = _tiny_weights(d=d, L=1, seed=94)["layers"][0]
+    extra["wo"][:] = 0
+    extra["wd"][:] = 0
+    W2 = dict(W1)
+    W2["layers"] = [W1["layers"][0], extra]
+    ctx = np.random.default_rng(96).standard_normal((9, d))
+    cu = [0, 4, 9]
+    kw = dict(block=B, n_heads=2, head_dim=8, rope_theta=1e4, norm_eps=1e-6, act_dtype="f64")
+    np.testing.assert_array_equal(O.draft_block(W2, ctx, cu, [3, 7], **kw), O.draft_block(W1, ctx, cu, [3, 7], **kw))
+
+
+def test_draft_tokens_are_block_slots_one_to_b_minus_one():
+    # slot 0 of each block is the anchor; drafts d_1 .. d_{B-1} are slots 1 .. B-1
+    B, batch = 5, 2
+    tok = np.arange(batch * B) * 10
+    np.testing.assert_array_equal(O.draft_tokens(tok, batch, B), [[10, 20, 30, 40], [60, 70, 80, 90]])
 
 
 def test_draft_block_sequences_are_independent():
