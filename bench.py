@@ -685,6 +685,13 @@ NCU_DRAM_BYTES_PER_CTX_ROW = {
 NCU_DRAM_BYTES_PER_TOKEN_SWEEP = (950845440 + 204011520) / 16384
 
 
+def workload_config(cfg, world):
+    """The workload keys of a bench line's config, the same on both arms."""
+    return {"workload": cfg.name, "m": cfg.m, "d": cfg.d, "ctx_per_seq": cfg.ctx_len, "batch_per_gpu": cfg.batch,
+            "block": cfg.block, "layers": cfg.n_layers, "heads": f"{cfg.n_heads}x{cfg.head_dim}", "ffn": cfg.ffn,
+            "vocab": cfg.vocab, "parallelism": f"replicas x{world}"}
+
+
 def tensor_peak(pk, step_ms):
     """bf16 tensor peak a kernel of the step is held against: the burst
     figure when the step is shorter than a second (each launch runs well
@@ -1107,7 +1114,8 @@ def run_reference(args):
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(wall / args.steps * 1e3, 3),
             "ms_per_block": round(spb * 1e3, 3), "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-            "config": {"workload": cfg.name, "batch": cfg.batch, "seq_len": cfg.ctx_len, "block": cfg.block},
+            "config": {**workload_config(cfg, args.gpus),
+                       "timing": "wall clock of stage-wise oracle samples on the host cores, one block each"},
             "cpu_baseline": {"value": round(val, 5), "unit": UNIT, "cores": host_cores(), "kind": "oracle",
                              "sample": sample_txt},
             "e2e": {"value": round(val, 5), "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
@@ -1190,10 +1198,7 @@ def main():
             "metric": METRIC, "value": round(val, 2), "unit": UNIT, "n_gpus": world, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": round(res["ms"], 5), "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": cfg.dtype, "data": "synthetic",
-            "config": {"workload": cfg.name, "m": cfg.m, "d": cfg.d, "ctx_per_seq": cfg.ctx_len,
-                       "batch_per_gpu": cfg.batch, "block": cfg.block, "layers": cfg.n_layers,
-                       "heads": f"{cfg.n_heads}x{cfg.head_dim}", "ffn": cfg.ffn, "vocab": cfg.vocab,
-                       "parallelism": f"replicas x{world}",
+            "config": {**workload_config(cfg, world),
                        "l2": f"no flush: one step moves {step_bytes / 1e6:.0f} MB of algorithmic traffic "
                              "(weights, residual, K/V), far above the 126 MB L2",
                        "timing": ("CUDA events on the launch stream around the K steps, " +
