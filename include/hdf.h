@@ -118,21 +118,25 @@ HDF_API int hdf_gated_reduce(const void* H, int dtype, int64_t n_tokens, int m, 
  * which fp32 summation order, another call uses).  The paper has no
  * counterpart: it is a tuning and test hook.  All kernels compute Eq. 1 and
  * agree within fp32 summation order.
- *   HDF_REDUCE_AUTO     what hdf_gated_reduce runs: the tile kernel for m = 4,
- *                       the general kernel otherwise, whatever n_tokens is,
- *                       so that a token's y does not depend on how many
- *                       tokens share the call
+ *   HDF_REDUCE_AUTO     what hdf_gated_reduce runs: the tile kernel for m = 4
+ *                       where it applies (below), the general kernel
+ *                       otherwise, whatever n_tokens is, so that a token's y
+ *                       does not depend on how many tokens share the call
  *   HDF_REDUCE_GENERAL  one CTA streams whole tokens and re-reads them from L2
  *                       for the weighted sum (every dtype and option)
  *   HDF_REDUCE_CLUSTER  8-CTA clusters split d, keep W_f slices in shared
  *                       memory and exchange the gate partials of small token
  *                       batches over distributed shared memory
- *   HDF_REDUCE_TILE     clusters split d over tiles of 32 tokens, gate dots on
- *                       the tensor cores, one exchange per tile
- * CLUSTER and TILE need bf16, m in {1,2,4}, d % 512 == 0 and neither
- * alpha_override nor path_norm_w (TILE also a whole number of its 4 box
- * phases per tile, always so for m = 4); the general kernel runs otherwise.
- * Another kernel value returns HDF_ERR_INVALID_ARG. */
+ *   HDF_REDUCE_TILE     persistent clusters of 4 (or, for wide slices, 8)
+ *                       CTAs split d over tiles of 16 or 32 tokens, gate dots
+ *                       on the tensor cores, one exchange per tile; the
+ *                       geometry depends on m and d only
+ * CLUSTER and TILE need bf16, m in {1,2,4} and neither alpha_override nor
+ * path_norm_w.  CLUSTER also needs d % 512 == 0; TILE needs d a multiple of
+ * 64 times its cluster size, a whole number of its 4 box phases per tile and
+ * a tile slice that fits its shared memory (for m = 4: every d % 256 == 0 up
+ * to 9728, and some wider).  The general kernel runs otherwise.  Another
+ * kernel value returns HDF_ERR_INVALID_ARG. */
 enum { HDF_REDUCE_AUTO = 0, HDF_REDUCE_GENERAL = 1, HDF_REDUCE_CLUSTER = 2, HDF_REDUCE_TILE = 3 };
 HDF_API int hdf_gated_reduce_kernel(int kernel, const void* H, int dtype, int64_t n_tokens, int m, int d,
                      const void* Wf, const float* b,
