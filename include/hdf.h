@@ -11,14 +11,23 @@
  * hdf_accept_sample is the temperature-1 (sampling) form of step 4, and
  * hdf_kl_distill the training-time distillation target (Eq. 2, Sec. 2.3).
  * hdf_ctx_append + hdf_draft_block_cached split step 2 for serving: the
- * context projection of each accepted token runs once, into a K/V cache.
+ * context projection of each accepted token runs once, into a K/V cache;
+ * hdf_draft_round does both in one call.  hdf_draft_loss is the training
+ * objective of Eq. 3, hdf_gated_reduce_backward the gradient of Eq. 1 with
+ * respect to W_f and b, and hdf_fc_reduce the generic fc collapse the paper
+ * compares against (and falls back to for unequal widths, Sec. 2.2).
  *
  * Conventions shared by every call
  *   - All tensor arguments are DEVICE pointers owned by the caller, row-major,
  *     16-byte aligned, densely packed unless a stride argument says otherwise.
  *     The library keeps no pointer after a call returns.
  *   - The library allocates nothing.  Scratch comes from a caller workspace
- *     (256-byte aligned) whose size the matching *_workspace_size() returns.
+ *     (256-byte aligned) whose size the matching *_workspace_size() returns
+ *     (hdf_lm_head_argmax_static uses a fixed device array of the library
+ *     instead).
+ *   - Calls may come from several host threads, and one process may drive
+ *     several GPUs: the per-device set-up the library does on first use
+ *     (kernel shared-memory limits, occupancy answers) is guarded by a lock.
  *   - Every call is asynchronous on the caller's CUDA stream (a cudaStream_t
  *     passed as hdf_stream_t; NULL = legacy default stream).  No call
  *     synchronises, and there is no host fallback: if the CUDA kernels cannot
