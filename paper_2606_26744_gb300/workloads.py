@@ -107,6 +107,8 @@ def _randn(shape, std, dtype, g, device, chunk_elems: Optional[int] = None):
     if chunk_elems is None:
         chunk_elems = 1 << 22 if torch.device(device).type == "cpu" else 1 << 27
     out = torch.empty(shape, dtype=dtype, device=device)
+    if out.numel() == 0:  # nothing to draw (e.g. a batch whose contexts are all empty)
+        return out
     flat = out.view(shape[0], -1)
     chunk_rows = max(1, chunk_elems // max(1, flat.shape[1]))
     for r0 in range(0, shape[0], chunk_rows):

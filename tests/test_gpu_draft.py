@@ -144,6 +144,29 @@ def test_batch8_block16_128_tokens():
     run_step(cfg, seed=11, ctx_lens=[200, 3, 64, 65, 130, 1, 199, 90])
 
 
+def test_block_of_two():
+    """The smallest block: the anchor and one mask slot, so each sequence drafts
+    one token and its accepted length is 0 or 1."""
+    cfg = W.DraftConfig("b2", m=4, d=512, block=2, n_layers=1, n_heads=4, head_dim=128, ffn=1024,
+                        vocab=4096, batch=4, ctx_len=300)
+    run_step(cfg, seed=15, ctx_lens=[300, 1, 64, 129])
+
+
+def test_every_context_empty():
+    """No context at all: each block attends to its own B keys only, and the
+    reducer and the context projection have no rows."""
+    cfg = W.DraftConfig("noctx", m=4, d=512, block=16, n_layers=2, n_heads=4, head_dim=128, ffn=1024,
+                        vocab=4096, batch=3, ctx_len=0)
+    run_step(cfg, seed=14, ctx_lens=[0, 0, 0])
+
+
+def test_two_paths_three_layers():
+    """m = 2 (the general reducer kernel) feeding a three-layer drafter."""
+    cfg = W.DraftConfig("m2l3", m=2, d=512, block=16, n_layers=3, n_heads=4, head_dim=128, ffn=1024,
+                        vocab=4096, batch=2, ctx_len=200)
+    run_step(cfg, seed=16, ctx_lens=[200, 77])
+
+
 def test_batch6_block16_96_tokens_fp32():
     cfg = W.DraftConfig("b6f32", m=4, d=256, block=16, n_layers=1, n_heads=2, head_dim=128, ffn=1024,
                         vocab=2048, batch=6, ctx_len=70, dtype="f32")

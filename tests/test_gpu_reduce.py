@@ -46,6 +46,9 @@ def _run(inp, **kw):
     (1000, 4, 7168, "bf16", 0.1),   # 56 k-blocks per CTA: the stage ring wraps in both passes
     (300, 4, 16384, "bf16", 0.1),   # the widest d: 16-token tiles in 8-CTA clusters
     (333, 2, 7168, "bf16", 0.1),    # m = 2 at the sweep width: 8-CTA clusters
+    (70, 4, 256, "bf16", 0.1),      # the narrowest tile width: one plane per slice
+    (50, 4, 9728, "bf16", 0.1),     # 8-CTA clusters, a three-plane tail box
+    (20, 4, 9984, "bf16", 0.1),     # no tile geometry fits: m = 4 takes the general kernel
 ])
 def test_reduce_parity(N, m, d, dtype, std, reduce_path):
     inp = W.make_reduce_inputs(N, m, d, dtype, std, seed=N * 131 + d)
