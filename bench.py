@@ -862,8 +862,8 @@ def run_kernel_only(args):
     """One kernel of the path alone, for profiling runs (not a bench line):
     3 warm-up launches, then args.steps launches timed with CUDA events.
       accept      hdf_accept_len over args.tokens blocks of 15 drafts
-      reduce_bwd  hdf_gated_reduce_backward over args.tokens tokens, m 4, d 7168
-      reduce      hdf_gated_reduce (tile kernel) over args.tokens tokens, m 4, d 7168
+      reduce_bwd  hdf_gated_reduce_backward over args.tokens tokens, m 4, d args.d
+      reduce      hdf_gated_reduce (tile kernel) over args.tokens tokens, m 4, d args.d
       loss        hdf_draft_loss over the large workload's blocks (8 x 16, P 2, V 129280)
       lmhead      hdf_lm_head_argmax at the large workload's widths: 128 tokens,
                   d 7168, V 129280, fp32 log-softmax"""
@@ -884,7 +884,7 @@ def run_kernel_only(args):
             hdf.hdf_accept_len(dr, tg, n_draft=nd, draft_stride=nd, batch=n, accept=acc)
         byt = 2 * n * nd * 4 + n * 4
     elif args.kernel_only in ("reduce_bwd", "reduce"):
-        m, d = 4, 7168
+        m, d = 4, args.d
         inp = W.make_reduce_inputs(n, m, d, "bf16", 0.1, seed=1004, device=dev)
         H, Wf, b = inp["H"], inp["Wf"], inp["b"]
         if args.kernel_only == "reduce":
@@ -1146,6 +1146,7 @@ def main():
     ap.add_argument("--kernel-only", default=None, choices=["accept", "reduce_bwd", "reduce", "loss", "lmhead"],
                     help="time one kernel alone (profiling runs; not a bench line)")
     ap.add_argument("--tokens", type=int, default=1 << 20, help="units of a --kernel-only run")
+    ap.add_argument("--d", type=int, default=7168, help="width of a --kernel-only reduce or reduce_bwd run")
     args = ap.parse_args()
     args.overrides = {k: v for k, v in (("batch", args.batch), ("vocab", args.vocab), ("n_layers", args.layers))
                       if v is not None}
