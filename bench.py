@@ -662,13 +662,16 @@ def measure_warm(cfg, inp, drafter, y, tok_cold, tgt, stream, steps, dev, pk):
 # were captured on fewer context rows and are scaled by the rows of the
 # launch: the traffic of that kernel grows in proportion to its rows).
 NCU_DRAM_BYTES = {
+    # the decode step's GEMMs and attention (profiles/ctx_kv_gemm_decode.md,
+    # block_gemms_decode.md, lm_head_gemm_decode.md, attention_decode.md)
     "decode": {
-        "L0.qkv_gemm": 25329664,
-        "L0.o_gemm": 8667136,
-        "L0.gate_up_gemm": 67264768 + 301568,
-        "L0.down_gemm": 34029312,
-        "lm_head": 134369536 + 3009280,
-        "L0.attention": 17011456,
+        "L0.ctx_kv_gemm": 26285568 + 1536,
+        "L0.qkv_gemm": 25311232,
+        "L0.o_gemm": 8667648,
+        "L0.gate_up_gemm": 67265280 + 371200,
+        "L0.down_gemm": 34030336,
+        "lm_head": 134368256 + 3628032,
+        "L0.attention": 17011200,
     },
 }
 NCU_DRAM_BYTES_PER_CTX_ROW = {
