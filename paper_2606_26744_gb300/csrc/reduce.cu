@@ -793,7 +793,9 @@ cudaError_t launch_gated_reduce_cluster(const ReduceArgs& a, const CUtensorMap* 
 // A cluster of S CTAs (S = 4, or 8 when the slices would not fit) walks
 // tiles of T = 32 (or 16, for wide slices) consecutive tokens; CTA rank c
 // owns elements [c*E, (c+1)*E) of each of the m paths (E = d/S), so its W_f
-// slice (m x m*E) stays in shared memory.  Roles, meeting only at mbarriers:
+// slice (m x m*E) stays in shared memory; it arrives by m*m bulk copies on
+// one mbarrier, in flight beside the first boxes of H.  Roles, meeting only
+// at mbarriers:
 //   producer warp   streams pass 1 of every tile from HBM into a 128 KB ring:
 //                   one TMA box per stage from the 3-D view {64 elements,
 //                   tokens, 128-byte chunks} of H, C chunks (C * 128
